@@ -1,0 +1,514 @@
+"""Plain numpy restatement of the UniQuan_F per-element quantizer.
+
+TEST INFRASTRUCTURE ONLY (see the package docstring): the product path never
+imports this module.
+
+Notation follows the paper: a weight group w (g values) is transformed by
+FlexRound's T_F (Eq. 1), mapped to the nearest of the 2^q BCQ levels
+(M_B, Sec. 2.3; or the local and periodic M*_B of Algorithm 4), reconstructed
+by R_B (C alpha + z_B) and detransformed by D_R (Delta (w~ - z_U)).  The
+bit-width is written q (the paper's k), L = 2^q.
+
+Conventions shared with the CUDA library (they are readings of points the
+paper leaves open; each one is listed with its reason in the design notes):
+
+* a code word is an integer in [0, L); bit (j-1) set  <=>  c_j = +1;
+* level of a code:  l(c) = ((c_1 a_1 + c_2 a_2) + ... + c_q a_q) + z_B,
+  fp32, summed left to right (the matrix-vector product C alpha first, then
+  the shift z_B, as R_B is written in Sec. 2.3);
+* levels are sorted ascending; equal values keep ascending code-word order;
+* full mapping M_B: argmin over ranks of |x - l|, fp32, ties -> lower rank;
+* local mapping M*_B on a remap step (step % p == 0): candidates are the
+  current rank d, then max(d-1, 0), then min(d+1, L-1); a candidate replaces
+  the best only if strictly nearer;
+* on a non-remap step the code word is kept and w~ = l(code) is recomputed
+  with the current alpha, z_B;
+* T_F: u = w / ((Delta * s) * s_r), x = u + z_U (fp32, IEEE division);
+* D_R: w^ = Delta * (w~ - z_U) (fp32);
+* gradient filter (App. C.1): tau = min_j |a_j|; the straight-through path
+  of an element is zeroed when |x - w~| > tau.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+__all__ = [
+    "MAP_FULL", "MAP_LOCAL_PERIODIC",
+    "EXPORT_REUSE_CODES", "EXPORT_REMAP_EQ4",
+    "CLIP_FIXED_MIN", "CLIP_FIXED_MAX", "CLIP_BALANCED",
+    "signs", "levels", "sorted_levels",
+    "transform_F", "map_full", "map_local", "reconstruct", "detransform",
+    "quantize_fwd", "quantize_bwd", "bwd_l1_mass",
+    "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
+    "clip_params", "greedy_init", "general_alternating", "unified_init",
+    "rtn",
+]
+
+F32 = np.float32
+F64 = np.float64
+
+MAP_FULL = 0
+MAP_LOCAL_PERIODIC = 1
+EXPORT_REUSE_CODES = 0
+EXPORT_REMAP_EQ4 = 1
+CLIP_FIXED_MIN = 0
+CLIP_FIXED_MAX = 1
+CLIP_BALANCED = 2
+
+
+# ---------------------------------------------------------------------------
+# BCQ levels (Sec. 2.3)
+# ---------------------------------------------------------------------------
+
+def signs(q: int, dtype=F32) -> np.ndarray:
+    """Binary codes of all L = 2^q code words as a [L, q] array of +-1.
+
+    Sec. 2.3: each weight carries c in {-1,+1}^q; row c of the result is the
+    code of code word c (bit j-1 set  <=>  c_j = +1).
+    """
+    words = np.arange(1 << q)[:, None]
+    bits = (words >> np.arange(q)[None, :]) & 1
+    return np.where(bits == 1, 1, -1).astype(dtype)
+
+
+def levels(alpha: np.ndarray, zb: np.ndarray) -> np.ndarray:
+    """All 2^q quantization levels l(c) = c . alpha + z_B, fp32 (Sec. 2.3).
+
+    alpha: [..., q]; zb: [...]  ->  [..., L] indexed by code word.
+    The dot product is accumulated j = 1..q left to right, then z_B added.
+    """
+    alpha = np.asarray(alpha, F32)
+    zb = np.asarray(zb, F32)
+    q = alpha.shape[-1]
+    S = signs(q)
+    acc = S[:, 0] * alpha[..., None, 0]
+    for j in range(1, q):
+        acc = acc + S[:, j] * alpha[..., None, j]
+    return acc + zb[..., None]
+
+
+def sorted_levels(lv: np.ndarray):
+    """Sort levels ascending (Algorithm 4 keeps the levels as an ordered list).
+
+    Returns (sorted values [..., L], code_of_rank [..., L], rank_of_code
+    [..., L]).  A stable sort orders equal levels by ascending code word.
+    """
+    code_of_rank = np.argsort(lv, axis=-1, kind="stable")
+    srt = np.take_along_axis(lv, code_of_rank, axis=-1)
+    rank_of_code = np.argsort(code_of_rank, axis=-1, kind="stable")
+    return srt, code_of_rank, rank_of_code
+
+
+# ---------------------------------------------------------------------------
+# Transform / mapping / reconstruction / detransform (Sec. 3.1-3.3)
+# ---------------------------------------------------------------------------
+
+def transform_F(w, s, delta, zu, sr):
+    """FlexRound transform T_F (Eq. 1): x = w / (Delta * s * s_r) + z_U.
+
+    All arrays grouped: w, s [..., g]; delta, zu, sr broadcastable to [...].
+    fp32, denominator formed left to right ((Delta * s) * s_r).
+    Returns (x, u) with u = x - z_U before the shift (u is also what the
+    backward pass differentiates).
+    """
+    w = np.asarray(w, F32)
+    s = np.asarray(s, F32)
+    denom = (np.asarray(delta, F32)[..., None] * s) * np.asarray(sr, F32)[..., None]
+    u = w / denom
+    x = u + np.asarray(zu, F32)[..., None]
+    return x, u
+
+
+def map_full(x, srt, code_of_rank):
+    """Full nearest-level mapping M_B (Sec. 2.3; Eq. 2): argmin_l |x - l|.
+
+    x [..., g]; srt, code_of_rank [..., L].  fp32 distances; the scan runs
+    over ranks in ascending order and only a strictly smaller distance
+    replaces the best, so ties go to the lower rank.  Returns code words.
+    """
+    x = np.asarray(x, F32)
+    dist = np.abs(x[..., :, None] - srt[..., None, :])     # [..., g, L], fp32
+    best_r = np.argmin(dist, axis=-1)                      # first minimum = lowest rank
+    return np.take_along_axis(code_of_rank, best_r, axis=-1)
+
+
+def map_local(x, codes, srt, code_of_rank, rank_of_code):
+    """Local mapping step of M*_B (Algorithm 4, one remap step).
+
+    Each element looks only at its current level d and the two neighbours
+    max(d-1, 0), min(d+1, L-1) in the sorted level list and takes the
+    nearest (|x - l|, fp32).  Candidates are examined in the order d, d-1,
+    d+1 and replace the best only when strictly nearer.
+    """
+    x = np.asarray(x, F32)
+    L = srt.shape[-1]
+    d = np.take_along_axis(rank_of_code, codes.astype(np.int64), axis=-1)
+    best_r = d
+    best_d = np.abs(x - np.take_along_axis(srt, d, axis=-1))
+    for cand in (np.maximum(d - 1, 0), np.minimum(d + 1, L - 1)):
+        dc = np.abs(x - np.take_along_axis(srt, cand, axis=-1))
+        upd = dc < best_d
+        best_d = np.where(upd, dc, best_d)
+        best_r = np.where(upd, cand, best_r)
+    return np.take_along_axis(code_of_rank, best_r, axis=-1)
+
+
+def reconstruct(codes, lv):
+    """R_B per element: w~ = l(code) (Sec. 2.3, C alpha + z_B)."""
+    return np.take_along_axis(lv, codes.astype(np.int64), axis=-1)
+
+
+def detransform(wt, delta, zu):
+    """D_R (Sec. 3.1): w^ = Delta * (w~ - z_U), fp32."""
+    return np.asarray(delta, F32)[..., None] * (np.asarray(wt, F32) - np.asarray(zu, F32)[..., None])
+
+
+def _grouped(a, out, g):
+    return np.asarray(a).reshape(out, -1, g)
+
+
+def quantize_fwd(W, s, sr, delta, zu, alpha, zb, codes, g, mode=MAP_LOCAL_PERIODIC, step=0, p=2):
+    """UniQuan_F quantizer Q*_IF = D_R o M*_B o T_F (Eq. 3), or Q_IF (Eq. 2).
+
+    W, s: [out, in] (W already as fp32 values); sr: [out]; delta, zu, zb:
+    [out, in/g]; alpha: [out, in/g, q]; codes: [out, in] code words (ignored
+    for MAP_FULL).  mode MAP_FULL re-maps every element to the nearest of all
+    levels (Eq. 2); MAP_LOCAL_PERIODIC applies Algorithm 4 (re-map locally
+    when step % p == 0, keep the codes otherwise).
+
+    Returns (w_hat fp32 [out, in], codes uint8 [out, in]).
+    """
+    out, n_in = np.shape(W)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    sg = _grouped(np.asarray(s, F32), out, g)
+    lv = levels(alpha, zb)
+    srt, cor, roc = sorted_levels(lv)
+    if mode == MAP_FULL:
+        x, _ = transform_F(Wg, sg, delta, zu, np.asarray(sr)[:, None])
+        new = map_full(x, srt, cor)
+    elif step % p == 0:
+        x, _ = transform_F(Wg, sg, delta, zu, np.asarray(sr)[:, None])
+        new = map_local(x, _grouped(codes, out, g).astype(np.int64), srt, cor, roc)
+    else:
+        new = _grouped(codes, out, g).astype(np.int64)
+    what = detransform(reconstruct(new, lv), delta, zu)
+    return what.reshape(out, n_in).astype(F32), new.reshape(out, n_in).astype(np.uint8)
+
+
+# ---------------------------------------------------------------------------
+# Backward: straight-through estimator with gradient filtering (App. C.1)
+# ---------------------------------------------------------------------------
+
+def _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+    out, n_in = np.shape(W)
+    q = np.shape(alpha)[-1]
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    sg = _grouped(np.asarray(s, F32), out, g)
+    cg = _grouped(codes, out, g).astype(np.int64)
+    # fp32 decision: the filter compares |x - w~| with tau = min_j |alpha_j|.
+    x32, _ = transform_F(Wg, sg, delta, zu, np.asarray(sr)[:, None])
+    m32 = reconstruct(cg, levels(alpha, zb))
+    tau = np.min(np.abs(np.asarray(alpha, F32)), axis=-1)
+    f = np.abs(x32 - m32) <= tau[..., None]
+    # fp64 values.
+    W64 = Wg.astype(F64)
+    s64 = sg.astype(F64)
+    d64 = np.asarray(delta, F64)[..., None]
+    zu64 = np.asarray(zu, F64)[..., None]
+    sr64 = np.asarray(sr, F64)
+    u64 = W64 / (d64 * s64 * sr64[:, None, None])
+    C = signs(q, F64)[cg]                                   # [out, Gr, g, q]
+    m64 = (C * np.asarray(alpha, F64)[..., None, :]).sum(-1) + np.asarray(zb, F64)[..., None]
+    G64 = _grouped(np.asarray(Gup, F64), out, g)
+    gbar = G64 * d64                                        # dL/dw~ = G * Delta
+    fu = np.where(f, u64, 0.0)
+    return dict(f=f, u=u64, m=m64, zu=zu64, s=s64, sr=sr64, G=G64, gbar=gbar, fu=fu, C=C)
+
+
+def quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+    """Gradients of L w.r.t. Theta_IF given G = dL/dW^ (App. C.1, Eq. 3).
+
+    Differentiates w^ = Delta * (w~ - z_U) with
+      w~ = c . alpha + z_B                   (codes held fixed),
+      dw~/dx = 1 if |x - w~| <= tau else 0   (straight-through estimator,
+                                              filtered as in App. C.1),
+      x = w / (Delta s s_r) + z_U            (Eq. 1).
+    With u = w / (Delta s s_r) and f the filter:
+      ds_i    = -G_i Delta f_i u_i / s_i
+      dDelta  = sum_i G_i ((w~_i - z_U) - f_i u_i)
+      dz_U    = sum_i G_i Delta (f_i - 1)
+      dz_B    = sum_i G_i Delta
+      dalpha_j= sum_i G_i Delta c_ij
+      ds_r    = -sum_{i in row} G_i Delta f_i u_i / s_r
+    Filter decisions in fp32, values and sums in fp64.  Returns a dict of
+    fp64 arrays shaped like the parameters.
+    """
+    out, n_in = np.shape(W)
+    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g)
+    gbar, fu = t["gbar"], t["fu"]
+    return dict(
+        ds=(-gbar * fu / t["s"]).reshape(out, n_in),
+        ddelta=(t["G"] * ((t["m"] - t["zu"]) - fu)).sum(-1),
+        dzu=(gbar * (t["f"].astype(F64) - 1.0)).sum(-1),
+        dzb=gbar.sum(-1),
+        dalpha=(gbar[..., None] * t["C"]).sum(-2),
+        dsr=-(gbar * fu).sum(axis=(1, 2)) / t["sr"],
+    )
+
+
+def bwd_l1_mass(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+    """L1 mass sum_i |term_i| of every reduction in quantize_bwd (fp64).
+
+    A summation of n terms in any order cannot be trusted beyond a multiple
+    of (unit roundoff) x (sum of |terms|); the parity tests scale their
+    tolerance by this mass.  ds gets its own per-element values back.
+    """
+    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g)
+    gbar, fu = t["gbar"], t["fu"]
+    q = np.shape(alpha)[-1]
+    mass_gbar = np.abs(gbar).sum(-1)
+    return dict(
+        ddelta=np.abs(t["G"] * ((t["m"] - t["zu"]) - fu)).sum(-1),
+        dzu=np.abs(gbar * (t["f"].astype(F64) - 1.0)).sum(-1),
+        dzb=mass_gbar,
+        dalpha=np.repeat(mass_gbar[..., None], q, axis=-1),
+        dsr=np.abs(gbar * fu).sum(axis=(1, 2)) / np.abs(t["sr"]),
+    )
+
+
+# ---------------------------------------------------------------------------
+# Export: unification theorem (Theorem 1) and final codes (Eq. 4)
+# ---------------------------------------------------------------------------
+
+def unify(delta, zu, alpha, zb):
+    """Theorem 1 (proof in App. E.5): alpha* = Delta alpha, z_B* = Delta (z_B - z_U).
+
+    fp32; z_B - z_U is formed first, then scaled.
+    """
+    delta = np.asarray(delta, F32)
+    alpha_star = delta[..., None] * np.asarray(alpha, F32)
+    zb_star = delta * (np.asarray(zb, F32) - np.asarray(zu, F32))
+    return alpha_star.astype(F32), zb_star.astype(F32)
+
+
+def codes_eq4(W, alpha_star, zb_star, g):
+    """Eq. 4: C = argmin_C' || w - (C' alpha* + z_B*) ||^2, per element.
+
+    Same nearest-level rule as map_full, on the levels of Theta_B* and the
+    original weights (no s, no s_r).
+    """
+    out, n_in = np.shape(W)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    srt, cor, _ = sorted_levels(levels(alpha_star, zb_star))
+    return map_full(Wg, srt, cor).reshape(out, n_in).astype(np.uint8)
+
+
+def pack_bitplanes(codes, q):
+    """Bit-plane layout of the binary code matrix C (App. F.1: 1 bit per code).
+
+    codes [out, in] uint8 -> planes uint32 [q, out, in/32] with
+    bit b of planes[j, r, t] = 1  <=>  c_{j+1} = +1 for column 32 t + b.
+    """
+    codes = np.asarray(codes, np.uint32)
+    out, n_in = codes.shape
+    bits = (codes[None, :, :] >> np.arange(q, dtype=np.uint32)[:, None, None]) & 1
+    bits = bits.reshape(q, out, n_in // 32, 32)
+    weights = (np.uint64(1) << np.arange(32, dtype=np.uint64))
+    return (bits.astype(np.uint64) * weights).sum(-1).astype(np.uint32)
+
+
+def export_bcq(W, delta, zu, alpha, zb, codes, g, mode=EXPORT_REUSE_CODES):
+    """Algorithm 1 lines 10-11: Theta_B* by Theorem 1, then the code matrix.
+
+    mode EXPORT_REUSE_CODES keeps the codes of the last quantizer step (for
+    which Theorem 1 makes R_B(C; Theta_B*) equal the quantizer output);
+    EXPORT_REMAP_EQ4 recomputes them from the original weights by Eq. 4.
+    Returns (planes [q, out, in/32] uint32, alpha* [out, in/g, q], z_B*
+    [out, in/g], codes used [out, in] uint8).
+    """
+    q = np.shape(alpha)[-1]
+    a_star, z_star = unify(delta, zu, alpha, zb)
+    if mode == EXPORT_REMAP_EQ4:
+        c = codes_eq4(W, a_star, z_star, g)
+    else:
+        c = np.asarray(codes, np.uint8)
+    return pack_bitplanes(c, q), a_star, z_star, c
+
+
+# ---------------------------------------------------------------------------
+# Unified initialization (Algorithm 2, App. E.2 clipping, Algorithm 3)
+# ---------------------------------------------------------------------------
+
+def clip_params(wm, wM, gamma, q, strategy=CLIP_FIXED_MIN):
+    """Candidate Delta', z'_U for clipping ratio gamma (App. E.2), fp32.
+
+    Delta' = gamma (w_M - w_m) / (2^q - 1) with w_M - w_m floored at 1e-12
+    (a constant group would otherwise divide by zero);
+      Fixed-minimum:  z'_U = -w_m / Delta'            (T_F(w_m) = 0)
+      Fixed-maximum:  z'_U = (2^q - 1) - w_M / Delta'  (T_F(w_M) = 2^q - 1)
+      Balanced:       z'_U = -(gamma w_m) / Delta'     (T_F(gamma w_m) = 0)
+    """
+    wm = np.asarray(wm, F32)
+    wM = np.asarray(wM, F32)
+    gamma = F32(gamma)
+    top = F32((1 << q) - 1)
+    rng = np.maximum(wM - wm, F32(1e-12))
+    delta = (gamma * rng) / top
+    if strategy == CLIP_FIXED_MIN:
+        zu = (-wm) / delta
+    elif strategy == CLIP_FIXED_MAX:
+        zu = top - wM / delta
+    elif strategy == CLIP_BALANCED:
+        zu = (-(gamma * wm)) / delta
+    else:
+        raise ValueError(f"unknown clipping strategy {strategy}")
+    return delta.astype(F32), zu.astype(F32)
+
+
+def greedy_init(x, zb, q):
+    """Greedy BCQ initialisation used by Algorithm 3 (one bit at a time).
+
+    With r = x - z_B: for j = 1..q, c_j = sign(r) (r >= 0 -> +1),
+    alpha_j = mean |r| (fp64 sum, stored fp32), r <- r - c_j alpha_j (fp32).
+    x [NG, g] fp32; zb [NG].  Returns (alpha [NG, q] fp32, codes [NG, g]).
+    """
+    x = np.asarray(x, F32)
+    NG, g = x.shape
+    r = x - np.asarray(zb, F32)[:, None]
+    alpha = np.zeros((NG, q), F32)
+    codes = np.zeros((NG, g), np.int64)
+    for j in range(q):
+        pos = r >= 0
+        a = (np.abs(r).astype(F64).sum(-1) / g).astype(F32)
+        alpha[:, j] = a
+        codes |= pos.astype(np.int64) << j
+        r = r - np.where(pos, F32(1), F32(-1)) * a[:, None]
+    return alpha, codes
+
+
+def _sq_err(x64, C, alpha, zb):
+    rec = (C * np.asarray(alpha, F64)[:, None, :]).sum(-1) + np.asarray(zb, F64)[:, None]
+    return ((x64 - rec) ** 2).sum(-1)
+
+
+def general_alternating(x, zb, G, T, q, trace=False):
+    """General alternating update (Algorithm 3) on transformed groups x.
+
+    Greedy start, then T rounds of
+      alpha <- (C^T C)^{-1} C^T (x - z_B 1)     (fp64; if C^T C is singular
+                                                  alpha is left unchanged)
+      C     <- argmin_C' || x - (C' alpha + z_B 1) ||^2   (= map_full)
+      z_B   <- sum_i (x_i - C_i alpha) / g       (only when G == 1)
+    alpha and z_B are stored in fp32 after each update.
+    x [NG, g]; zb [NG].  Returns (alpha, zb, codes[, errors per round]).
+    """
+    x = np.asarray(x, F32)
+    NG, g = x.shape
+    zb = np.array(zb, F32, copy=True).reshape(NG)
+    x64 = x.astype(F64)
+    S = signs(q, F64)
+    alpha, codes = greedy_init(x, zb, q)
+    errs = []
+    for _ in range(T):
+        C = S[codes]                                         # [NG, g, q]
+        Ct = C.transpose(0, 2, 1)
+        CtC = Ct @ C
+        Cty = (Ct @ (x64 - zb.astype(F64)[:, None])[..., None])[..., 0]
+        det = np.rint(np.linalg.det(CtC))                    # integer matrix
+        ok = det != 0
+        if ok.any():
+            inv = np.linalg.inv(CtC[ok])
+            alpha[ok] = (inv @ Cty[ok][..., None])[..., 0].astype(F32)
+        srt, cor, _ = sorted_levels(levels(alpha, zb))
+        codes = map_full(x, srt, cor)
+        if G == 1:
+            C = S[codes]
+            resid = x64 - (C * alpha.astype(F64)[:, None, :]).sum(-1)
+            zb = (resid.sum(-1) / g).astype(F32)
+        if trace:
+            errs.append(_sq_err(x64, S[codes], alpha, zb))
+    if trace:
+        return alpha, zb, codes, errs
+    return alpha, zb, codes
+
+
+def unified_init(W, q, g, G=30, T=15, clip=CLIP_FIXED_MIN, return_errors=False):
+    """Unified initialization (Algorithm 2) of every group of W [out, in].
+
+    s = 1, s_r = 1, z_B starts at (2^q - 1)/2.  For gamma = 1/G, 2/G, ..., 1
+    (gamma_i = float32(i) / float32(G)): clip (App. E.2) -> T_F -> general
+    alternating update (Algorithm 3) -> quantize with the full mapping ->
+    e' = ||w - w^||^2 (fp64); a candidate replaces the kept one only when
+    e' < e.  The initial codes are the full mapping of T_F(w) under the kept
+    parameters (App. E.4: the mapping starts from distances to all levels).
+
+    Returns dict(delta, zu, alpha, zb [per group], s [out, in], sr [out],
+    codes [out, in] uint8) and, if return_errors, the per-candidate errors
+    [G, NG] and the chosen candidate index per group.
+    """
+    W = np.asarray(W, F32)
+    out, n_in = W.shape
+    Gr = n_in // g
+    NG = out * Gr
+    w = W.reshape(NG, g)
+    w64 = w.astype(F64)
+    wm = w.min(-1)
+    wM = w.max(-1)
+    ones_g = np.ones((NG, g), F32)
+    ones_r = np.ones(NG, F32)
+    zb = np.full(NG, F32(((1 << q) - 1) / 2), F32)
+    best = dict(delta=np.zeros(NG, F32), zu=np.zeros(NG, F32),
+                alpha=np.zeros((NG, q), F32), zb=zb.copy())
+    e_best = np.full(NG, np.inf)
+    chosen = np.full(NG, -1, np.int64)
+    all_errs = []
+    for i in range(1, G + 1):
+        gamma = F32(i) / F32(G)
+        d_c, zu_c = clip_params(wm, wM, gamma, q, clip)
+        x, _ = transform_F(w, ones_g, d_c, zu_c, ones_r)
+        a_c, zb_c, _ = general_alternating(x, best["zb"], G, T, q)
+        lv = levels(a_c, zb_c)
+        srt, cor, _ = sorted_levels(lv)
+        what = detransform(reconstruct(map_full(x, srt, cor), lv), d_c, zu_c)
+        e = ((w64 - what.astype(F64)) ** 2).sum(-1)
+        all_errs.append(e)
+        acc = e < e_best
+        best["delta"] = np.where(acc, d_c, best["delta"])
+        best["zu"] = np.where(acc, zu_c, best["zu"])
+        best["alpha"] = np.where(acc[:, None], a_c, best["alpha"])
+        best["zb"] = np.where(acc, zb_c, best["zb"])
+        e_best = np.where(acc, e, e_best)
+        chosen = np.where(acc, i - 1, chosen)
+    x, _ = transform_F(w, ones_g, best["delta"], best["zu"], ones_r)
+    srt, cor, _ = sorted_levels(levels(best["alpha"], best["zb"]))
+    codes = map_full(x, srt, cor)
+    res = dict(
+        delta=best["delta"].reshape(out, Gr).astype(F32),
+        zu=best["zu"].reshape(out, Gr).astype(F32),
+        alpha=best["alpha"].reshape(out, Gr, q).astype(F32),
+        zb=best["zb"].reshape(out, Gr).astype(F32),
+        s=np.ones((out, n_in), F32),
+        sr=np.ones(out, F32),
+        codes=codes.reshape(out, n_in).astype(np.uint8),
+    )
+    if return_errors:
+        return res, np.stack(all_errs), chosen.reshape(out, Gr)
+    return res
+
+
+# ---------------------------------------------------------------------------
+# Round-to-nearest (Sec. 2.2) -- only used to pin M_B by reduction
+# ---------------------------------------------------------------------------
+
+def rtn(w, delta, zu, q):
+    """RTN quantizer Q_R (Sec. 2.2): Delta (Clip(round(w/Delta + z_U), 0, 2^q-1) - z_U).
+
+    fp32; round half to even.  Not part of the product: the tests use it to
+    pin the full mapping on the uniform BCQ level set.
+    """
+    w = np.asarray(w, F32)
+    delta = np.asarray(delta, F32)[..., None]
+    zu = np.asarray(zu, F32)[..., None]
+    wt = np.clip(np.rint(w / delta + zu), 0, (1 << q) - 1).astype(F32)
+    return delta * (wt - zu)
