@@ -1,0 +1,436 @@
+"""Benchmark of the UniQuan_F quantizer step on GB300.
+
+One step = the quantizer forward (Eq. 3, local and periodic mapping with
+p = 2: remap on even steps, keep on odd steps) + its backward (App. C.1) over
+the whole workload matrix, W resident in HBM.  Between steps the parameters
+change as they would after an SGD update: a ring of parameter sets is
+prepared before timing, each the previous one multiplied by 1 + eps N(0, 1)
+(eps chosen so that ~0.03 % of the codes move per remap step, the paper's
+per-step rate); the ring is generated outside the timed region.
+
+Prints ONE JSON line (rank 0).  --impl reference times the CPU oracle on a
+bounded sample of the same workload instead.  Under torchrun every rank runs
+its own copy of the workload (rows are independent, no exchange step) and
+the slowest rank's time is reported.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "quantizer fwd+bwd weights/sec and achieved HBM GB/s (% of GB300 peak) at q=3,g=128"
+RING = 16                       # parameter sets prepared before timing
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (host logic, tested with gloo on CPU)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Largest value over all ranks (the slowest rank's time)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_value(units_per_rank: int, steps: int, world: int, seconds: float) -> float:
+    """Whole-job throughput: units all ranks processed / the slowest rank's time."""
+    return units_per_rank * steps * world / seconds
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.proc = None
+        self.path = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            cmd = ["nvidia-smi", f"--query-gpu=timestamp,{self.FIELDS}", "--format=csv,noheader,nounits",
+                   "-lms", "100"]
+            if self.gpu_id:
+                cmd += ["-i", self.gpu_id]
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            self.t0 = time.time()
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        time.sleep(max(0.0, 0.35 - (time.time() - self.t0)))
+        self.proc.terminate()
+        self.proc.wait()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+def kernel_hash():
+    h = hashlib.sha256()
+    for f in ("uq_bwd.cu", "uq_common.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2506_03781_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload, q):
+    """DRAM bytes per backward launch from the committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "bwd_traffic.json")
+    try:
+        rec = json.load(open(path))
+    except Exception:
+        return None
+    key = f"{workload}/q{q}"
+    ent = rec.get(key)
+    if not ent or ent.get("kernel_hash") != kernel_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the cpu_baseline / --impl reference legs)
+# ---------------------------------------------------------------------------
+
+def oracle_sample_inputs(wl, q, rows):
+    """Oracle-initialised inputs of the first ``rows`` rows of the workload."""
+    import oracle as O
+    from paper_2506_03781_gb300 import synth
+    _, W = synth.workload_weights(wl, 0, slice(0, rows))
+    g = wl.g
+    init = O.unified_init(W, q, g, G=2, T=2)
+    P = {k: init[k] for k in ("delta", "zu", "s", "sr", "alpha", "zb")}
+    P = synth.jitter(P, synth.perturb_factors(synth.param_shapes(rows, W.shape[1], g, q), wl.init_eps, 0))
+    Gup = synth.upstream_grad(rows, W.shape[1], wl.grad_var, 0)
+    return W, P, init["codes"], Gup
+
+
+def time_oracle_step(wl, q, rows, budget_s):
+    """Runs oracle steps (fwd at step t + bwd) until budget_s elapses; returns
+    (weights per second, steps run, seconds)."""
+    import oracle as O
+    W, P, codes, Gup = oracle_sample_inputs(wl, q, rows)
+    g = wl.g
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        _, codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes, g,
+                                  O.MAP_LOCAL_PERIODIC, n, wl.p)
+        O.quantize_bwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes, Gup, g)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s and n >= 2:
+            break
+    return W.size * n / el, n, el
+
+
+# ---------------------------------------------------------------------------
+# GPU run
+# ---------------------------------------------------------------------------
+
+def run_gpu(args):
+    import torch
+    from paper_2506_03781_gb300 import api, roofline, synth
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    wl = synth.WORKLOADS[args.workload]
+    m = wl.matrices[0]
+    q, g = args.q, wl.g
+    out, n_in = m.out, m.n_in
+    N = out * n_in
+
+    raw, _ = synth.workload_weights(wl, 0)
+    Wd = api.weights_tensor(raw, dev)
+    wbytes = Wd.element_size()
+    p0 = api.empty_params(out, n_in, q, g, dev)
+    codes = torch.empty(out, n_in, dtype=torch.uint8, device=dev)
+    api.uq_init_params(Wd, q, g, p0, codes, G=wl.G, T=wl.T)
+
+    # parameter ring: set_0 = init * (1 + init_eps N), set_t = set_{t-1} * (1 + step_eps N)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 * wl.seed + q)
+    jit = ("delta", "s", "sr", "alpha")
+
+    def jitter(p, eps):
+        outp = dict(p)
+        for k in jit:
+            outp[k] = p[k] * (1.0 + eps * torch.randn(p[k].shape, generator=gen, device=dev))
+        return outp
+
+    ring = [jitter(p0, wl.init_eps)]
+    for _ in range(1, min(RING, args.warmup + args.steps)):
+        ring.append(jitter(ring[-1], wl.step_eps))
+    Gup = torch.randn(out, n_in, generator=gen, device=dev) * float(np.sqrt(wl.grad_var))
+    what = torch.empty(out, n_in, dtype=torch.float32, device=dev)
+    grads = api.empty_grads(out, n_in, q, g, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(t, ev=None):
+        P = ring[t % len(ring)]
+        if ev is not None:
+            ev[0].record(stream)
+        api.uq_quantize_fwd(Wd, q, g, P, codes, what, api.MAP_LOCAL_PERIODIC, t, wl.p, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        api.uq_quantize_bwd(Wd, q, g, P, codes, Gup, grads, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for t in range(args.warmup):
+        step(t)
+    torch.cuda.synchronize()
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    gpu_id = None
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        gpu_id = gpu_id if gpu_id.startswith("GPU-") else "GPU-" + gpu_id
+    except Exception:
+        gpu_id = None
+    clk = ClockSampler(gpu_id)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clk.start()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for t in range(args.steps):
+        step(args.warmup + t, evs[t])
+    end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = clk.stop()
+    ms = start.elapsed_time(end)
+    ms_max = max_over_ranks(ms, world, dev)
+    secs = ms_max / 1e3
+    value = weak_scaling_value(N, args.steps, world, secs)
+
+    fwd_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    bwd_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    bwd_bytes = roofline.bytes_per_launch("bwd", out, n_in, q, g, wbytes)
+    steps_idx = [args.warmup + t for t in range(args.steps)]
+    step_bytes = sum(roofline.step_bytes(out, n_in, q, g, wbytes, t % wl.p == 0) for t in steps_idx)
+    peaks = measured_peaks()
+    peak = peaks["hbm_gbs"] if peaks else 6800.0
+    bwd_avg_s = statistics.mean(bwd_ms) / 1e3
+    achieved = bwd_bytes / bwd_avg_s / 1e9
+    fwd_remap = [f for f, t in zip(fwd_ms, steps_idx) if t % wl.p == 0]
+    fwd_keep = [f for f, t in zip(fwd_ms, steps_idx) if t % wl.p != 0]
+
+    # export timed separately (one launch after the steps)
+    planes = torch.empty(q, out, n_in // 32, dtype=torch.int32, device=dev)
+    a_s = torch.empty(out, n_in // g, q, dtype=torch.float32, device=dev)
+    z_s = torch.empty(out, n_in // g, dtype=torch.float32, device=dev)
+    P_last = ring[(args.warmup + args.steps - 1) % len(ring)]
+    ex = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for _ in range(3):
+        api.uq_export_bcq(Wd, q, g, P_last, codes, planes, a_s, z_s, api.EXPORT_REUSE_CODES, stream=stream)
+    ex[0].record(stream)
+    api.uq_export_bcq(Wd, q, g, P_last, codes, planes, a_s, z_s, api.EXPORT_REUSE_CODES, stream=stream)
+    ex[1].record(stream)
+    torch.cuda.synchronize()
+    exp_ms = ex[0].elapsed_time(ex[1])
+    exp_bytes = roofline.bytes_per_launch("export_reuse", out, n_in, q, g, wbytes)
+
+    # end-to-end through the public host-buffer API: H2D inputs, fwd+bwd, D2H results
+    hs = api.HostStep(out, n_in, q, g, Wd.dtype, dev)
+    hin, hout = hs.empty_host(pinned=True)
+    hin["W"].copy_(Wd.cpu())
+    for k in api.PARAM_NAMES:
+        hin[k].copy_(ring[0][k].cpu())
+    hin["codes"].copy_(codes.cpu())
+    hin["dL_dWhat"].copy_(Gup.cpu())
+    e2e_steps = max(3, min(args.steps, 20))
+    for t in range(2):
+        hs.run(hin, hout, t, wl.p)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(hs.stream)
+    for t in range(e2e_steps):
+        hs.run(hin, hout, t, wl.p)
+    e1.record(hs.stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
+    e2e_value = weak_scaling_value(N, e2e_steps, world, e2e_ms / 1e3)
+
+    result = None
+    if rank == 0:
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            rows = 96
+            v, n, el = time_oracle_step(wl, q, rows, args.cpu_budget)
+            cpu = {"value": v, "unit": "weights/s", "cores": 1, "kind": "oracle",
+                   "sample": f"first {rows} rows of {out}x{n_in} ({rows * n_in} weights), {n} oracle steps "
+                             f"(local remap/keep alternating + backward) in {el:.1f} s, numpy single thread"}
+        result = {
+            "metric": METRIC,
+            "value": value,
+            "unit": "weights/s",
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": ms_max / args.steps,
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "f32 (bf16 W)",
+            "data": "synthetic (seeded Student-t(4) weights with outlier columns; no model weights)",
+            "config": {"workload": wl.name, "shape": [out, n_in], "q": q, "g": g, "mapping": "local, p=2",
+                       "weights_per_step": N, "ring_of_parameter_sets": len(ring),
+                       "l2": "inputs larger than L2 (about 1.5 GB moved per step vs 129 MB L2)",
+                       "step_bytes_avg": step_bytes / args.steps,
+                       "hbm_gbs_step": step_bytes / secs / 1e9 * world},
+            "roofline": {"bound": "hbm", "kernel": "uq_bwd", "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": recorded_traffic(wl.name, q),
+                         "algorithmic_bytes": bwd_bytes, "avg_ms": bwd_avg_s * 1e3,
+                         "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback"},
+            "kernels": {
+                "fwd_remap": {"avg_ms": statistics.mean(fwd_remap) if fwd_remap else None,
+                              "gbs": (roofline.bytes_per_launch("fwd_remap", out, n_in, q, g, wbytes) / 1e6
+                                      / statistics.mean(fwd_remap)) if fwd_remap else None},
+                "fwd_keep": {"avg_ms": statistics.mean(fwd_keep) if fwd_keep else None,
+                             "gbs": (roofline.bytes_per_launch("fwd_keep", out, n_in, q, g, wbytes) / 1e6
+                                     / statistics.mean(fwd_keep)) if fwd_keep else None},
+                "bwd": {"avg_ms": bwd_avg_s * 1e3, "gbs": achieved},
+                "export_reuse": {"ms": exp_ms, "gbs": exp_bytes / 1e6 / exp_ms},
+            },
+            "e2e": {"value": e2e_value, "unit": "weights/s",
+                    "h2d_bytes_per_step": hs.bytes_in(hin), "d2h_bytes_per_step": hs.bytes_out(hout),
+                    "steps": e2e_steps, "api": "paper_2506_03781_gb300.api.HostStep (pinned host buffers)"},
+            "gpu_launches": 2 * args.steps,
+            "clocks": clocks,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(result))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return result
+
+
+def run_reference(args):
+    """The CPU oracle as it stands, on a bounded sample of the same workload."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    from paper_2506_03781_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    m = wl.matrices[0]
+    rows = 64
+    per_step = max(1.0, args.cpu_budget / max(1, args.steps))
+    vals = []
+    t_all = 0.0
+    for _ in range(args.warmup):
+        time_oracle_step(wl, args.q, rows, 0.0)
+    for _ in range(args.steps):
+        v, n, el = time_oracle_step(wl, args.q, rows, per_step)
+        vals.append(v)
+        t_all += el
+    value = statistics.median(vals)
+    sample = (f"first {rows} rows of {m.out}x{m.n_in} per step ({rows * m.n_in} weights), oracle fwd "
+              f"(local mapping) + bwd, numpy single thread")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "weights/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": rows * m.n_in / value * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32/f64 (oracle)",
+            "data": "synthetic", "config": {"workload": wl.name, "shape": [m.out, m.n_in], "q": args.q, "g": wl.g},
+            "cpu_baseline": {"value": value, "unit": "weights/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "weights/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return line
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default="mlp14336x4096_bf16")
+    ap.add_argument("--q", type=int, default=3)
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU work")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)          # at least 3 untimed warm-up steps
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,202 @@
+/*
+ * uq_api.h -- C ABI of the GB300 (sm_103a) UniQuan_F weight quantizer.
+ *
+ * UniQuan_F (arXiv 2506.03781) quantizes each group of g weights of a
+ * weight matrix W [out, in] with
+ *     w^ = Q*_IF(w) = D_R( M*_B( T_F(w; Delta, z_U, s, s_r); alpha, z_B ); Delta, z_U )   (Eq. 3)
+ *   T_F  (Eq. 1)       x   = w / (Delta * s * s_r) + z_U
+ *   M_B  (Sec. 2.3)    code of the nearest of the 2^q BCQ levels  l(c) = c . alpha + z_B
+ *   M*_B (Algorithm 4) every p steps, nearest among the current level and its two
+ *                      neighbours in the sorted level list; codes kept in between
+ *   D_R  (Sec. 3.1)    w^  = Delta * (l(c) - z_U)
+ * and trains Delta, z_U, s, s_r, alpha, z_B by SGD through a straight-through
+ * estimator with gradient filtering (App. C.1).  After training, Theorem 1
+ * folds D_R into the BCQ parameters (alpha* = Delta alpha,
+ * z_B* = Delta (z_B - z_U)) and the binary codes are exported as bit-planes
+ * (Algorithm 1, lines 10-11; Eq. 4).
+ *
+ * Conventions common to every entry point
+ * ---------------------------------------
+ * Memory.  Every pointer argument is DEVICE memory owned by the caller
+ *   (except the return value of uq_last_error).  The library never allocates,
+ *   frees or keeps a pointer after a call returns.
+ * Asynchrony.  Work is enqueued on `stream` (a cudaStream_t; NULL = the
+ *   legacy default stream) and the call returns without synchronising.
+ *   UQ_OK means "validated and launched"; execution errors surface on the
+ *   stream as usual.
+ * Layouts (row-major, contiguous, no padding):
+ *   W       [out, in]      fp32 (UQ_W_F32) or bf16 (UQ_W_BF16), read only
+ *   s       [out, in]      fp32   per-element FlexRound scale
+ *   s_r     [out]          fp32   per-row scale
+ *   Delta, z_U, z_B [out, in/g] fp32   per-group parameters
+ *   alpha   [out, in/g, q] fp32   alpha_1 first
+ *   codes   [out, in]      uint8  code word: bit (j-1) set <=> c_j = +1; bits
+ *                                 at or above q are ignored on input and
+ *                                 written as zero
+ *   W_hat, dL/dW_hat, ds [out, in] fp32
+ *   bit-planes [q, out, in/32] uint32: bit b of planes[j][r][t] is c_{j+1}
+ *                                 of column 32 t + b (1 <=> +1)
+ * Shapes.  1 <= q <= 4; g in {32, 64} or g a multiple of 128; in a multiple
+ *   of g; out >= 1; in <= 196608 (the backward pass keeps one row's group
+ *   partial sums on chip for g > 128).
+ * Alignment.  Every pointer must be 16-byte aligned.
+ * Errors.  Arguments are checked before anything is launched; on error the
+ *   call returns a non-zero uq_status, launches nothing, writes nothing, and
+ *   uq_last_error() describes the problem.  UQ_ERR_CUDA reports a failed
+ *   launch (cudaGetLastError after the launch).  No entry point aborts,
+ *   exits or traps the device.
+ * Determinism.  No atomics are used; a call repeated on the same inputs
+ *   gives bitwise-identical outputs.
+ * Numerics.  Every value that decides an integer (x, the levels, the
+ *   distances, the filter test) is computed in IEEE fp32 with the operation
+ *   order written at each entry point, no FMA contraction; gradients are
+ *   accumulated in fp32.
+ */
+#ifndef UQ_API_H
+#define UQ_API_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    UQ_OK = 0,
+    UQ_ERR_ARG = 1,          /* null pointer, bad shape, bad enum value      */
+    UQ_ERR_UNSUPPORTED = 2,  /* valid per the method but not built (q, g)    */
+    UQ_ERR_ALIGN = 3,        /* a pointer is not 16-byte aligned             */
+    UQ_ERR_CUDA = 4          /* the CUDA runtime reported an error           */
+} uq_status;
+
+typedef enum { UQ_W_F32 = 0, UQ_W_BF16 = 1 } uq_wdtype;
+
+/* Clipping strategies of the unified initialization (App. E.2). */
+typedef enum { UQ_CLIP_FIXED_MIN = 0, UQ_CLIP_FIXED_MAX = 1, UQ_CLIP_BALANCED = 2 } uq_clip;
+
+/* Mapping: full nearest level every call (Eq. 2, "UniQuan_F-0"), or the
+ * local and periodic mapping M*_B of Algorithm 4 (Eq. 3). */
+typedef enum { UQ_MAP_FULL = 0, UQ_MAP_LOCAL_PERIODIC = 1 } uq_map;
+
+/* Export: reuse the codes of the last quantizer call (for which Theorem 1
+ * makes R_B(C; Theta_B*) equal the quantizer output), or recompute them
+ * from the original weights by Eq. 4. */
+typedef enum { UQ_EXPORT_REUSE_CODES = 0, UQ_EXPORT_REMAP_EQ4 = 1 } uq_export_mode;
+
+/* The learnable parameters Theta_IF = Theta_F u Theta_B (Eq. 1, Sec. 2.3). */
+typedef struct {
+    float* delta;   /* [out, in/g]    Delta                                */
+    float* zu;      /* [out, in/g]    z_U                                  */
+    float* s;       /* [out, in]      s   (element-wise scale)             */
+    float* sr;      /* [out]          s_r (row-wise scale)                 */
+    float* alpha;   /* [out, in/g, q] alpha                                */
+    float* zb;      /* [out, in/g]    z_B                                  */
+} uq_params;
+
+/* Gradients of the loss w.r.t. each parameter, same shapes as uq_params. */
+typedef struct {
+    float* ddelta;
+    float* dzu;
+    float* ds;
+    float* dsr;
+    float* dalpha;
+    float* dzb;
+} uq_grads;
+
+/*
+ * uq_init_params -- unified initialization (Algorithm 2 with the general
+ * alternating update of Algorithm 3 and the clipping strategies of App. E.2).
+ *
+ * For every group: w_m, w_M = min, max of the group; z_B starts at
+ * (2^q - 1)/2, s = 1, s_r = 1.  For gamma_i = float(i)/float(G), i = 1..G:
+ *   Delta' = (gamma (w_M - w_m)) / (2^q - 1)   (w_M - w_m floored at 1e-12)
+ *   z'_U   = -w_m/Delta' | (2^q-1) - w_M/Delta' | -(gamma w_m)/Delta'   (clip)
+ *   x      = T_F(w) with s = s_r = 1
+ *   greedy start: r = x - z_B; for j: c_j = sign(r) (0 -> +1),
+ *                 alpha_j = mean |r| (fp64 sum), r -= c_j alpha_j
+ *   T rounds of: alpha <- (C^T C)^{-1} C^T (x - z_B)  (fp64; unchanged when
+ *                C^T C is singular), C <- nearest level, and if G == 1
+ *                z_B <- mean(x - C alpha) (fp64)
+ *   e' = sum (w - w^)^2 in fp64 with the full mapping; kept if e' < e.
+ * Writes delta, zu, alpha, zb for every group, s = 1 for every element,
+ * sr = 1 for every row, and the codes of the full mapping under the kept
+ * parameters.  G >= 1, T >= 0, g <= 32768.  Not on the per-step path.
+ * W is read only; every params pointer and `codes` is written.
+ */
+uq_status uq_init_params(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                         int G, int T, uq_clip clip, uq_params params, uint8_t* codes, void* stream);
+
+/*
+ * uq_quantize_fwd -- the quantizer Q*_IF (Eq. 3) or Q_IF (Eq. 2).
+ *
+ * map == UQ_MAP_FULL: every element is mapped to the nearest of all 2^q
+ *   levels: codes is written (not read), W_hat is written.
+ * map == UQ_MAP_LOCAL_PERIODIC and step % p_period == 0 (a remap step,
+ *   Algorithm 4): for each element with current rank d in the ascending
+ *   level order of its group, the nearest of ranks d, max(d-1,0),
+ *   min(d+1,2^q-1) (examined in that order, replaced only when strictly
+ *   nearer) is taken; codes is read and rewritten, W_hat written.
+ * map == UQ_MAP_LOCAL_PERIODIC and step % p_period != 0: codes is kept (not
+ *   written) and W_hat = D_R(l(code)) with the current alpha, z_B; W, s and
+ *   s_r are not read (they may be NULL).
+ * Arithmetic (fp32): den = (Delta * s) * s_r; x = w / den + z_U;
+ *   l(c) = ((c_1 a_1 + c_2 a_2) + ... + c_q a_q) + z_B; levels sorted
+ *   ascending, equal values by ascending code word; full mapping ties go to
+ *   the lower rank; W_hat = Delta * (l(c) - z_U).
+ * params.delta/zu/alpha/zb are read; s, sr read on remap/full calls.
+ * step >= 0, p_period >= 1.
+ */
+uq_status uq_quantize_fwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                          uq_params params, uint8_t* codes, uq_map map, int64_t step, int p_period,
+                          float* W_hat, void* stream);
+
+/*
+ * uq_quantize_bwd -- gradients through Eq. 3 with the straight-through
+ * estimator and gradient filtering of App. C.1, given G = dL/dW_hat.
+ *
+ * The codes are those of the forward call this backward belongs to.  With
+ * u = w / ((Delta s) s_r), x = u + z_U, m = l(code), tau = min_j |alpha_j|
+ * and f = (|x - m| <= tau) (fp32 decision):
+ *   ds_i     = -G_i Delta f_i u_i / s_i
+ *   dDelta   = sum_{i in group} G_i ((m_i - z_U) - f_i u_i)
+ *   dz_U     = sum G_i Delta (f_i - 1)
+ *   dz_B     = sum G_i Delta
+ *   dalpha_j = sum G_i Delta c_ij
+ *   ds_r     = -sum_{i in row} G_i Delta f_i u_i / s_r
+ * Every grads pointer is written (overwritten, not accumulated).  Group
+ * sums are reduced inside each group's warp(s) and row sums inside the
+ * row's thread block: no atomics.
+ */
+uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                          uq_params params, const uint8_t* codes, const float* dL_dWhat,
+                          uq_grads grads, void* stream);
+
+/*
+ * uq_export_bcq -- Theorem 1 and the final binary codes (Algorithm 1,
+ * lines 10-11).
+ *
+ * alpha_star[r, k, j] = Delta * alpha_j and zb_star[r, k] = Delta * (z_B - z_U)
+ * (fp32, z_B - z_U first).  The code matrix is the stored codes
+ * (UQ_EXPORT_REUSE_CODES; W may be NULL) or, for UQ_EXPORT_REMAP_EQ4, the
+ * nearest level of Theta_B* to each original weight w (Eq. 4, same sorting
+ * and tie rule as the full mapping; codes may be NULL).  Writes
+ * bitplanes [q, out, in/32], alpha_star [out, in/g, q], zb_star [out, in/g].
+ * params.s and params.sr are not used (may be NULL).
+ */
+uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                        uq_params params, const uint8_t* codes, uq_export_mode mode,
+                        uint32_t* bitplanes, float* alpha_star, float* zb_star, void* stream);
+
+/* Message for the last non-OK status returned on the calling thread (never
+ * NULL; "" if none).  Owned by the library, valid until the next call on
+ * the same thread. */
+const char* uq_last_error(void);
+
+/* Version of this ABI (incremented on any incompatible change). */
+int uq_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* UQ_API_H */

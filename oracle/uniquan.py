@@ -31,6 +31,8 @@ paper leaves open; each one is listed with its reason in the design notes):
 
 from __future__ import annotations
 
+import itertools
+
 import numpy as np
 
 __all__ = [
@@ -392,6 +394,27 @@ def _sq_err(x64, C, alpha, zb):
     return ((x64 - rec) ** 2).sum(-1)
 
 
+def _int_det(M):
+    """Exact determinant of integer matrices M [..., q, q] (Leibniz formula).
+
+    Used only to decide whether C^T C is singular.  C^T C is a Gram matrix of
+    +-1 columns, so by Hadamard's inequality |det| <= g^q < 2^63 for g <= 2^15;
+    int64 products and sums may wrap but the result is exact modulo 2^64 and
+    therefore exact.
+    """
+    M = np.asarray(M).astype(np.int64)
+    q = M.shape[-1]
+    total = np.zeros(M.shape[:-2], np.int64)
+    with np.errstate(over="ignore"):
+        for perm in itertools.permutations(range(q)):
+            inversions = sum(1 for a in range(q) for b in range(a + 1, q) if perm[a] > perm[b])
+            term = np.ones(M.shape[:-2], np.int64)
+            for i, j in enumerate(perm):
+                term = term * M[..., i, j]
+            total = total - term if inversions % 2 else total + term
+    return total
+
+
 def general_alternating(x, zb, G, T, q, trace=False):
     """General alternating update (Algorithm 3) on transformed groups x.
 
@@ -415,8 +438,7 @@ def general_alternating(x, zb, G, T, q, trace=False):
         Ct = C.transpose(0, 2, 1)
         CtC = Ct @ C
         Cty = (Ct @ (x64 - zb.astype(F64)[:, None])[..., None])[..., 0]
-        det = np.rint(np.linalg.det(CtC))                    # integer matrix
-        ok = det != 0
+        ok = _int_det(np.rint(CtC)) != 0                     # exact integer test
         if ok.any():
             inv = np.linalg.inv(CtC[ok])
             alpha[ok] = (inv @ Cty[ok][..., None])[..., 0].astype(F32)

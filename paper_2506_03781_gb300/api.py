@@ -1,0 +1,298 @@
+"""ctypes binding of the C ABI declared in ``include/uq_api.h``.
+
+Same entry-point names as the C library; the only work done here is
+argument marshalling (tensor -> device pointer, shape/dtype/device checks so
+that no call can hand the kernels a buffer of the wrong size).  Every step of
+the quantizer runs in the CUDA library: if ``_build/libuq.so`` is missing,
+the first call raises -- there is no other implementation to fall back to.
+
+Tensors are ``torch`` tensors on a CUDA device, contiguous, with the layouts
+of the header: W [out, in] fp32 or bf16; s [out, in]; sr [out];
+delta, zu, zb [out, in/g]; alpha [out, in/g, q]; codes [out, in] uint8.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from .build import LIB
+
+UQ_OK, UQ_ERR_ARG, UQ_ERR_UNSUPPORTED, UQ_ERR_ALIGN, UQ_ERR_CUDA = range(5)
+W_F32, W_BF16 = 0, 1
+CLIP_FIXED_MIN, CLIP_FIXED_MAX, CLIP_BALANCED = 0, 1, 2
+MAP_FULL, MAP_LOCAL_PERIODIC = 0, 1
+EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
+
+PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
+GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
+ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq",
+                "uq_last_error", "uq_abi_version")
+
+
+class UQError(RuntimeError):
+    """A C entry point returned a non-OK status."""
+
+    def __init__(self, status: int, message: str):
+        super().__init__(f"uq status {status}: {message}")
+        self.status = status
+
+
+class uq_params(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in PARAM_NAMES]
+
+
+class uq_grads(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in GRAD_NAMES]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded C library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB):
+            raise RuntimeError(f"{LIB} is missing: build it with `python -m paper_2506_03781_gb300.build` "
+                               "(or __graft_entry__.build()); there is no fallback implementation")
+        L = ctypes.CDLL(LIB)
+        i64, i32, vp = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p
+        L.uq_init_params.argtypes = [vp, i32, i64, i64, i32, i32, i32, i32, i32, uq_params, vp, vp]
+        L.uq_quantize_fwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, i64, i32, vp, vp]
+        L.uq_quantize_bwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, vp]
+        L.uq_export_bcq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
+        for name in ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq"):
+            getattr(L, name).restype = ctypes.c_int
+        L.uq_last_error.argtypes = []
+        L.uq_last_error.restype = ctypes.c_char_p
+        L.uq_abi_version.argtypes = []
+        L.uq_abi_version.restype = ctypes.c_int
+        _lib = L
+    return _lib
+
+
+def uq_last_error() -> str:
+    return lib().uq_last_error().decode()
+
+
+def uq_abi_version() -> int:
+    return lib().uq_abi_version()
+
+
+# ---------------------------------------------------------------------------
+# marshalling helpers
+# ---------------------------------------------------------------------------
+
+def _check(t, name, shape, dtype, device):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.device.type != "cuda" or (device is not None and t.device != device):
+        raise ValueError(f"{name} must be on {device or 'a CUDA device'} (got {t.device})")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _wdtype(W):
+    if W.dtype == torch.float32:
+        return W_F32
+    if W.dtype == torch.bfloat16:
+        return W_BF16
+    raise ValueError(f"W must be float32 or bfloat16 (got {W.dtype})")
+
+
+def _stream(stream, device):
+    if stream is None:
+        return torch.cuda.current_stream(device).cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _params(p, out, n_in, q, g, device, need=PARAM_NAMES):
+    Gr = n_in // g
+    shapes = {"delta": (out, Gr), "zu": (out, Gr), "s": (out, n_in), "sr": (out,),
+              "alpha": (out, Gr, q), "zb": (out, Gr)}
+    ptrs = {}
+    for n in PARAM_NAMES:
+        if n in need:
+            ptrs[n] = _check(p[n], f"params['{n}']", shapes[n], torch.float32, device)
+        else:
+            t = p.get(n) if p is not None else None
+            ptrs[n] = _check(t, f"params['{n}']", shapes[n], torch.float32, device) if t is not None else None
+    return uq_params(**ptrs)
+
+
+def _raise(status):
+    if status != UQ_OK:
+        raise UQError(status, uq_last_error())
+
+
+def _dims(W, g):
+    if W.dim() != 2:
+        raise ValueError("W must be 2-D [out, in]")
+    out, n_in = W.shape
+    if g <= 0 or n_in % g:
+        # let the library produce the error message for bad g
+        return out, n_in
+    return out, n_in
+
+
+# ---------------------------------------------------------------------------
+# entry points
+# ---------------------------------------------------------------------------
+
+def uq_init_params(W, q, g, params, codes, G=30, T=15, clip=CLIP_FIXED_MIN, stream=None):
+    """Unified initialization (Algorithm 2); writes every tensor of ``params`` and ``codes``."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    st = lib().uq_init_params(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, G, T, clip,
+        _params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_quantize_fwd(W, q, g, params, codes, W_hat, map_mode=MAP_LOCAL_PERIODIC, step=0, p_period=2,
+                    stream=None, shape=None, wdtype=None):
+    """Quantizer forward Q*_IF (Eq. 3) / Q_IF (Eq. 2) into ``W_hat``; updates ``codes`` on remap steps.
+
+    On a non-remap step of the local mapping W may be None (pass ``shape`` =
+    (out, in) and ``wdtype``)."""
+    if W is not None:
+        out, n_in = _dims(W, g)
+        wd, dev, wptr = _wdtype(W), W.device, W.data_ptr()
+    else:
+        out, n_in = shape
+        wd, dev, wptr = (W_BF16 if wdtype is None else wdtype), codes.device, None
+    keep = map_mode == MAP_LOCAL_PERIODIC and p_period >= 1 and step % p_period != 0
+    need = ("delta", "zu", "alpha", "zb") if keep else PARAM_NAMES
+    st = lib().uq_quantize_fwd(
+        wptr, wd, out, n_in, q, g, _params(params, out, n_in, q, g, dev, need),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev), map_mode, step, p_period,
+        _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_quantize_bwd(W, q, g, params, codes, dL_dWhat, grads, stream=None):
+    """Backward (App. C.1 STE with gradient filtering); overwrites every tensor of ``grads``."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"ddelta": (out, Gr), "dzu": (out, Gr), "ds": (out, n_in), "dsr": (out,),
+              "dalpha": (out, Gr, q), "dzb": (out, Gr)}
+    gp = uq_grads(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev) for n in GRAD_NAMES})
+    st = lib().uq_quantize_bwd(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), gp, _stream(stream, dev))
+    _raise(st)
+
+
+def uq_export_bcq(W, q, g, params, codes, bitplanes, alpha_star, zb_star, mode=EXPORT_REUSE_CODES,
+                  stream=None, shape=None, wdtype=None):
+    """Theorem 1 + bit-plane export; writes ``bitplanes`` [q, out, in/32], ``alpha_star``, ``zb_star``."""
+    if W is not None:
+        out, n_in = _dims(W, g)
+        wd, dev, wptr = _wdtype(W), W.device, W.data_ptr()
+    else:
+        out, n_in = shape if shape is not None else codes.shape
+        wd, dev, wptr = (W_BF16 if wdtype is None else wdtype), codes.device, None
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    cptr = _check(codes, "codes", (out, n_in), torch.uint8, dev) if codes is not None else None
+    st = lib().uq_export_bcq(
+        wptr, wd, out, n_in, q, g, _params(params, out, n_in, q, g, dev, ("delta", "zu", "alpha", "zb")),
+        cptr, mode, _check(bitplanes, "bitplanes", (q, out, n_in // 32), torch.int32, dev),
+        _check(alpha_star, "alpha_star", (out, Gr, q), torch.float32, dev),
+        _check(zb_star, "zb_star", (out, Gr), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+# ---------------------------------------------------------------------------
+# buffer helpers
+# ---------------------------------------------------------------------------
+
+def empty_params(out, n_in, q, g, device="cuda"):
+    Gr = n_in // g
+    f = dict(dtype=torch.float32, device=device)
+    return {"delta": torch.empty(out, Gr, **f), "zu": torch.empty(out, Gr, **f), "s": torch.empty(out, n_in, **f),
+            "sr": torch.empty(out, **f), "alpha": torch.empty(out, Gr, q, **f), "zb": torch.empty(out, Gr, **f)}
+
+
+def empty_grads(out, n_in, q, g, device="cuda"):
+    Gr = n_in // g
+    f = dict(dtype=torch.float32, device=device)
+    return {"ddelta": torch.empty(out, Gr, **f), "dzu": torch.empty(out, Gr, **f),
+            "ds": torch.empty(out, n_in, **f), "dsr": torch.empty(out, **f),
+            "dalpha": torch.empty(out, Gr, q, **f), "dzb": torch.empty(out, Gr, **f)}
+
+
+def weights_tensor(stored, device="cuda"):
+    """Device tensor from a stored numpy weight array (fp32, or uint16 bf16 bits)."""
+    import numpy as np
+    if stored.dtype == np.uint16:
+        return torch.from_numpy(stored.view(np.int16)).to(device).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(stored, np.float32)).to(device)
+
+
+class HostStep:
+    """One quantizer optimisation step on HOST buffers, through the C ABI.
+
+    ``run`` copies the step's inputs (W, the six parameter tensors, the code
+    words and dL/dW^) from host tensors -- pinned, for asynchronous copies --
+    into device buffers owned by this object, runs ``uq_quantize_fwd`` and
+    ``uq_quantize_bwd`` on the device, and copies the results (W^, the new
+    code words and the six gradients) back into host tensors.  All work is
+    queued on ``stream``; ``run`` returns without synchronising.
+    """
+
+    IN_KEYS = ("W",) + PARAM_NAMES + ("codes", "dL_dWhat")
+    OUT_KEYS = ("W_hat", "codes") + GRAD_NAMES
+
+    def __init__(self, out, n_in, q, g, w_dtype=torch.bfloat16, device="cuda", stream=None):
+        self.out, self.n_in, self.q, self.g = out, n_in, q, g
+        self.device = torch.device(device)
+        self.stream = stream or torch.cuda.Stream(self.device)
+        d = self.device
+        self.dev = {"W": torch.empty(out, n_in, dtype=w_dtype, device=d),
+                    "codes": torch.empty(out, n_in, dtype=torch.uint8, device=d),
+                    "dL_dWhat": torch.empty(out, n_in, dtype=torch.float32, device=d),
+                    "W_hat": torch.empty(out, n_in, dtype=torch.float32, device=d)}
+        self.params = empty_params(out, n_in, q, g, d)
+        self.grads = empty_grads(out, n_in, q, g, d)
+
+    def empty_host(self, pinned=True):
+        """Host tensors of the right shapes for ``run``'s inputs and outputs."""
+        mk = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=pinned)
+        ins = {"W": mk(self.dev["W"]), "codes": mk(self.dev["codes"]), "dL_dWhat": mk(self.dev["dL_dWhat"])}
+        ins.update({k: mk(v) for k, v in self.params.items()})
+        outs = {"W_hat": mk(self.dev["W_hat"]), "codes": mk(self.dev["codes"])}
+        outs.update({k: mk(v) for k, v in self.grads.items()})
+        return ins, outs
+
+    def bytes_in(self, host_in):
+        return sum(host_in[k].numel() * host_in[k].element_size() for k in self.IN_KEYS)
+
+    def bytes_out(self, host_out):
+        return sum(host_out[k].numel() * host_out[k].element_size() for k in self.OUT_KEYS)
+
+    def run(self, host_in, host_out, step, p_period=2, map_mode=MAP_LOCAL_PERIODIC):
+        dev = {**self.dev, **self.params}
+        with torch.cuda.stream(self.stream):
+            for k in self.IN_KEYS:
+                dev[k].copy_(host_in[k], non_blocking=True)
+            uq_quantize_fwd(self.dev["W"], self.q, self.g, self.params, self.dev["codes"], self.dev["W_hat"],
+                            map_mode, step, p_period, stream=self.stream)
+            uq_quantize_bwd(self.dev["W"], self.q, self.g, self.params, self.dev["codes"], self.dev["dL_dWhat"],
+                            self.grads, stream=self.stream)
+            host_out["W_hat"].copy_(self.dev["W_hat"], non_blocking=True)
+            host_out["codes"].copy_(self.dev["codes"], non_blocking=True)
+            for k in GRAD_NAMES:
+                host_out[k].copy_(self.grads[k], non_blocking=True)

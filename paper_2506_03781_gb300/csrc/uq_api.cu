@@ -1,0 +1,155 @@
+// C-ABI front end: argument validation, error reporting, dispatch to the
+// kernel launchers.  Nothing here allocates device memory or keeps a
+// pointer beyond the call.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "uq_launch.h"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+uq_status fail(uq_status st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+uq_status ok() {
+    g_err[0] = '\0';
+    return UQ_OK;
+}
+
+constexpr int64_t kMaxIn = 196608;   // one row's per-warp-step partials fit in shared memory
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Checks shape, q, g, W dtype.  Returns UQ_OK or an error status.
+uq_status check_shape(int64_t out, int64_t in, int q, int g, int wdtype) {
+    if (q < 1 || q > 4) return fail(UQ_ERR_UNSUPPORTED, "q=%d: bit-widths 1..4 are supported", q);
+    if (out < 1 || in < 1) return fail(UQ_ERR_ARG, "empty matrix: out=%lld in=%lld", (long long)out, (long long)in);
+    if (out > 0x7fffffffLL) return fail(UQ_ERR_ARG, "out=%lld exceeds 2^31-1 rows", (long long)out);
+    if (g < 32 || g % 32 != 0) return fail(UQ_ERR_ARG, "g=%d must be a positive multiple of 32", g);
+    if (in % g != 0) return fail(UQ_ERR_ARG, "in=%lld is not a multiple of g=%d", (long long)in, g);
+    if (!(g == 32 || g == 64 || g % 128 == 0))
+        return fail(UQ_ERR_UNSUPPORTED, "g=%d: supported group sizes are 32, 64 and multiples of 128", g);
+    if (in > kMaxIn) return fail(UQ_ERR_UNSUPPORTED, "in=%lld exceeds %lld", (long long)in, (long long)kMaxIn);
+    if (wdtype != UQ_W_F32 && wdtype != UQ_W_BF16) return fail(UQ_ERR_ARG, "unknown weight dtype %d", wdtype);
+    return UQ_OK;
+}
+
+uq_status check_ptr(const void* p, const char* name) {
+    if (p == nullptr) return fail(UQ_ERR_ARG, "%s is NULL", name);
+    if (!aligned16(p)) return fail(UQ_ERR_ALIGN, "%s=%p is not 16-byte aligned", name, p);
+    return UQ_OK;
+}
+
+#define UQ_TRY(expr)                      \
+    do {                                  \
+        uq_status _s = (expr);            \
+        if (_s != UQ_OK) return _s;       \
+    } while (0)
+
+uq_status cuda_status(cudaError_t e, const char* what) {
+    if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+    return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+int uq_abi_version(void) { return 1; }
+
+const char* uq_last_error(void) { return g_err; }
+
+uq_status uq_init_params(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, int G, int T,
+                         uq_clip clip, uq_params p, uint8_t* codes, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (g > 32768) return fail(UQ_ERR_UNSUPPORTED, "initialization supports g <= 32768 (g=%d)", g);
+    if (G < 1) return fail(UQ_ERR_ARG, "G=%d must be >= 1", G);
+    if (T < 0) return fail(UQ_ERR_ARG, "T=%d must be >= 0", T);
+    if (clip != UQ_CLIP_FIXED_MIN && clip != UQ_CLIP_FIXED_MAX && clip != UQ_CLIP_BALANCED)
+        return fail(UQ_ERR_ARG, "unknown clipping strategy %d", (int)clip);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.s, "params.s"));
+    UQ_TRY(check_ptr(p.sr, "params.sr"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_init(sh, W, G, T, (int)clip, p, codes, (cudaStream_t)stream), "uq_init_params");
+}
+
+uq_status uq_quantize_fwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                          uint8_t* codes, uq_map map, int64_t step, int p_period, float* W_hat, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (map != UQ_MAP_FULL && map != UQ_MAP_LOCAL_PERIODIC) return fail(UQ_ERR_ARG, "unknown mapping %d", (int)map);
+    if (p_period < 1) return fail(UQ_ERR_ARG, "p_period=%d must be >= 1", p_period);
+    if (step < 0) return fail(UQ_ERR_ARG, "step=%lld must be >= 0", (long long)step);
+    const int mode = map == UQ_MAP_FULL ? uq::FWD_FULL : (step % p_period == 0 ? uq::FWD_REMAP : uq::FWD_KEEP);
+    if (mode != uq::FWD_KEEP) {
+        UQ_TRY(check_ptr(W, "W"));
+        UQ_TRY(check_ptr(p.s, "params.s"));
+        UQ_TRY(check_ptr(p.sr, "params.sr"));
+    }
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(W_hat, "W_hat"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_fwd(sh, W, p, codes, mode, W_hat, (cudaStream_t)stream), "uq_quantize_fwd");
+}
+
+uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                          const uint8_t* codes, const float* dL_dWhat, uq_grads gr, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.s, "params.s"));
+    UQ_TRY(check_ptr(p.sr, "params.sr"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(gr.ddelta, "grads.ddelta"));
+    UQ_TRY(check_ptr(gr.dzu, "grads.dzu"));
+    UQ_TRY(check_ptr(gr.ds, "grads.ds"));
+    UQ_TRY(check_ptr(gr.dsr, "grads.dsr"));
+    UQ_TRY(check_ptr(gr.dalpha, "grads.dalpha"));
+    UQ_TRY(check_ptr(gr.dzb, "grads.dzb"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_bwd(sh, W, p, codes, dL_dWhat, gr, (cudaStream_t)stream), "uq_quantize_bwd");
+}
+
+uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                        const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes, float* alpha_star,
+                        float* zb_star, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (mode != UQ_EXPORT_REUSE_CODES && mode != UQ_EXPORT_REMAP_EQ4)
+        return fail(UQ_ERR_ARG, "unknown export mode %d", (int)mode);
+    if (mode == UQ_EXPORT_REMAP_EQ4) UQ_TRY(check_ptr(W, "W"));
+    else UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(bitplanes, "bitplanes"));
+    UQ_TRY(check_ptr(alpha_star, "alpha_star"));
+    UQ_TRY(check_ptr(zb_star, "zb_star"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_export(sh, W, p, codes, (int)mode, bitplanes, alpha_star, zb_star,
+                                         (cudaStream_t)stream),
+                       "uq_export_bcq");
+}
+
+}  // extern "C"

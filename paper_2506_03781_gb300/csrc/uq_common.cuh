@@ -1,0 +1,204 @@
+// Device helpers shared by the UniQuan_F kernels (sm_103a).
+//
+// Work decomposition used by the per-step kernels (forward, backward,
+// export): one thread block per weight-matrix row, 8 warps; the row is cut
+// into "warp-steps" of 128 consecutive elements, each lane owning 4
+// consecutive elements (one 16-byte fp32 vector).  Since g is 32, 64 or a
+// multiple of 128, a warp-step holds GPS = 4, 2 or 1 groups (or a 128-wide
+// slice of one group), each group on a contiguous run of 32/GPS lanes.
+// Every value that decides an integer is computed with explicitly rounded
+// intrinsics (__fadd_rn, __fmul_rn, __fdiv_rn): no FMA contraction, IEEE
+// division, the operation order written in uq_api.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/uq_api.h"
+
+namespace uq {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kVec = 4;                     // elements per lane per warp-step
+constexpr int kStep = 32 * kVec;            // 128 elements per warp-step
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kSlots = 4;                   // group tables per warp and batch
+
+// Weight-storage adaptors: 4 consecutive weights per lane.
+struct WF32 {
+    using raw = float4;
+    static __device__ __forceinline__ raw load(const void* base, int64_t i) {
+        return __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(base) + i));
+    }
+    static __device__ __forceinline__ void unpack(const raw& r, float v[4]) {
+        v[0] = r.x; v[1] = r.y; v[2] = r.z; v[3] = r.w;
+    }
+};
+
+struct WBF16 {
+    using raw = uint2;   // 4 x bf16, element k in bits [16k, 16k+16) (little endian)
+    static __device__ __forceinline__ raw load(const void* base, int64_t i) {
+        return __ldg(reinterpret_cast<const uint2*>(static_cast<const uint16_t*>(base) + i));
+    }
+    static __device__ __forceinline__ void unpack(const raw& r, float v[4]) {
+        v[0] = __uint_as_float(r.x << 16);
+        v[1] = __uint_as_float(r.x & 0xffff0000u);
+        v[2] = __uint_as_float(r.y << 16);
+        v[3] = __uint_as_float(r.y & 0xffff0000u);
+    }
+};
+
+__device__ __forceinline__ float4 ldg4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+__device__ __forceinline__ void f4_to(const float4& r, float v[4]) { v[0] = r.x; v[1] = r.y; v[2] = r.z; v[3] = r.w; }
+
+// T_F (Eq. 1): den = (Delta * s) * s_r; u = w / den; x = u + z_U.
+__device__ __forceinline__ float transform_x(float w, float s, float delta, float sr, float zu, float& u) {
+    const float den = __fmul_rn(__fmul_rn(delta, s), sr);
+    u = __fdiv_rn(w, den);
+    return __fadd_rn(u, zu);
+}
+
+// BCQ level of code word c (Sec. 2.3): ((c_1 a_1 + c_2 a_2) + ... ) + z_B.
+template <int Q>
+__device__ __forceinline__ float level_of(int c, const float a[Q], float zb) {
+    float acc = (c & 1) ? a[0] : -a[0];
+#pragma unroll
+    for (int j = 1; j < Q; ++j) acc = __fadd_rn(acc, ((c >> j) & 1) ? a[j] : -a[j]);
+    return __fadd_rn(acc, zb);
+}
+
+// Per-warp group tables: levels by code word, sorted levels, code of each
+// rank, rank of each code, and for the local mapping the (lower, own, upper)
+// neighbour levels with the neighbours' code words packed in .w.
+template <int Q>
+struct GroupTables {
+    static constexpr int L = 1 << Q;
+    float lv[kSlots][L];
+    float srt[kSlots][L];
+    float4 nb[kSlots][L];
+    float tau[kSlots];
+    uint8_t cor[kSlots][L];
+    uint8_t rk[kSlots][L];
+};
+
+// Builds the tables of up to kSlots groups (slot k -> group grp_of_slot(k),
+// valid if ok_of_slot(k)).  Whole warp; ends with __syncwarp().
+// Levels come from (alpha, z_B) by level_of; the rank of code c is the
+// number of codes whose level is smaller, or equal with a smaller code word
+// (the stable ascending order).
+template <int Q, bool NEED_SORT, bool NEED_NB, typename GrpFn, typename OkFn>
+__device__ __forceinline__ void build_tables(GroupTables<Q>& t, int lane, const float* __restrict__ alpha,
+                                             const float* __restrict__ zb, GrpFn grp_of_slot, OkFn ok_of_slot) {
+    constexpr int L = 1 << Q;
+    constexpr int E = kSlots * L;
+#pragma unroll
+    for (int e = lane; e < E; e += 32) {
+        const int k = e / L, c = e % L;
+        float lvv = 0.f;
+        if (ok_of_slot(k)) {
+            const int64_t grp = grp_of_slot(k);
+            float a[Q];
+#pragma unroll
+            for (int j = 0; j < Q; ++j) a[j] = __ldg(alpha + grp * Q + j);
+            lvv = level_of<Q>(c, a, __ldg(zb + grp));
+            if (c == 0) {
+                float m = fabsf(a[0]);
+#pragma unroll
+                for (int j = 1; j < Q; ++j) m = fminf(m, fabsf(a[j]));
+                t.tau[k] = m;
+            }
+        } else if (c == 0) {
+            t.tau[k] = 0.f;
+        }
+        t.lv[k][c] = lvv;
+    }
+    __syncwarp();
+    if constexpr (NEED_SORT) {
+#pragma unroll
+        for (int e = lane; e < E; e += 32) {
+            const int k = e / L, c = e % L;
+            const float v = t.lv[k][c];
+            int r = 0;
+#pragma unroll
+            for (int c2 = 0; c2 < L; ++c2) {
+                const float v2 = t.lv[k][c2];
+                r += (v2 < v) || (v2 == v && c2 < c);
+            }
+            t.srt[k][r] = v;
+            t.cor[k][r] = static_cast<uint8_t>(c);
+            t.rk[k][c] = static_cast<uint8_t>(r);
+        }
+        __syncwarp();
+    }
+    if constexpr (NEED_NB) {
+#pragma unroll
+        for (int e = lane; e < E; e += 32) {
+            const int k = e / L, c = e % L;
+            const int r = t.rk[k][c];
+            const int rl = r > 0 ? r - 1 : 0;
+            const int rh = r < L - 1 ? r + 1 : L - 1;
+            const uint32_t packed = uint32_t(t.cor[k][rl]) | (uint32_t(t.cor[k][rh]) << 8);
+            t.nb[k][c] = make_float4(t.srt[k][rl], t.lv[k][c], t.srt[k][rh], __uint_as_float(packed));
+        }
+        __syncwarp();
+    }
+}
+
+// Full mapping M_B over the sorted levels held in registers: argmin over
+// ranks of |x - l|, first (lowest) rank wins ties.  Returns the rank; m is
+// the chosen level.
+template <int L>
+__device__ __forceinline__ int nearest_rank(float x, const float srt[L], float& m) {
+    float best = fabsf(__fsub_rn(x, srt[0]));
+    int br = 0;
+    m = srt[0];
+#pragma unroll
+    for (int r = 1; r < L; ++r) {
+        const float d = fabsf(__fsub_rn(x, srt[r]));
+        if (d < best) { best = d; br = r; m = srt[r]; }
+    }
+    return br;
+}
+
+// Segmented reduce-scatter of 8 partial sums over SEGL consecutive lanes
+// (SEGL = 8, 16 or 32).  Three butterfly levels halve the number of live
+// values (8 -> 4 -> 2 -> 1) while exchanging the other half with the
+// partner lane; the remaining levels sum the single value.  On return the
+// lane holds the segment-wide total of slot `slot`; lanes whose index is a
+// multiple of SEGL/8 hold distinct slots 0..7.  Fixed order: deterministic.
+template <int SEGL>
+__device__ __forceinline__ float seg_reduce8(float v[8], int lane, int& slot) {
+    int base = 0;
+#pragma unroll
+    for (int lvl = 0; lvl < 3; ++lvl) {
+        const int off = SEGL >> (lvl + 1);
+        const int h = 4 >> lvl;
+        const bool up = (lane & off) != 0;
+#pragma unroll
+        for (int i = 0; i < h; ++i) {
+            const float send = up ? v[i] : v[i + h];
+            const float keep = up ? v[i + h] : v[i];
+            v[i] = keep + __shfl_xor_sync(kFull, send, off);
+        }
+        base += up ? h : 0;
+    }
+#pragma unroll
+    for (int off = SEGL >> 4; off >= 1; off >>= 1) v[0] += __shfl_xor_sync(kFull, v[0], off);
+    slot = base;
+    return v[0];
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+    return v;
+}
+
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+    return v;
+}
+
+}  // namespace uq

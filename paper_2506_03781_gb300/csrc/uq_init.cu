@@ -1,0 +1,329 @@
+// Unified initialization (Algorithm 2) with the clipping strategies of
+// App. E.2 and the general alternating update of Algorithm 3: one warp per
+// group, the group's transformed weights x and code words kept in shared
+// memory.  Runs once before training; not on the per-step path.
+//
+// Sums that feed alpha and z_B are taken in fp64 (the group's fp32 values
+// are summed exactly in practice); the normal equations C^T C alpha =
+// C^T (x - z_B) have an integer matrix, so singularity is decided exactly
+// by an integer determinant and the system is solved in fp64 by Gaussian
+// elimination with partial pivoting.
+#include "uq_common.cuh"
+#include "uq_launch.h"
+
+namespace uq {
+
+constexpr int kInitMaxWarps = 8;
+
+template <int Q>
+struct InitTab {
+    static constexpr int L = 1 << Q;
+    float lv[L];
+    float srt[L];
+    uint8_t cor[L];
+};
+
+// Sorted levels of (a, zb) into registers of every lane (via the warp's table).
+template <int Q>
+__device__ __forceinline__ void sorted_levels(InitTab<Q>& tb, int lane, const float a[Q], float zb,
+                                              float srt[1 << Q]) {
+    constexpr int L = 1 << Q;
+    __syncwarp();
+    if (lane < L) tb.lv[lane] = level_of<Q>(lane, a, zb);
+    __syncwarp();
+    if (lane < L) {
+        const float v = tb.lv[lane];
+        int r = 0;
+#pragma unroll
+        for (int c2 = 0; c2 < L; ++c2) {
+            const float v2 = tb.lv[c2];
+            r += (v2 < v) || (v2 == v && c2 < lane);
+        }
+        tb.srt[r] = v;
+        tb.cor[r] = static_cast<uint8_t>(lane);
+    }
+    __syncwarp();
+#pragma unroll
+    for (int r = 0; r < L; ++r) srt[r] = tb.srt[r];
+}
+
+// Exact singularity test of the integer matrix C^T C.  C^T C is a Gram
+// matrix of +-1 columns, so |det| <= g^q <= 2^60 (Hadamard); the cofactor
+// expansion below is evaluated with wrapping 64-bit unsigned arithmetic,
+// which is exact modulo 2^64 and hence exact.
+template <int Q>
+__device__ __forceinline__ bool int_singular(const long long Min[Q][Q]) {
+    using u64 = unsigned long long;
+    u64 M[Q][Q];
+#pragma unroll
+    for (int i = 0; i < Q; ++i)
+#pragma unroll
+        for (int j = 0; j < Q; ++j) M[i][j] = (u64)Min[i][j];
+    auto det3 = [&](int r0, int r1, int r2, int c0, int c1, int c2) -> u64 {
+        return M[r0][c0] * (M[r1][c1] * M[r2][c2] - M[r1][c2] * M[r2][c1])
+             - M[r0][c1] * (M[r1][c0] * M[r2][c2] - M[r1][c2] * M[r2][c0])
+             + M[r0][c2] * (M[r1][c0] * M[r2][c1] - M[r1][c1] * M[r2][c0]);
+    };
+    u64 det;
+    if constexpr (Q == 1) {
+        det = M[0][0];
+    } else if constexpr (Q == 2) {
+        det = M[0][0] * M[1][1] - M[0][1] * M[1][0];
+    } else if constexpr (Q == 3) {
+        det = det3(0, 1, 2, 0, 1, 2);
+    } else {
+        det = M[0][0] * det3(1, 2, 3, 1, 2, 3) - M[0][1] * det3(1, 2, 3, 0, 2, 3)
+            + M[0][2] * det3(1, 2, 3, 0, 1, 3) - M[0][3] * det3(1, 2, 3, 0, 1, 2);
+    }
+    return det == 0ull;
+}
+
+// Solves A x = b in fp64 (Gaussian elimination, partial pivoting).
+template <int Q>
+__device__ __forceinline__ void solve_fp64(const long long Ain[Q][Q], const double bin[Q], double x[Q]) {
+    double A[Q][Q], b[Q];
+#pragma unroll
+    for (int i = 0; i < Q; ++i) {
+        b[i] = bin[i];
+#pragma unroll
+        for (int j = 0; j < Q; ++j) A[i][j] = (double)Ain[i][j];
+    }
+    for (int k = 0; k < Q; ++k) {
+        int p = k;
+        for (int i = k + 1; i < Q; ++i)
+            if (fabs(A[i][k]) > fabs(A[p][k])) p = i;
+        if (p != k) {
+            for (int j = 0; j < Q; ++j) { const double tmp = A[k][j]; A[k][j] = A[p][j]; A[p][j] = tmp; }
+            const double tb = b[k]; b[k] = b[p]; b[p] = tb;
+        }
+        for (int i = k + 1; i < Q; ++i) {
+            const double f = A[i][k] / A[k][k];
+            for (int j = k; j < Q; ++j) A[i][j] -= f * A[k][j];
+            b[i] -= f * b[k];
+        }
+    }
+    for (int i = Q - 1; i >= 0; --i) {
+        double s = b[i];
+        for (int j = i + 1; j < Q; ++j) s -= A[i][j] * x[j];
+        x[i] = s / A[i][i];
+    }
+}
+
+template <int Q, typename WT>
+__global__ void init_kernel(const void* __restrict__ W, int64_t n_groups, int n_in, int g, int G, int T, int clip,
+                            float* __restrict__ DELTA, float* __restrict__ ZU, float* __restrict__ S,
+                            float* __restrict__ SR, float* __restrict__ ALPHA, float* __restrict__ ZB,
+                            uint8_t* __restrict__ CODES) {
+    constexpr int L = 1 << Q;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wpc = blockDim.x >> 5;
+    __shared__ InitTab<Q> tabs[kInitMaxWarps];
+    InitTab<Q>& tb = tabs[warp];
+    float* xs = reinterpret_cast<float*>(smem) + (size_t)warp * g;
+    uint8_t* cs = smem + (size_t)wpc * g * sizeof(float) + (size_t)warp * g;
+
+    const int64_t grp = (int64_t)blockIdx.x * wpc + warp;
+    if (grp >= n_groups) return;                       // whole warp; no block barrier follows
+    const int Gr = n_in / g;
+    const int64_t row = grp / Gr;
+    const int64_t eoff = row * (int64_t)n_in + (grp % Gr) * (int64_t)g;
+    auto wval = [&](int i) -> float {
+        if constexpr (sizeof(typename WT::raw) == sizeof(float4))
+            return __ldg(static_cast<const float*>(W) + eoff + i);
+        else
+            return __uint_as_float(uint32_t(__ldg(static_cast<const unsigned short*>(W) + eoff + i)) << 16);
+    };
+
+    float wmin = INFINITY, wmax = -INFINITY;
+    for (int i = lane; i < g; i += 32) {
+        const float w = wval(i);
+        wmin = fminf(wmin, w);
+        wmax = fmaxf(wmax, w);
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+        wmin = fminf(wmin, __shfl_xor_sync(kFull, wmin, off));
+        wmax = fmaxf(wmax, __shfl_xor_sync(kFull, wmax, off));
+    }
+    const float top = (float)(L - 1);
+    const float rng = fmaxf(__fsub_rn(wmax, wmin), 1e-12f);
+
+    double e_best = INFINITY;
+    float bd = 0.f, bz = 0.f, bzb = top * 0.5f, ba[Q];
+#pragma unroll
+    for (int j = 0; j < Q; ++j) ba[j] = 0.f;
+
+    for (int gi = 1; gi <= G; ++gi) {
+        const float gamma = __fdiv_rn((float)gi, (float)G);
+        const float dc = __fdiv_rn(__fmul_rn(gamma, rng), top);
+        float zc;
+        if (clip == UQ_CLIP_FIXED_MIN) zc = __fdiv_rn(-wmin, dc);
+        else if (clip == UQ_CLIP_FIXED_MAX) zc = __fsub_rn(top, __fdiv_rn(wmax, dc));
+        else zc = __fdiv_rn(-__fmul_rn(gamma, wmin), dc);
+        __syncwarp();
+        for (int i = lane; i < g; i += 32) {
+            float u;
+            xs[i] = transform_x(wval(i), 1.f, dc, 1.f, zc, u);
+            cs[i] = 0;
+        }
+        __syncwarp();
+
+        // --- Algorithm 3: greedy start (one bit at a time) ---
+        float a[Q], zb = bzb;
+#pragma unroll
+        for (int j = 0; j < Q; ++j) {
+            double sabs = 0.0;
+            for (int i = lane; i < g; i += 32) {
+                float r = __fsub_rn(xs[i], zb);
+                const int c = cs[i];
+#pragma unroll
+                for (int jj = 0; jj < j; ++jj) r = __fsub_rn(r, ((c >> jj) & 1) ? a[jj] : -a[jj]);
+                sabs += (double)fabsf(r);
+                if (r >= 0.f) cs[i] = (uint8_t)(c | (1 << j));
+            }
+            sabs = warp_sum_d(sabs);
+            a[j] = (float)(sabs / (double)g);
+        }
+        __syncwarp();
+
+        // --- T rounds of alpha, C (and z_B when G == 1) ---
+        for (int it = 0; it < T; ++it) {
+            long long ctc[Q][Q];
+            double cty[Q];
+#pragma unroll
+            for (int j = 0; j < Q; ++j) {
+                cty[j] = 0.0;
+#pragma unroll
+                for (int k = 0; k < Q; ++k) ctc[j][k] = 0;
+            }
+            const double zbd = (double)zb;
+            for (int i = lane; i < g; i += 32) {
+                const int c = cs[i];
+                const double y = (double)xs[i] - zbd;
+#pragma unroll
+                for (int j = 0; j < Q; ++j) {
+                    const int sj = ((c >> j) & 1) ? 1 : -1;
+                    cty[j] += sj > 0 ? y : -y;
+#pragma unroll
+                    for (int k = j; k < Q; ++k) ctc[j][k] += (((c >> k) & 1) ? 1 : -1) * sj;
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < Q; ++j) {
+                cty[j] = warp_sum_d(cty[j]);
+#pragma unroll
+                for (int k = j; k < Q; ++k) {
+                    long long v = ctc[j][k];
+#pragma unroll
+                    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+                    ctc[j][k] = v;
+                    ctc[k][j] = v;
+                }
+            }
+            if (!int_singular<Q>(ctc)) {
+                double sol[Q];
+                solve_fp64<Q>(ctc, cty, sol);
+#pragma unroll
+                for (int j = 0; j < Q; ++j) a[j] = (float)sol[j];
+            }
+            float srt[L];
+            sorted_levels<Q>(tb, lane, a, zb, srt);
+            for (int i = lane; i < g; i += 32) {
+                float m;
+                const int r = nearest_rank<L>(xs[i], srt, m);
+                cs[i] = tb.cor[r];
+            }
+            __syncwarp();
+            if (G == 1) {
+                double sres = 0.0;
+                for (int i = lane; i < g; i += 32) {
+                    const int c = cs[i];
+                    double ca = 0.0;
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) ca += ((c >> j) & 1) ? (double)a[j] : -(double)a[j];
+                    sres += (double)xs[i] - ca;
+                }
+                sres = warp_sum_d(sres);
+                zb = (float)(sres / (double)g);
+            }
+        }
+
+        // --- candidate error with the full mapping (Eq. 2), s = s_r = 1 ---
+        float srt[L];
+        sorted_levels<Q>(tb, lane, a, zb, srt);
+        double e = 0.0;
+        for (int i = lane; i < g; i += 32) {
+            float m;
+            nearest_rank<L>(xs[i], srt, m);
+            const float what = __fmul_rn(dc, __fsub_rn(m, zc));
+            const double df = (double)wval(i) - (double)what;
+            e += df * df;
+        }
+        e = warp_sum_d(e);
+        if (e < e_best) {
+            e_best = e;
+            bd = dc;
+            bz = zc;
+            bzb = zb;
+#pragma unroll
+            for (int j = 0; j < Q; ++j) ba[j] = a[j];
+        }
+    }
+
+    if (lane == 0) {
+        DELTA[grp] = bd;
+        ZU[grp] = bz;
+        ZB[grp] = bzb;
+#pragma unroll
+        for (int j = 0; j < Q; ++j) ALPHA[grp * Q + j] = ba[j];
+        if (grp % Gr == 0) SR[row] = 1.f;
+    }
+    float srt[L];
+    sorted_levels<Q>(tb, lane, ba, bzb, srt);
+    for (int i = lane; i < g; i += 32) {
+        float u, m;
+        const float x = transform_x(wval(i), 1.f, bd, 1.f, bz, u);
+        const int r = nearest_rank<L>(x, srt, m);
+        CODES[eoff + i] = tb.cor[r];
+        S[eoff + i] = 1.f;
+    }
+}
+
+template <int Q, typename WT>
+static cudaError_t run_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
+                            cudaStream_t st) {
+    const int64_t n_groups = sh.out * (int64_t)(sh.n_in / sh.g);
+    const size_t per_warp = (size_t)sh.g * (sizeof(float) + 1);
+    int wpc = (int)((96 * 1024) / per_warp);
+    wpc = wpc < 1 ? 1 : (wpc > kInitMaxWarps ? kInitMaxWarps : wpc);
+    const size_t dyn = per_warp * wpc;
+    auto kern = init_kernel<Q, WT>;
+    if (dyn > 32 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t blocks = (n_groups + wpc - 1) / wpc;
+    kern<<<dim3((unsigned)blocks), wpc * 32, dyn, st>>>(W, n_groups, sh.n_in, sh.g, G, T, clip, p.delta, p.zu,
+                                                          p.s, p.sr, p.alpha, p.zb, codes);
+    return cudaGetLastError();
+}
+
+template <int Q>
+static cudaError_t init_w(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
+                          cudaStream_t st) {
+    if (sh.wdtype == UQ_W_BF16) return run_init<Q, WBF16>(sh, W, G, T, clip, p, codes, st);
+    return run_init<Q, WF32>(sh, W, G, T, clip, p, codes, st);
+}
+
+cudaError_t launch_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
+                        cudaStream_t st) {
+    switch (sh.q) {
+        case 1: return init_w<1>(sh, W, G, T, clip, p, codes, st);
+        case 2: return init_w<2>(sh, W, G, T, clip, p, codes, st);
+        case 3: return init_w<3>(sh, W, G, T, clip, p, codes, st);
+        default: return init_w<4>(sh, W, G, T, clip, p, codes, st);
+    }
+}
+
+}  // namespace uq

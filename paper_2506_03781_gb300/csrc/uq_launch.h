@@ -1,0 +1,34 @@
+// Internal interface between the C-ABI front end (uq_api.cu, which validates
+// arguments) and the kernel translation units (which pick a template
+// instantiation and launch).  Each launcher returns the cudaError_t of its
+// launch.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/uq_api.h"
+
+namespace uq {
+
+struct Shape {
+    int64_t out;
+    int n_in;
+    int q;
+    int g;
+    int wdtype;     // uq_wdtype
+};
+
+cudaError_t launch_fwd(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                       float* what, cudaStream_t st);
+cudaError_t launch_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
+                       uq_grads gr, cudaStream_t st);
+cudaError_t launch_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
+                          uint32_t* planes, float* astar, float* zstar, cudaStream_t st);
+cudaError_t launch_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
+                        cudaStream_t st);
+
+// Forward modes (see uq_api.h): full mapping, local remap step, keep codes.
+enum { FWD_FULL = 0, FWD_REMAP = 1, FWD_KEEP = 2 };
+
+}  // namespace uq

@@ -1,0 +1,34 @@
+"""Algorithmic HBM bytes of each kernel launch: what the method must move.
+
+Per element: weights (2 B bf16 / 4 B fp32), s (4 B), code word (1 B),
+w^ / dL/dw^ / ds (4 B each).  Per group: the parameters Delta, z_U, z_B and
+alpha_1..q ((3 + q) * 4 B) read once, and the same number of gradient
+values written by the backward.  Per row: s_r (4 B) read, ds_r written.
+"""
+
+from __future__ import annotations
+
+
+def bytes_per_launch(kind: str, out: int, n_in: int, q: int, g: int, wbytes: int) -> int:
+    n = out * n_in
+    groups = out * (n_in // g)
+    gp = groups * (3 + q) * 4
+    if kind == "fwd_remap":        # read W, s, codes; write w^, codes
+        return n * (wbytes + 4 + 1 + 4 + 1) + gp + out * 4
+    if kind == "fwd_keep":         # read codes; write w^
+        return n * (1 + 4) + gp
+    if kind == "fwd_full":         # read W, s; write w^, codes
+        return n * (wbytes + 4 + 4 + 1) + gp + out * 4
+    if kind == "bwd":              # read W, s, codes, dL/dw^; write ds; group/row grads
+        return n * (wbytes + 4 + 1 + 4 + 4) + 2 * gp + 2 * out * 4
+    if kind == "export_reuse":     # read codes; write planes, alpha*, z*
+        return n * 1 + q * n // 8 + gp + groups * (q + 1) * 4
+    if kind == "export_eq4":       # read W; write planes, alpha*, z*
+        return n * wbytes + q * n // 8 + gp + groups * (q + 1) * 4
+    raise ValueError(kind)
+
+
+def step_bytes(out: int, n_in: int, q: int, g: int, wbytes: int, remap: bool) -> int:
+    """One optimisation step of the quantizer: forward (remap or keep) + backward."""
+    return (bytes_per_launch("fwd_remap" if remap else "fwd_keep", out, n_in, q, g, wbytes)
+            + bytes_per_launch("bwd", out, n_in, q, g, wbytes))

@@ -1,0 +1,113 @@
+"""Helpers for the GPU parity tests: run the CUDA library through the C ABI
+and the CPU oracle on identical seeded inputs, and compare.
+
+Comparison rules (derived from the arithmetic; see the design notes):
+* codes and bit-planes: bit-exact (both sides take every decision in fp32
+  with the same operations and the same tie rules);
+* w^ and alpha*, z_B*: bit-exact where the codes agree (same fp32 ops);
+  the stated bound is 1e-6 relative to max(|ref|, Delta max|alpha|);
+* gradient sums: |gpu - oracle| <= 1e-4 * (sum of |terms|), the L1 mass of
+  the reduction (fp32 accumulation error is at most ~n u times that mass);
+* ds: |gpu - oracle| <= 1e-4 * max(|oracle|, 1e-6 max|ds|).
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+from paper_2506_03781_gb300 import api, synth
+
+F32 = np.float32
+PKEYS = ("delta", "zu", "s", "sr", "alpha", "zb")
+GTOL = 1e-4
+
+
+def dev():
+    return torch.device("cuda:0")
+
+
+def to_dev(P, d=None):
+    d = d or dev()
+    return {k: torch.from_numpy(np.ascontiguousarray(P[k], F32)).to(d) for k in PKEYS}
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def make_inputs(out, n_in, q, g, seed, wdtype="bf16", std=0.02, init_G=6, init_T=3, eps=0.01):
+    """Weights, oracle-initialised (then jittered) parameters, codes and dL/dW^."""
+    rng = np.random.default_rng(seed)
+    W32 = (rng.standard_t(4, (out, n_in)) * std / np.sqrt(2)).astype(F32)
+    if wdtype == "bf16":
+        raw, W = synth.bf16_round(W32)
+    else:
+        raw, W = W32, W32
+    init = O.unified_init(W, q, g, G=init_G, T=init_T)
+    fac = synth.perturb_factors(synth.param_shapes(out, n_in, g, q), eps, seed)
+    P = synth.jitter({k: init[k] for k in PKEYS}, fac)
+    Gup = synth.upstream_grad(out, n_in, 1e-4, seed)
+    return raw, W, P, init["codes"], Gup
+
+
+def gpu_fwd(raw, P, codes, q, g, mode, step, p, stream=None):
+    out, n_in = raw.shape
+    Wd = api.weights_tensor(raw, dev())
+    pd = to_dev(P)
+    cd = torch.from_numpy(np.ascontiguousarray(codes)).to(dev()) if codes is not None else \
+        torch.zeros(out, n_in, dtype=torch.uint8, device=dev())
+    what = torch.empty(out, n_in, dtype=torch.float32, device=dev())
+    api.uq_quantize_fwd(Wd, q, g, pd, cd, what, mode, step, p, stream=stream)
+    return host(what), host(cd)
+
+
+def gpu_bwd(raw, P, codes, Gup, q, g):
+    out, n_in = raw.shape
+    Wd = api.weights_tensor(raw, dev())
+    gr = api.empty_grads(out, n_in, q, g, dev())
+    api.uq_quantize_bwd(Wd, q, g, to_dev(P), torch.from_numpy(np.ascontiguousarray(codes)).to(dev()),
+                        torch.from_numpy(np.ascontiguousarray(Gup, F32)).to(dev()), gr)
+    return {k: host(v) for k, v in gr.items()}
+
+
+def gpu_export(raw, P, codes, q, g, mode):
+    out, n_in = raw.shape
+    Wd = api.weights_tensor(raw, dev())
+    planes = torch.full((q, out, n_in // 32), -1, dtype=torch.int32, device=dev())
+    a_s = torch.empty(out, n_in // g, q, dtype=torch.float32, device=dev())
+    z_s = torch.empty(out, n_in // g, dtype=torch.float32, device=dev())
+    cd = torch.from_numpy(np.ascontiguousarray(codes)).to(dev()) if codes is not None else None
+    api.uq_export_bcq(Wd, q, g, to_dev(P), cd, planes, a_s, z_s, mode)
+    return host(planes).view(np.uint32), host(a_s), host(z_s)
+
+
+def assert_fwd_equal(what, codes, r_what, r_codes, label=""):
+    n_code = int((codes != r_codes).sum())
+    assert n_code == 0, f"{label}: {n_code} code mismatches of {codes.size}"
+    n_w = int((what != r_what).sum())
+    assert n_w == 0, f"{label}: {n_w} w_hat mismatches (max abs {np.abs(what - r_what).max()})"
+
+
+def assert_grads_close(gr, ref, mass, label=""):
+    for k in ("ddelta", "dzu", "dzb", "dalpha", "dsr"):
+        err = np.abs(gr[k].astype(np.float64) - ref[k])
+        bad = err > GTOL * mass[k] + 1e-30
+        assert not bad.any(), (f"{label}: {k}: {int(bad.sum())} outside tol; worst ratio "
+                               f"{(err / (mass[k] + 1e-30)).max():.3e}")
+    ds_ref = ref["ds"]
+    floor = 1e-6 * np.abs(ds_ref).max()
+    err = np.abs(gr["ds"].astype(np.float64) - ds_ref)
+    bad = err > GTOL * np.maximum(np.abs(ds_ref), floor)
+    assert not bad.any(), f"{label}: ds: {int(bad.sum())} outside tol"
+
+
+def oracle_bwd(W, P, codes, Gup, g):
+    args = (W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes, Gup, g)
+    return O.quantize_bwd(*args), O.bwd_l1_mass(*args)
+
+
+def slice_rows(P, rows):
+    return {k: np.ascontiguousarray(np.asarray(v)[rows]) for k, v in P.items()}

@@ -1,0 +1,162 @@
+"""Host-side checks of the C ABI that need no GPU.
+
+* the library builds and exports every function declared in include/*.h;
+* argument validation rejects bad calls before anything is launched, with
+  the documented status codes and a message;
+* the oracle and the product package do not import each other.
+
+The validation tests hand the library fake (but aligned, non-null) pointers,
+so they only run where no CUDA device is present: every case must be
+rejected by validation, and on a CPU-only machine even a validation bug could
+only produce UQ_ERR_CUDA, never touch memory.
+"""
+
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def libpath():
+    from paper_2506_03781_gb300 import build
+    return build.build()
+
+
+def declared_functions():
+    names = []
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        txt = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names += re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*(uq_[a-z_0-9]+)\s*\(", txt, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_abi():
+    names = declared_functions()
+    for n in ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq", "uq_last_error"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(libpath):
+    lib = ctypes.CDLL(libpath)
+    for n in declared_functions():
+        assert hasattr(lib, n), n
+    from paper_2506_03781_gb300 import api
+    assert set(api.ENTRY_POINTS) == set(declared_functions())
+    assert api.uq_abi_version() == 1
+    assert api.uq_last_error() == ""
+
+
+def _no_gpu():
+    try:
+        import torch
+        return not torch.cuda.is_available()
+    except Exception:
+        return True
+
+
+cpu_only = pytest.mark.skipif(not _no_gpu(), reason="fake-pointer validation tests run only without a GPU")
+
+FAKE = 0x7f0000000000          # 16-byte aligned, never dereferenced
+
+
+def _params(api, **over):
+    d = {n: FAKE + 0x1000 * i for i, n in enumerate(api.PARAM_NAMES)}
+    d.update(over)
+    return api.uq_params(**d)
+
+
+def _grads(api, **over):
+    d = {n: FAKE + 0x100000 + 0x1000 * i for i, n in enumerate(api.GRAD_NAMES)}
+    d.update(over)
+    return api.uq_grads(**d)
+
+
+@cpu_only
+@pytest.mark.parametrize("case,expect", [
+    (dict(q=0), "UNSUPPORTED"), (dict(q=5), "UNSUPPORTED"),
+    (dict(g=48), "ARG"), (dict(g=16), "ARG"), (dict(g=96, n_in=384), "UNSUPPORTED"),
+    (dict(n_in=200), "ARG"), (dict(out=0), "ARG"), (dict(n_in=0), "ARG"),
+    (dict(n_in=196608 * 2, g=128), "UNSUPPORTED"),
+    (dict(wd=7), "ARG"), (dict(map_mode=3), "ARG"), (dict(p_period=0), "ARG"), (dict(step=-1), "ARG"),
+    (dict(W=0), "ARG"), (dict(W=FAKE + 8), "ALIGN"), (dict(what=0), "ARG"), (dict(codes=FAKE + 4), "ALIGN"),
+    (dict(params=dict(delta=0)), "ARG"), (dict(params=dict(alpha=FAKE + 2)), "ALIGN"),
+])
+def test_fwd_validation(libpath, case, expect):
+    from paper_2506_03781_gb300 import api
+    a = dict(W=FAKE, wd=api.W_BF16, out=8, n_in=256, q=3, g=128, codes=FAKE + 0x9000, map_mode=1, step=0,
+             p_period=2, what=FAKE + 0xA000)
+    a.update({k: v for k, v in case.items() if k != "params"})
+    p = _params(api, **case.get("params", {}))
+    st = api.lib().uq_quantize_fwd(a["W"], a["wd"], a["out"], a["n_in"], a["q"], a["g"], p, a["codes"],
+                                   a["map_mode"], a["step"], a["p_period"], a["what"], None)
+    assert st == getattr(api, "UQ_ERR_" + expect), (st, api.uq_last_error())
+    assert api.uq_last_error() != ""
+
+
+@cpu_only
+def test_fwd_keep_step_does_not_need_weights(libpath):
+    """On a non-remap local step W, s and s_r are not read, so NULL is accepted
+    by validation (on this GPU-less machine the launch itself then fails)."""
+    from paper_2506_03781_gb300 import api
+    p = _params(api, s=0, sr=0)
+    st = api.lib().uq_quantize_fwd(0, api.W_BF16, 8, 256, 3, 128, p, FAKE + 0x9000, 1, 1, 2, FAKE + 0xA000, None)
+    assert st == api.UQ_ERR_CUDA
+    assert "uq_quantize_fwd" in api.uq_last_error()
+
+
+@cpu_only
+@pytest.mark.parametrize("field", ["ddelta", "dzu", "ds", "dsr", "dalpha", "dzb"])
+def test_bwd_validation_each_grad(libpath, field):
+    from paper_2506_03781_gb300 import api
+    st = api.lib().uq_quantize_bwd(FAKE, api.W_BF16, 8, 256, 3, 128, _params(api), FAKE + 0x9000,
+                                   FAKE + 0xB000, _grads(api, **{field: 0}), None)
+    assert st == api.UQ_ERR_ARG and field in api.uq_last_error()
+
+
+@cpu_only
+def test_export_and_init_validation(libpath):
+    from paper_2506_03781_gb300 import api
+    L = api.lib()
+    # export: unknown mode, EQ4 without W, REUSE without codes, misaligned planes
+    assert L.uq_export_bcq(FAKE, 1, 8, 256, 3, 128, _params(api), FAKE, 9, FAKE, FAKE, FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_export_bcq(0, 1, 8, 256, 3, 128, _params(api), FAKE, 1, FAKE, FAKE, FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_export_bcq(FAKE, 1, 8, 256, 3, 128, _params(api), 0, 0, FAKE, FAKE, FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_export_bcq(FAKE, 1, 8, 256, 3, 128, _params(api), FAKE, 0, FAKE + 4, FAKE, FAKE,
+                           None) == api.UQ_ERR_ALIGN
+    # init: G < 1, T < 0, bad clip, g too large, missing s
+    assert L.uq_init_params(FAKE, 1, 8, 256, 3, 128, 0, 15, 0, _params(api), FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_init_params(FAKE, 1, 8, 256, 3, 128, 30, -1, 0, _params(api), FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_init_params(FAKE, 1, 8, 256, 3, 128, 30, 15, 5, _params(api), FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_init_params(FAKE, 1, 1, 65536, 3, 65536, 30, 15, 0, _params(api), FAKE,
+                            None) == api.UQ_ERR_UNSUPPORTED
+    assert L.uq_init_params(FAKE, 1, 8, 256, 3, 128, 30, 15, 0, _params(api, s=0), FAKE, None) == api.UQ_ERR_ARG
+
+
+def test_binding_rejects_host_tensors_before_calling(libpath):
+    import torch
+    from paper_2506_03781_gb300 import api
+    W = torch.zeros(4, 128)
+    with pytest.raises(ValueError):
+        api.uq_quantize_fwd(W, 3, 128, {n: torch.zeros(1) for n in api.PARAM_NAMES}, torch.zeros(4, 128, dtype=torch.uint8),
+                            torch.zeros(4, 128))
+
+
+def test_oracle_and_product_are_independent():
+    """The oracle imports nothing from the product package and vice versa;
+    the only shared module is the seeded input generator."""
+    prod = os.path.join(ROOT, "paper_2506_03781_gb300")
+    for f in glob.glob(os.path.join(ROOT, "oracle", "*.py")):
+        src = open(f).read()
+        assert not re.search(r"^\s*(from|import)\s+paper_2506_03781_gb300", src, flags=re.M), f
+    for f in glob.glob(os.path.join(prod, "**", "*"), recursive=True):
+        if f.endswith((".py", ".cu", ".cuh", ".h")):
+            src = open(f).read()
+            assert not re.search(r"^\s*(from|import)\s+oracle", src, flags=re.M), f
+    synth_src = open(os.path.join(prod, "synth.py")).read()
+    for word in ("levels", "transform", "argmin", "bitplane"):
+        assert word not in synth_src.lower(), word
