@@ -415,12 +415,41 @@ def _int_det(M):
     return total
 
 
+def _solve(A, b):
+    """Solves the stacked systems A x = b (fp64): Gaussian elimination with
+    partial pivoting (the first largest |pivot| wins), then back substitution;
+    every product and difference rounded separately."""
+    A = np.array(A, F64)
+    b = np.array(b, F64)
+    n, q = b.shape
+    rows = np.arange(n)
+    for k in range(q):
+        p = k + np.argmax(np.abs(A[:, k:, k]), axis=1)
+        Ak, Ap = A[rows, k].copy(), A[rows, p].copy()
+        A[rows, k], A[rows, p] = Ap, Ak
+        bk, bp = b[rows, k].copy(), b[rows, p].copy()
+        b[rows, k], b[rows, p] = bp, bk
+        for i in range(k + 1, q):
+            f = A[:, i, k] / A[:, k, k]
+            A[:, i, k:] = A[:, i, k:] - f[:, None] * A[:, k, k:]
+            b[:, i] = b[:, i] - f * b[:, k]
+    xs = np.zeros((n, q), F64)
+    for i in range(q - 1, -1, -1):
+        acc = b[:, i].copy()
+        for j in range(i + 1, q):
+            acc = acc - A[:, i, j] * xs[:, j]
+        xs[:, i] = acc / A[:, i, i]
+    return xs
+
+
 def general_alternating(x, zb, G, T, q, trace=False):
     """General alternating update (Algorithm 3) on transformed groups x.
 
     Greedy start, then T rounds of
-      alpha <- (C^T C)^{-1} C^T (x - z_B 1)     (fp64; if C^T C is singular
-                                                  alpha is left unchanged)
+      alpha <- (C^T C)^{-1} C^T (x - z_B 1)     (fp64 normal equations solved
+                                                  by Gaussian elimination; if
+                                                  C^T C is singular alpha is
+                                                  left unchanged)
       C     <- argmin_C' || x - (C' alpha + z_B 1) ||^2   (= map_full)
       z_B   <- sum_i (x_i - C_i alpha) / g       (only when G == 1)
     alpha and z_B are stored in fp32 after each update.
@@ -440,8 +469,7 @@ def general_alternating(x, zb, G, T, q, trace=False):
         Cty = (Ct @ (x64 - zb.astype(F64)[:, None])[..., None])[..., 0]
         ok = _int_det(np.rint(CtC)) != 0                     # exact integer test
         if ok.any():
-            inv = np.linalg.inv(CtC[ok])
-            alpha[ok] = (inv @ Cty[ok][..., None])[..., 0].astype(F32)
+            alpha[ok] = _solve(CtC[ok], Cty[ok]).astype(F32)
         srt, cor, _ = sorted_levels(levels(alpha, zb))
         codes = map_full(x, srt, cor)
         if G == 1:

@@ -1,173 +1,169 @@
 // Backward of the quantizer: straight-through estimator with gradient
-// filtering (App. C.1) through Eq. 3, one thread block per row.
+// filtering (App. C.1) through Eq. 3.
 //
-// Per element (4 per lane per warp-step): recompute x = T_F(w) and
-// m = l(code), filter f = |x - m| <= tau (fp32 decision), write ds.  Per
-// group: 3 + q partial sums (dDelta, dz_U, dz_B, dalpha_j) are reduced over
-// the group's lanes by a segmented butterfly (no atomics); for g > 128 the
-// per-warp-step partials of a row go to shared memory and are summed per
-// group in warp-step order after the row is done.  ds_r: per-lane partials,
-// warp sums, then the 8 warp sums in warp order.
-// HBM traffic per element (bf16 W): 2 + 4 + 1 + 4 read, 4 written.
+// Per element (NV vectors of 4 per lane and group, see uq_common.cuh):
+// recompute x = T_F(w) and m = l(code), filter f = |x - m| <= tau (fp32
+// decision), write ds = -(Delta G f u) / s.  Per group, with G = dL/dW^:
+//   S0 = sum G ((m - z_U) - f u)   -> dDelta = S0
+//   S1 = sum_{f = 0} G             -> dz_U   = -Delta S1
+//   S2 = sum G                     -> dz_B   =  Delta S2
+//   S3 = sum G f u                 -> row partial Delta S3 of ds_r
+//   S4+j = sum G c_j               -> dalpha_j = Delta S4+j
+// are reduced over the group's LPG lanes (SegReduce, no atomics); groups of
+// more than 512 elements accumulate over several vector chunks first.
+// ds_r = -(sum over the row of Delta S3) / s_r, summed per row in warp and
+// lane order.  HBM traffic per element (bf16 W): 2 + 4 + 1 + 4 read, 4
+// written.
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
 namespace uq {
 
-template <int Q, typename WT, int GPS>
-__global__ void __launch_bounds__(kThreads)
+// Minimum resident blocks per SM the register allocation is bounded for.
+#ifndef UQ_BWD_MIN_BLOCKS
+#define UQ_BWD_MIN_BLOCKS 3
+#endif
+
+template <int Q, typename WT, int LPG>
+__global__ void __launch_bounds__(kThreads, UQ_BWD_MIN_BLOCKS)
 bwd_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
            const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
            const float* __restrict__ ZB, const uint8_t* __restrict__ CODES, const float* __restrict__ GUP,
            float* __restrict__ DS, float* __restrict__ DSR, float* __restrict__ DDELTA, float* __restrict__ DZU,
-           float* __restrict__ DZB, float* __restrict__ DALPHA, int n_in, int g) {
+           float* __restrict__ DZB, float* __restrict__ DALPHA, int64_t out, int n_in, int g, int R) {
     constexpr int L = 1 << Q;
-    constexpr int WB = kSlots / GPS;
-    constexpr int SH = GPS == 4 ? 3 : (GPS == 2 ? 4 : 5);
-    constexpr int SEGL = 32 / GPS;              // lanes per group within a warp-step
-    constexpr int NSUM = 3 + Q;                 // dDelta, dz_U, dz_B, dalpha_1..q
-    __shared__ GroupTables<Q> tabs[kWarps];
+    constexpr int NG = 32 / LPG;                 // groups per unit
+    using SR8 = SegReduce<LPG>;
+    __shared__ LvTab<Q, NG> tabs[kWarps];
+    __shared__ float tau_s[kWarps][NG];
     __shared__ float red[kWarps];
-    extern __shared__ float part[];             // [n_ws][8] when g > 128
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    GroupTables<Q>& t = tabs[warp];
-    const int64_t row = blockIdx.x;
-    const int n_ws = (n_in + kStep - 1) / kStep;
+    LvTab<Q, NG>& t = tabs[warp];
+    const int WPR = kWarps / R;
+    const int64_t row = (int64_t)blockIdx.x * R + warp / WPR;
+    const int wr = warp % WPR;
     const int Gr = n_in / g;
-    const int64_t eoff = row * (int64_t)n_in;
-    const int64_t goff = row * (int64_t)Gr;
-    const float sr = __ldg(SR + row);
-    const bool big = g > kStep;
-    float pacc = 0.f;                           // sum of G Delta f u over this lane's elements
+    const int units = (Gr + NG - 1) / NG;
+    const int nv = g / (4 * LPG);                // vectors per lane and group
+    const int sub = lane / LPG, li = lane % LPG;
+    float prow = 0.f;                            // this lane's share of sum Delta S3 over the row
 
-    for (int base = warp; base < n_ws; base += kWarps * WB) {
-        typename WT::raw wraw[WB];
-        float4 sv[WB], gv[WB];
-        uint32_t cv[WB];
-        float dl[WB], zu[WB];
-        bool ok[WB];
-        int col[WB];
+    if (row < out) {
+        const float sr = __ldg(SR + row);
+        const int64_t rbase = row * (int64_t)n_in;
+        for (int u = wr; u < units; u += WPR) {
+            const int gi = u * NG + sub;
+            const bool ok = gi < Gr;
+            const int64_t grp = row * Gr + gi;
+            const int64_t ebase = rbase + (int64_t)gi * g + 4 * li;
+            float dl = 0.f, zu = 0.f;
+            typename WT::raw wr4[4];
+            float4 sv[4], gv[4];
+            uint32_t cv[4];
+            auto load_chunk = [&](int c0) {
 #pragma unroll
-        for (int b = 0; b < WB; ++b) {
-            const int ws = base + b * kWarps;
-            col[b] = ws * kStep + lane * kVec;
-            ok[b] = ws < n_ws && col[b] < n_in;
-            if (ok[b]) {
-                const int64_t grp = goff + (ws * kStep) / g + (lane >> SH);
-                dl[b] = __ldg(DELTA + grp);
-                zu[b] = __ldg(ZU + grp);
-                wraw[b] = WT::load(W, eoff + col[b]);
-                sv[b] = ldg4(S + eoff + col[b]);
-                gv[b] = ldg4(GUP + eoff + col[b]);
-                cv[b] = __ldg(reinterpret_cast<const unsigned int*>(CODES + eoff + col[b]));
+                for (int v = 0; v < 4; ++v) {
+                    if (ok && c0 + v < nv) {
+                        const int64_t e = ebase + 4 * LPG * (c0 + v);
+                        wr4[v] = WT::load(W, e);
+                        sv[v] = ldg4(S + e);
+                        gv[v] = ldg4(GUP + e);
+                        cv[v] = __ldg(reinterpret_cast<const unsigned int*>(CODES + e));
+                    }
+                }
+            };
+            load_chunk(0);
+            if (ok) {
+                dl = __ldg(DELTA + grp);
+                zu = __ldg(ZU + grp);
             }
-        }
-        auto grp_of_slot = [&](int k) -> int64_t {
-            return goff + ((base + (k / GPS) * kWarps) * kStep) / g + (k % GPS);
-        };
-        auto ok_of_slot = [&](int k) -> bool {
-            const int ws = base + (k / GPS) * kWarps;
-            return ws < n_ws && (ws * kStep) / g + (k % GPS) < Gr;
-        };
-        __syncwarp();
-        build_tables<Q, false, false>(t, lane, ALPHA, ZB, grp_of_slot, ok_of_slot);
-
-#pragma unroll
-        for (int b = 0; b < WB; ++b) {
-            const int ws = base + b * kWarps;
-            if (ws >= n_ws) break;                      // warp-uniform
-            const int k = b * GPS + (lane >> SH);
+            __syncwarp();                        // previous unit is done with the tables
+            unit_levels<Q, NG>(t, tau_s[warp], lane, ALPHA, ZB, row * Gr + u * NG, min(NG, Gr - u * NG));
+            const float tau = tau_s[warp][sub];
             float acc[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-            if (ok[b]) {
-                float w[4], s[4], G[4], ds[4];
-                WT::unpack(wraw[b], w);
-                f4_to(sv[b], s);
-                f4_to(gv[b], G);
-                const float tau = t.tau[k];
-                const float d = dl[b], z = zu[b];
+            for (int c0 = 0; c0 < nv; c0 += 4) {
+                if (c0 > 0) load_chunk(c0);
 #pragma unroll
                 for (int v = 0; v < 4; ++v) {
-                    const int c = (cv[b] >> (8 * v)) & (L - 1);
-                    const float m = t.lv[k][c];
-                    float u;
-                    const float x = transform_x(w[v], s[v], d, sr, z, u);
-                    const bool f = fabsf(__fsub_rn(x, m)) <= tau;
-                    const float gb = G[v] * d;                   // dL/dw~
-                    const float fu = f ? u : 0.f;
-                    ds[v] = __fdividef(-(gb * fu), s[v]);
-                    acc[0] += G[v] * ((m - z) - fu);
-                    acc[1] += f ? 0.f : -gb;
-                    acc[2] += gb;
+                    if (!(ok && c0 + v < nv)) continue;
+                    float w[4], s[4], G[4], ds[4];
+                    WT::unpack(wr4[v], w);
+                    f4_to(sv[v], s);
+                    f4_to(gv[v], G);
 #pragma unroll
-                    for (int j = 0; j < Q; ++j) acc[3 + j] += ((c >> j) & 1) ? gb : -gb;
-                    pacc += gb * fu;
+                    for (int k = 0; k < 4; ++k) {
+                        const int c = (cv[v] >> (8 * k)) & (L - 1);
+                        const float m = t.lv[sub][c];
+                        float uu;
+                        const float x = transform_x(w[k], s[k], dl, sr, zu, uu);
+                        const bool f = fabsf(__fsub_rn(x, m)) <= tau;
+                        const float fu = f ? uu : 0.f;
+                        const float gfu = G[k] * fu;
+                        ds[k] = -__fdividef(dl * gfu, s[k]);
+                        acc[0] += G[k] * ((m - zu) - fu);
+                        acc[1] += f ? 0.f : G[k];
+                        acc[2] += G[k];
+                        acc[3] += gfu;
+#pragma unroll
+                        for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? G[k] : -G[k];
+                    }
+                    *reinterpret_cast<float4*>(DS + ebase + 4 * LPG * (c0 + v)) = make_float4(ds[0], ds[1], ds[2], ds[3]);
                 }
-                *reinterpret_cast<float4*>(DS + eoff + col[b]) = make_float4(ds[0], ds[1], ds[2], ds[3]);
             }
-            int slot;
-            const float tot = seg_reduce8<SEGL>(acc, lane, slot);
-            const bool writer = (lane & (SEGL / 8 - 1)) == 0 && slot < NSUM;
-            if (!big) {
-                const int gi = (ws * kStep) / g + (lane >> SH);
-                if (writer && gi < Gr) {
-                    const int64_t grp = goff + gi;
-                    float* dst = slot == 0 ? DDELTA + grp : slot == 1 ? DZU + grp : slot == 2 ? DZB + grp
-                                                                                : DALPHA + grp * Q + (slot - 3);
-                    *dst = tot;
+            const int slot0 = SR8::run(acc, lane);
+            if (ok && SR8::writer(lane)) {
+#pragma unroll
+                for (int i = 0; i < SR8::NOUT; ++i) {
+                    const int slot = slot0 + i;
+                    const float tot = acc[i];
+                    if (slot == 0) DDELTA[grp] = tot;
+                    else if (slot == 1) DZU[grp] = -(dl * tot);
+                    else if (slot == 2) DZB[grp] = dl * tot;
+                    else if (slot == 3) prow += dl * tot;
+                    else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * tot;
                 }
-            } else if (writer) {
-                part[ws * 8 + slot] = tot;
             }
         }
     }
 
-    pacc = warp_sum(pacc);
-    if (lane == 0) red[warp] = pacc;
+    // ds_r: the row's lane shares, summed in lane order, then in warp order.
+    prow = warp_sum(prow);
+    if (lane == 0) red[warp] = prow;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        float s = red[0];
-#pragma unroll
-        for (int w = 1; w < kWarps; ++w) s += red[w];
-        DSR[row] = -s / sr;
-    }
-    if (big) {
-        const int spg = g / kStep;                  // warp-steps per group
-        for (int idx = threadIdx.x; idx < Gr * NSUM; idx += kThreads) {
-            const int gi = idx / NSUM, slot = idx % NSUM;
-            float s = part[(gi * spg) * 8 + slot];
-            for (int st = 1; st < spg; ++st) s += part[(gi * spg + st) * 8 + slot];
-            const int64_t grp = goff + gi;
-            float* dst = slot == 0 ? DDELTA + grp : slot == 1 ? DZU + grp : slot == 2 ? DZB + grp
-                                                                        : DALPHA + grp * Q + (slot - 3);
-            *dst = s;
+    if (threadIdx.x < R) {
+        const int64_t r = (int64_t)blockIdx.x * R + threadIdx.x;
+        if (r < out) {
+            float s = red[threadIdx.x * WPR];
+            for (int w = 1; w < WPR; ++w) s += red[threadIdx.x * WPR + w];
+            DSR[r] = -s / __ldg(SR + r);
         }
     }
 }
 
-template <int Q, typename WT, int GPS>
+template <int Q, typename WT, int LPG>
 static cudaError_t run_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
                            uq_grads gr, cudaStream_t st) {
-    const int n_ws = (sh.n_in + kStep - 1) / kStep;
-    const size_t dyn = sh.g > kStep ? (size_t)n_ws * 8 * sizeof(float) : 0;
-    auto kern = bwd_kernel<Q, WT, GPS>;
-    if (dyn > 32 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-        if (e != cudaSuccess) return e;
-    }
-    kern<<<dim3((unsigned)sh.out), kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup,
-                                                        gr.ds, gr.dsr, gr.ddelta, gr.dzu, gr.dzb, gr.dalpha,
-                                                        sh.n_in, sh.g);
+    constexpr int NG = 32 / LPG;
+    const int Gr = sh.n_in / sh.g;
+    const int R = rows_per_block((Gr + NG - 1) / NG);
+    const int64_t blocks = (sh.out + R - 1) / R;
+    bwd_kernel<Q, WT, LPG><<<dim3((unsigned)blocks), kThreads, 0, st>>>(
+        W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr, gr.ddelta, gr.dzu, gr.dzb, gr.dalpha,
+        sh.out, sh.n_in, sh.g, R);
     return cudaGetLastError();
 }
 
 template <int Q, typename WT>
 static cudaError_t bwd_g(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
                          uq_grads gr, cudaStream_t st) {
-    if (sh.g == 32) return run_bwd<Q, WT, 4>(sh, W, p, codes, gup, gr, st);
-    if (sh.g == 64) return run_bwd<Q, WT, 2>(sh, W, p, codes, gup, gr, st);
-    return run_bwd<Q, WT, 1>(sh, W, p, codes, gup, gr, st);
+    switch (lanes_per_group(sh.g)) {
+        case 4: return run_bwd<Q, WT, 4>(sh, W, p, codes, gup, gr, st);
+        case 8: return run_bwd<Q, WT, 8>(sh, W, p, codes, gup, gr, st);
+        case 16: return run_bwd<Q, WT, 16>(sh, W, p, codes, gup, gr, st);
+        default: return run_bwd<Q, WT, 32>(sh, W, p, codes, gup, gr, st);
+    }
 }
 
 template <int Q>

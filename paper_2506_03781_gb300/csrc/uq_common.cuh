@@ -1,14 +1,18 @@
 // Device helpers shared by the UniQuan_F kernels (sm_103a).
 //
-// Work decomposition used by the per-step kernels (forward, backward,
-// export): one thread block per weight-matrix row, 8 warps; the row is cut
-// into "warp-steps" of 128 consecutive elements, each lane owning 4
-// consecutive elements (one 16-byte fp32 vector).  Since g is 32, 64 or a
-// multiple of 128, a warp-step holds GPS = 4, 2 or 1 groups (or a 128-wide
-// slice of one group), each group on a contiguous run of 32/GPS lanes.
-// Every value that decides an integer is computed with explicitly rounded
-// intrinsics (__fadd_rn, __fmul_rn, __fdiv_rn): no FMA contraction, IEEE
-// division, the operation order written in uq_api.h.
+// Work decomposition of the per-step kernels (forward, backward): thread
+// blocks of 8 warps own R whole rows (R = 1 for long rows, up to 8 when a
+// row has fewer work units than warps).  A warp's work unit is a set of
+// whole groups: NG = 32/LPG groups, LPG lanes per group, each lane owning
+// vectors of 4 consecutive elements at element offsets 4*(lane%LPG) +
+// 4*LPG*v of its group (v = 0..NV-1, NV = g/(4*LPG)).  One warp instruction
+// for a given v therefore reads 4*LPG contiguous elements of each of the NG
+// groups -- whole 128-byte segments of the fp32 streams -- and a group's
+// partial sums live on LPG neighbouring lanes only.  LPG = 4 for g = 32
+// (NV = 2) and g = 64, LPG = g/16 for g = 128, 256, and LPG = 32 with
+// NV = g/128 for the other multiples of 128.  Every value that decides an integer is computed with explicitly
+// rounded intrinsics (__fadd_rn, __fmul_rn, __fdiv_rn): no FMA contraction,
+// IEEE division, the operation order written in uq_api.h.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -199,6 +203,140 @@ __device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
     return v;
+}
+
+
+// ---------------------------------------------------------------------------
+// Unit-mapped tables (NS group slots per warp)
+// ---------------------------------------------------------------------------
+
+template <int Q, int NS>
+struct LvTab {                       // levels by code word and tau per slot
+    static constexpr int L = 1 << Q;
+    float lv[NS][L];
+    float tau[NS];
+};
+
+template <int Q, int NS>
+struct MapTab {                      // + sorted order and local-mapping neighbours
+    static constexpr int L = 1 << Q;
+    float lv[NS][L];
+    float srt[NS][L];
+    float4 nb[NS][L];
+    uint8_t cor[NS][L];
+    uint8_t rk[NS][L];
+};
+
+// Levels l(c) of the NS groups grp0 + k (k < n_ok) and tau = min_j |alpha_j|.
+// Whole warp; ends with __syncwarp().
+template <int Q, int NS, typename TAB>
+__device__ __forceinline__ void unit_levels(TAB& t, float* tau, int lane, const float* __restrict__ alpha,
+                                            const float* __restrict__ zb, int64_t grp0, int n_ok) {
+    constexpr int L = 1 << Q;
+    constexpr int E = NS * L;
+#pragma unroll
+    for (int e = lane; e < E; e += 32) {
+        const int k = e / L, c = e % L;
+        float lvv = 0.f;
+        if (k < n_ok) {
+            const int64_t grp = grp0 + k;
+            float a[Q];
+#pragma unroll
+            for (int j = 0; j < Q; ++j) a[j] = __ldg(alpha + grp * Q + j);
+            lvv = level_of<Q>(c, a, __ldg(zb + grp));
+            if (tau != nullptr && c == 0) {
+                float m = fabsf(a[0]);
+#pragma unroll
+                for (int j = 1; j < Q; ++j) m = fminf(m, fabsf(a[j]));
+                tau[k] = m;
+            }
+        }
+        t.lv[k][c] = lvv;
+    }
+    __syncwarp();
+}
+
+// Sorted order (ascending, ties by code word) and, if NB, the neighbour
+// triples of the local mapping.  Requires t.lv; ends with __syncwarp().
+template <int Q, int NS, bool NB>
+__device__ __forceinline__ void unit_sort(MapTab<Q, NS>& t, int lane) {
+    constexpr int L = 1 << Q;
+    constexpr int E = NS * L;
+#pragma unroll
+    for (int e = lane; e < E; e += 32) {
+        const int k = e / L, c = e % L;
+        const float v = t.lv[k][c];
+        int r = 0;
+#pragma unroll
+        for (int c2 = 0; c2 < L; ++c2) {
+            const float v2 = t.lv[k][c2];
+            r += (v2 < v) || (v2 == v && c2 < c);
+        }
+        t.srt[k][r] = v;
+        t.cor[k][r] = static_cast<uint8_t>(c);
+        t.rk[k][c] = static_cast<uint8_t>(r);
+    }
+    __syncwarp();
+    if constexpr (NB) {
+#pragma unroll
+        for (int e = lane; e < E; e += 32) {
+            const int k = e / L, c = e % L;
+            const int r = t.rk[k][c];
+            const int rl = r > 0 ? r - 1 : 0;
+            const int rh = r < L - 1 ? r + 1 : L - 1;
+            const uint32_t packed = uint32_t(t.cor[k][rl]) | (uint32_t(t.cor[k][rh]) << 8);
+            t.nb[k][c] = make_float4(t.srt[k][rl], t.lv[k][c], t.srt[k][rh], __uint_as_float(packed));
+        }
+        __syncwarp();
+    }
+}
+
+// Reduce-scatter of 8 partial sums over LPG consecutive lanes (LPG = 2..32).
+// The first min(3, log2 LPG) butterfly levels halve the live values while
+// exchanging the other half with the partner lane; remaining levels sum the
+// last value.  On return v[0..NOUT) hold the segment totals of slots
+// slot0 .. slot0+NOUT-1; lanes with (lane % LPG) a multiple of LPG/8 (all
+// lanes if LPG <= 8) hold distinct slots.  Fixed order: deterministic.
+template <int LPG>
+struct SegReduce {
+    static constexpr int HALV = LPG >= 8 ? 3 : (LPG == 4 ? 2 : 1);
+    static constexpr int NOUT = 8 >> HALV;
+    static __device__ __forceinline__ int run(float v[8], int lane) {
+        int base = 0;
+#pragma unroll
+        for (int lvl = 0; lvl < HALV; ++lvl) {
+            const int off = LPG >> (lvl + 1);
+            const int h = 4 >> lvl;
+            const bool up = (lane & off) != 0;
+#pragma unroll
+            for (int i = 0; i < h; ++i) {
+                const float send = up ? v[i] : v[i + h];
+                const float keep = up ? v[i + h] : v[i];
+                v[i] = keep + __shfl_xor_sync(kFull, send, off);
+            }
+            base += up ? h : 0;
+        }
+#pragma unroll
+        for (int off = LPG >> (HALV + 1); off >= 1; off >>= 1) v[0] += __shfl_xor_sync(kFull, v[0], off);
+        return base;
+    }
+    static __device__ __forceinline__ bool writer(int lane) {
+        return LPG <= 8 ? true : ((lane % LPG) % (LPG / 8)) == 0;
+    }
+};
+
+// Rows per block for the unit mapping: the largest power of two R <= 8 with
+// R * units_per_row <= 8 (at least 1).
+__host__ __device__ inline int rows_per_block(int units_per_row) {
+    int R = 1;
+    while (R < kWarps && 2 * R * units_per_row <= kWarps) R *= 2;
+    return R;
+}
+
+// LPG for a group size: 4 for g = 32 (NV = 2) and g = 64, g/16 for g = 128
+// and 256, else 32 (g = 512: NV = 4; larger multiples of 128: NV = g/128).
+__host__ __device__ inline int lanes_per_group(int g) {
+    return g <= 64 ? 4 : (g == 128 || g == 256) ? g / 16 : 32;
 }
 
 }  // namespace uq

@@ -78,7 +78,10 @@ __device__ __forceinline__ bool int_singular(const long long Min[Q][Q]) {
     return det == 0ull;
 }
 
-// Solves A x = b in fp64 (Gaussian elimination, partial pivoting).
+// Solves A x = b in fp64: Gaussian elimination with partial pivoting (first
+// largest |pivot| wins) and back substitution, every product and difference
+// rounded separately (no FMA contraction).  The exact solution is often an
+// fp32 rounding tie (short dyadic values), so the rounding order is fixed.
 template <int Q>
 __device__ __forceinline__ void solve_fp64(const long long Ain[Q][Q], const double bin[Q], double x[Q]) {
     double A[Q][Q], b[Q];
@@ -88,24 +91,34 @@ __device__ __forceinline__ void solve_fp64(const long long Ain[Q][Q], const doub
 #pragma unroll
         for (int j = 0; j < Q; ++j) A[i][j] = (double)Ain[i][j];
     }
+#pragma unroll
     for (int k = 0; k < Q; ++k) {
         int p = k;
+#pragma unroll
         for (int i = k + 1; i < Q; ++i)
             if (fabs(A[i][k]) > fabs(A[p][k])) p = i;
-        if (p != k) {
-            for (int j = 0; j < Q; ++j) { const double tmp = A[k][j]; A[k][j] = A[p][j]; A[p][j] = tmp; }
-            const double tb = b[k]; b[k] = b[p]; b[p] = tb;
-        }
+#pragma unroll
         for (int i = k + 1; i < Q; ++i) {
-            const double f = A[i][k] / A[k][k];
-            for (int j = k; j < Q; ++j) A[i][j] -= f * A[k][j];
-            b[i] -= f * b[k];
+            if (i == p) {
+#pragma unroll
+                for (int j = 0; j < Q; ++j) { const double tmp = A[k][j]; A[k][j] = A[i][j]; A[i][j] = tmp; }
+                const double tb = b[k]; b[k] = b[i]; b[i] = tb;
+            }
+        }
+#pragma unroll
+        for (int i = k + 1; i < Q; ++i) {
+            const double f = __ddiv_rn(A[i][k], A[k][k]);
+#pragma unroll
+            for (int j = k; j < Q; ++j) A[i][j] = __dsub_rn(A[i][j], __dmul_rn(f, A[k][j]));
+            b[i] = __dsub_rn(b[i], __dmul_rn(f, b[k]));
         }
     }
+#pragma unroll
     for (int i = Q - 1; i >= 0; --i) {
         double s = b[i];
-        for (int j = i + 1; j < Q; ++j) s -= A[i][j] * x[j];
-        x[i] = s / A[i][i];
+#pragma unroll
+        for (int j = i + 1; j < Q; ++j) s = __dsub_rn(s, __dmul_rn(A[i][j], x[j]));
+        x[i] = __ddiv_rn(s, A[i][i]);
     }
 }
 
