@@ -187,6 +187,17 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                         uq_params params, const uint8_t* codes, uq_export_mode mode,
                         uint32_t* bitplanes, float* alpha_star, float* zb_star, void* stream);
 
+/*
+ * uq_check_device -- waits for `stream` to finish, then reports whether a
+ * pipelined kernel of this library gave up waiting for its own data copies
+ * since the last check (every wait on an mbarrier is bounded to about one
+ * second of GPU clock; when one runs out the warp stops computing and a
+ * device-side indicator is set instead of hanging).  Clears the indicator.
+ * UQ_OK if none ran out; UQ_ERR_CUDA if one did or the synchronisation
+ * failed.  Needs no arguments beyond the stream; allocates nothing.
+ */
+uq_status uq_check_device(void* stream);
+
 /* Message for the last non-OK status returned on the calling thread (never
  * NULL; "" if none).  Owned by the library, valid until the next call on
  * the same thread. */

@@ -152,4 +152,14 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                        "uq_export_bcq");
 }
 
+uq_status uq_check_device(void* stream) {
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
+    unsigned int flag = 0;
+    e = uq::stream_error(true, &flag);
+    if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
+    if (flag) return fail(UQ_ERR_CUDA, "a pipelined kernel gave up waiting for its own data copies (bounded wait ran out)");
+    return ok();
+}
+
 }  // extern "C"

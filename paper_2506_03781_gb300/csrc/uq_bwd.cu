@@ -175,6 +175,7 @@ static cudaError_t bwd_w(const Shape& sh, const void* W, uq_params p, const uint
 
 cudaError_t launch_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
                        uq_grads gr, cudaStream_t st) {
+    if (stream_path_ok(sh)) return launch_bwd_stream(sh, W, p, codes, gup, gr, st);
     switch (sh.q) {
         case 1: return bwd_w<1>(sh, W, p, codes, gup, gr, st);
         case 2: return bwd_w<2>(sh, W, p, codes, gup, gr, st);

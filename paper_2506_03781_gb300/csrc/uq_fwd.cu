@@ -163,6 +163,7 @@ static cudaError_t fwd_w(const Shape& sh, const void* W, uq_params p, uint8_t* c
 
 cudaError_t launch_fwd(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode, float* what,
                        cudaStream_t st) {
+    if (stream_path_ok(sh)) return launch_fwd_stream(sh, W, p, codes, mode, what, st);
     switch (sh.q) {
         case 1: return fwd_w<1>(sh, W, p, codes, mode, what, st);
         case 2: return fwd_w<2>(sh, W, p, codes, mode, what, st);

@@ -28,6 +28,16 @@ cudaError_t launch_export(const Shape& sh, const void* W, uq_params p, const uin
 cudaError_t launch_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
                         cudaStream_t st);
 
+// Persistent TMA-pipelined kernels (uq_stream.cu): used when stream_path_ok.
+bool stream_path_ok(const Shape& sh);
+cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                              float* what, cudaStream_t st);
+cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
+                              const float* gup, uq_grads gr, cudaStream_t st);
+// Reads (and optionally clears) the flag a pipelined kernel sets when a
+// bounded wait runs out.
+cudaError_t stream_error(bool clear, unsigned int* flag);
+
 // Forward modes (see uq_api.h): full mapping, local remap step, keep codes.
 enum { FWD_FULL = 0, FWD_REMAP = 1, FWD_KEEP = 2 };
 

@@ -1,0 +1,542 @@
+// Persistent, TMA-pipelined forward and backward kernels (the fast path for
+// g in {32, 64, 128} and rows that split into whole work units).
+//
+// Each warp runs its own pipeline over its work units (NG whole groups =
+// UE contiguous elements of one row, the lane mapping of uq_common.cuh):
+// lane 0 issues one bulk copy (cp.async.bulk, completion counted on an
+// mbarrier) per input stream of a unit -- weights, s, dL/dW^, code words and
+// the unit's group parameters -- into one of NST shared-memory stages, and
+// the warp computes from shared memory while the copies of the next units
+// are in flight.  Thread blocks are persistent: block b handles row blocks
+// b, b + gridDim.x, ...; within a row block the warps split the row's units
+// as in the non-pipelined kernels, and one block barrier per row block
+// orders the ds_r sum.  Every mbarrier wait is bounded (about one second of
+// GPU clock); a wait that runs out sets g_stream_err, which
+// uq_check_device() reports, and the warp stops computing.
+#include "uq_common.cuh"
+#include "uq_launch.h"
+
+namespace uq {
+
+__device__ unsigned int g_stream_err = 0;
+
+namespace tma {
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void bar_init_fence() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void bar_arrive_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void bar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool bar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: gives up after ~2^31 GPU clock cycles (about one second).
+__device__ __forceinline__ bool bar_wait(uint32_t bar, uint32_t parity) {
+    if (bar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!bar_try_wait(bar, parity)) {
+        if (clock64() - t0 > (1ll << 31)) return false;
+    }
+    return true;
+}
+__device__ __forceinline__ void fence_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// Global -> shared bulk copy; bytes a multiple of 16, both addresses 16-byte aligned.
+__device__ __forceinline__ void copy_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+}  // namespace tma
+
+constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
+
+// Shared-memory stage layout of one work unit.
+template <int Q, typename WT, int G_>
+struct Stage {
+    static constexpr int LPG = G_ <= 64 ? 4 : 8;
+    static constexpr int NG = 32 / LPG;                  // groups per unit
+    static constexpr int NV = G_ / (4 * LPG);            // vectors per lane
+    static constexpr int UE = NG * G_;                   // elements per unit
+    static constexpr int WBYTES = sizeof(typename WT::raw) / 4;
+    static constexpr int SZ_W = UE * WBYTES, SZ_F = UE * 4, SZ_C = UE, SZ_P = NG * 4, SZ_A = NG * Q * 4;
+    static constexpr int OFF_W = 0;
+    static constexpr int OFF_S = align_up(OFF_W + SZ_W, 16);
+    static constexpr int OFF_G = OFF_S + SZ_F;
+    static constexpr int OFF_C = OFF_G + SZ_F;
+    static constexpr int OFF_D = align_up(OFF_C + SZ_C, 16);
+    static constexpr int OFF_Z = OFF_D + SZ_P;
+    static constexpr int OFF_B = OFF_Z + SZ_P;
+    static constexpr int OFF_A = OFF_B + SZ_P;
+    static constexpr int BYTES = align_up(OFF_A + SZ_A, 128);
+    static_assert(SZ_P % 16 == 0 && SZ_A % 16 == 0 && SZ_C % 16 == 0, "bulk copy sizes must be multiples of 16");
+};
+
+// Work-item bookkeeping shared by the two kernels: item i of a warp is unit
+// wr + WPR * (i % n_w) of row (blockIdx.x + (i / n_w) * gridDim.x) * R + row_sub.
+struct Items {
+    int R, WPR, row_sub, wr, n_w;
+    long long total;
+    __device__ Items(int U, int Rr, int n_rb, int warp) {
+        R = Rr;
+        WPR = kWarps / R;
+        row_sub = warp / WPR;
+        wr = warp % WPR;
+        n_w = wr < U ? (U - wr + WPR - 1) / WPR : 0;
+        const int mine = (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+        total = (long long)mine * n_w;
+    }
+    __device__ int64_t row_of(long long i) const {
+        return ((int64_t)blockIdx.x + (i / n_w) * (int64_t)gridDim.x) * R + row_sub;
+    }
+    __device__ int unit_of(long long i) const { return wr + WPR * (int)(i % n_w); }
+};
+
+// ---------------------------------------------------------------------------
+// Backward
+// ---------------------------------------------------------------------------
+
+template <int Q, typename WT, int G_, int NST>
+__global__ void __launch_bounds__(kThreads, 2)
+bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
+                  const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
+                  const float* __restrict__ ZB, const uint8_t* __restrict__ CODES, const float* __restrict__ GUP,
+                  float* __restrict__ DS, float* __restrict__ DSR, float* __restrict__ DDELTA,
+                  float* __restrict__ DZU, float* __restrict__ DZB, float* __restrict__ DALPHA, int64_t out,
+                  int n_in, int R, int n_rb) {
+    using St = Stage<Q, WT, G_>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE;
+    constexpr uint32_t TX = St::SZ_W + 2 * St::SZ_F + St::SZ_C + 3 * St::SZ_P + St::SZ_A;
+    using SR8 = SegReduce<LPG>;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) unsigned long long bars[kWarps][NST];
+    __shared__ LvTab<Q, NG> tabs[kWarps];
+    __shared__ float tau_s[kWarps][NG];
+    __shared__ float red[2][kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sub = lane / LPG, li = lane % LPG;
+    const int U = n_in / UE, Gr = n_in / G_;
+    const Items it(U, R, n_rb, warp);
+    unsigned char* wsm = smem + (size_t)warp * NST * St::BYTES;
+    LvTab<Q, NG>& t = tabs[warp];
+
+    if (lane == 0) {
+        for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
+        tma::bar_init_fence();
+    }
+    __syncthreads();
+
+    auto issue = [&](long long i) {                       // lane 0 only
+        const int s = (int)(i % NST);
+        const uint32_t bar = tma::smem_addr(&bars[warp][s]);
+        const int64_t row = it.row_of(i);
+        if (row >= out) { tma::bar_arrive(bar); return; }
+        const int64_t e0 = row * n_in + (int64_t)it.unit_of(i) * UE;
+        const int64_t g0 = row * Gr + (int64_t)it.unit_of(i) * NG;
+        const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+        tma::fence_async_smem();
+        tma::bar_arrive_tx(bar, TX);
+        tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
+        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_F, bar);
+        tma::copy_g2s(d + St::OFF_G, GUP + e0, St::SZ_F, bar);
+        tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+        tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+    };
+    if (lane == 0)
+        for (long long i = 0; i < NST && i < it.total; ++i) issue(i);
+
+    bool alive = true;
+    long long i = 0;
+    const int n_mine = it.n_w > 0 ? (int)(it.total / it.n_w)
+                                  : (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+    for (int k = 0; k < n_mine; ++k) {
+        const int64_t rb = (int64_t)blockIdx.x + (int64_t)k * gridDim.x;
+        const int64_t row = rb * R + it.row_sub;
+        const bool row_ok = row < out;
+        const float sr = row_ok ? __ldg(SR + row) : 1.f;
+        float prow = 0.f;
+        for (int j = 0; j < it.n_w; ++j, ++i) {
+            const int s = (int)(i % NST);
+            if (alive && !tma::bar_wait(tma::smem_addr(&bars[warp][s]), (uint32_t)((i / NST) & 1))) {
+                alive = false;
+                if (lane == 0) atomicOr(&g_stream_err, 1u);
+            }
+            if (alive && row_ok) {
+                const unsigned char* st = wsm + (size_t)s * St::BYTES;
+                const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
+                const float* pz = reinterpret_cast<const float*>(st + St::OFF_Z);
+                const float* pb = reinterpret_cast<const float*>(st + St::OFF_B);
+                const float* pa = reinterpret_cast<const float*>(st + St::OFF_A);
+                // levels and tau of the unit's groups, from the staged parameters
+#pragma unroll
+                for (int e = lane; e < NG * L; e += 32) {
+                    const int kk = e / L, c = e % L;
+                    float a[Q];
+#pragma unroll
+                    for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
+                    t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+                    if (c == 0) {
+                        float m = fabsf(a[0]);
+#pragma unroll
+                        for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
+                        tau_s[warp][kk] = m;
+                    }
+                }
+                __syncwarp();
+                const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub];
+                const int unit = it.unit_of(i);
+                const int64_t ebase = row * n_in + (int64_t)unit * UE;
+                float acc[8];
+#pragma unroll
+                for (int q8 = 0; q8 < 8; ++q8) acc[q8] = 0.f;
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int el = sub * G_ + 4 * li + 4 * LPG * v;
+                    float w[4], s4[4], G[4], ds[4];
+                    WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
+                    f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
+                    f4_to(*reinterpret_cast<const float4*>(st + St::OFF_G + el * 4), G);
+                    const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+#pragma unroll
+                    for (int kq = 0; kq < 4; ++kq) {
+                        const int c = (cv >> (8 * kq)) & (L - 1);
+                        const float m = t.lv[sub][c];
+                        float uu;
+                        const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
+                        const bool f = fabsf(__fsub_rn(x, m)) <= tau;
+                        const float fu = f ? uu : 0.f;
+                        const float gfu = G[kq] * fu;
+                        ds[kq] = -__fdividef(dl * gfu, s4[kq]);
+                        acc[0] += G[kq] * ((m - zu) - fu);
+                        acc[1] += f ? 0.f : G[kq];
+                        acc[2] += G[kq];
+                        acc[3] += gfu;
+#pragma unroll
+                        for (int jj = 0; jj < Q; ++jj) acc[4 + jj] += ((c >> jj) & 1) ? G[kq] : -G[kq];
+                    }
+                    *reinterpret_cast<float4*>(DS + ebase + el) = make_float4(ds[0], ds[1], ds[2], ds[3]);
+                }
+                const int slot0 = SR8::run(acc, lane);
+                if (SR8::writer(lane)) {
+                    const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
+#pragma unroll
+                    for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
+                        const int slot = slot0 + q8;
+                        const float tot = acc[q8];
+                        if (slot == 0) DDELTA[grp] = tot;
+                        else if (slot == 1) DZU[grp] = -(dl * tot);
+                        else if (slot == 2) DZB[grp] = dl * tot;
+                        else if (slot == 3) prow += dl * tot;
+                        else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * tot;
+                    }
+                }
+            }
+            __syncwarp();                                // stage s and the tables are free again
+            if (alive && lane == 0 && i + NST < it.total) issue(i + NST);
+        }
+        prow = warp_sum(prow);
+        if (lane == 0) red[k & 1][warp] = prow;
+        __syncthreads();
+        if (threadIdx.x < R) {
+            const int64_t r = rb * R + threadIdx.x;
+            if (r < out) {
+                const int WPR = kWarps / R;
+                float s = red[k & 1][threadIdx.x * WPR];
+                for (int w = 1; w < WPR; ++w) s += red[k & 1][threadIdx.x * WPR + w];
+                DSR[r] = -s / __ldg(SR + r);
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Forward
+// ---------------------------------------------------------------------------
+
+template <int Q, typename WT, int G_, int NST>
+__global__ void __launch_bounds__(kThreads, 2)
+fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
+                  const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
+                  const float* __restrict__ ZB, uint8_t* __restrict__ CODES, float* __restrict__ WHAT,
+                  int64_t out, int n_in, int R, int n_rb, int mode) {
+    using St = Stage<Q, WT, G_>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) unsigned long long bars[kWarps][NST];
+    __shared__ MapTab<Q, NG> tabs[kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sub = lane / LPG, li = lane % LPG;
+    const int U = n_in / UE, Gr = n_in / G_;
+    const Items it(U, R, n_rb, warp);
+    unsigned char* wsm = smem + (size_t)warp * NST * St::BYTES;
+    MapTab<Q, NG>& t = tabs[warp];
+    const bool need_x = mode != FWD_KEEP, need_c = mode != FWD_FULL;
+    const uint32_t TX = (need_x ? St::SZ_W + St::SZ_F : 0) + (need_c ? St::SZ_C : 0) + 3 * St::SZ_P + St::SZ_A;
+
+    if (lane == 0) {
+        for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+
+    auto issue = [&](long long i) {
+        const int s = (int)(i % NST);
+        const uint32_t bar = tma::smem_addr(&bars[warp][s]);
+        const int64_t row = it.row_of(i);
+        if (row >= out) { tma::bar_arrive(bar); return; }
+        const int64_t e0 = row * n_in + (int64_t)it.unit_of(i) * UE;
+        const int64_t g0 = row * Gr + (int64_t)it.unit_of(i) * NG;
+        const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+        tma::fence_async_smem();
+        tma::bar_arrive_tx(bar, TX);
+        if (need_x) {
+            tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
+            tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_F, bar);
+        }
+        if (need_c) tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+        tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+    };
+    if (lane == 0)
+        for (long long i = 0; i < NST && i < it.total; ++i) issue(i);
+
+    for (long long i = 0; i < it.total; ++i) {
+        const int s = (int)(i % NST);
+        if (!tma::bar_wait(tma::smem_addr(&bars[warp][s]), (uint32_t)((i / NST) & 1))) {
+            if (lane == 0) atomicOr(&g_stream_err, 1u);
+            return;                                      // no block barrier in this kernel
+        }
+        const int64_t row = it.row_of(i);
+        if (row < out) {
+            const unsigned char* st = wsm + (size_t)s * St::BYTES;
+            const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
+            const float* pz = reinterpret_cast<const float*>(st + St::OFF_Z);
+            const float* pb = reinterpret_cast<const float*>(st + St::OFF_B);
+            const float* pa = reinterpret_cast<const float*>(st + St::OFF_A);
+#pragma unroll
+            for (int e = lane; e < NG * L; e += 32) {
+                const int kk = e / L, c = e % L;
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
+                t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+            }
+            __syncwarp();
+            if (mode == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
+            else if (mode == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            const float dl = pd[sub], zu = pz[sub];
+            const float sr = need_x ? __ldg(SR + row) : 0.f;
+            const int64_t ebase = row * n_in + (int64_t)it.unit_of(i) * UE;
+            float srt[L];
+            if (mode == FWD_FULL) {
+#pragma unroll
+                for (int r = 0; r < L; ++r) srt[r] = t.srt[sub][r];
+            }
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                const int el = sub * G_ + 4 * li + 4 * LPG * v;
+                float o[4];
+                uint32_t nc = 0;
+                const uint32_t cv = need_c ? *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el) : 0u;
+                if (mode == FWD_KEEP) {
+#pragma unroll
+                    for (int kq = 0; kq < 4; ++kq) {
+                        const int c = (cv >> (8 * kq)) & (L - 1);
+                        o[kq] = __fmul_rn(dl, __fsub_rn(t.lv[sub][c], zu));
+                    }
+                } else {
+                    float w[4], s4[4];
+                    WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
+                    f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
+                    if (mode == FWD_REMAP) {
+#pragma unroll
+                        for (int kq = 0; kq < 4; ++kq) {
+                            const int c = (cv >> (8 * kq)) & (L - 1);
+                            const float4 nb = t.nb[sub][c];
+                            float uu;
+                            const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
+                            const uint32_t packed = __float_as_uint(nb.w);
+                            float best = fabsf(__fsub_rn(x, nb.y));
+                            float m = nb.y;
+                            uint32_t code = c;
+                            const float dlo = fabsf(__fsub_rn(x, nb.x));
+                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
+                            const float dhi = fabsf(__fsub_rn(x, nb.z));
+                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                            o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
+                            nc |= code << (8 * kq);
+                        }
+                    } else {
+#pragma unroll
+                        for (int kq = 0; kq < 4; ++kq) {
+                            float uu, m;
+                            const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
+                            const int r = nearest_rank<L>(x, srt, m);
+                            o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
+                            nc |= uint32_t(t.cor[sub][r]) << (8 * kq);
+                        }
+                    }
+                    *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
+                }
+                *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
+            }
+        }
+        __syncwarp();
+        if (lane == 0 && i + NST < it.total) issue(i + NST);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Launchers
+// ---------------------------------------------------------------------------
+
+constexpr int kStreamStages = 2;
+
+static int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return 1;
+    return n;
+}
+
+bool stream_path_ok(const Shape& sh) {
+    if (!(sh.g == 32 || sh.g == 64 || sh.g == 128)) return false;
+    const int ue = sh.g == 32 ? 256 : 512;
+    return sh.n_in % ue == 0;
+}
+
+template <typename KERN>
+static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
+    int per_sm = 0;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    const long long cap = (long long)sm_count() * per_sm;
+    grid = (int)(n_rb < cap ? n_rb : cap);
+    return cudaSuccess;
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
+                                  const float* gup, uq_grads gr, cudaStream_t st) {
+    using St = Stage<Q, WT, G_>;
+    const int U = sh.n_in / St::UE;
+    const int R = rows_per_block(U);
+    const int n_rb = (int)((sh.out + R - 1) / R);
+    const size_t dyn = (size_t)kWarps * kStreamStages * St::BYTES;
+    auto kern = bwd_stream_kernel<Q, WT, G_, kStreamStages>;
+    int grid = 0;
+    cudaError_t e = grid_for(kern, dyn, n_rb, grid);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr,
+                                      gr.ddelta, gr.dzu, gr.dzb, gr.dalpha, sh.out, sh.n_in, R, n_rb);
+    return cudaGetLastError();
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t run_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                                  float* what, cudaStream_t st) {
+    using St = Stage<Q, WT, G_>;
+    const int U = sh.n_in / St::UE;
+    const int R = rows_per_block(U);
+    const int n_rb = (int)((sh.out + R - 1) / R);
+    const size_t dyn = (size_t)kWarps * kStreamStages * St::BYTES;
+    auto kern = fwd_stream_kernel<Q, WT, G_, kStreamStages>;
+    int grid = 0;
+    cudaError_t e = grid_for(kern, dyn, n_rb, grid);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R,
+                                      n_rb, mode);
+    return cudaGetLastError();
+}
+
+template <int Q, typename WT>
+static cudaError_t bwd_stream_g(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
+                                const float* gup, uq_grads gr, cudaStream_t st) {
+    if (sh.g == 32) return run_bwd_stream<Q, WT, 32>(sh, W, p, codes, gup, gr, st);
+    if (sh.g == 64) return run_bwd_stream<Q, WT, 64>(sh, W, p, codes, gup, gr, st);
+    return run_bwd_stream<Q, WT, 128>(sh, W, p, codes, gup, gr, st);
+}
+
+template <int Q, typename WT>
+static cudaError_t fwd_stream_g(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                                float* what, cudaStream_t st) {
+    if (sh.g == 32) return run_fwd_stream<Q, WT, 32>(sh, W, p, codes, mode, what, st);
+    if (sh.g == 64) return run_fwd_stream<Q, WT, 64>(sh, W, p, codes, mode, what, st);
+    return run_fwd_stream<Q, WT, 128>(sh, W, p, codes, mode, what, st);
+}
+
+template <int Q>
+static cudaError_t bwd_stream_w(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
+                                const float* gup, uq_grads gr, cudaStream_t st) {
+    if (sh.wdtype == UQ_W_BF16) return bwd_stream_g<Q, WBF16>(sh, W, p, codes, gup, gr, st);
+    return bwd_stream_g<Q, WF32>(sh, W, p, codes, gup, gr, st);
+}
+
+template <int Q>
+static cudaError_t fwd_stream_w(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                                float* what, cudaStream_t st) {
+    if (sh.wdtype == UQ_W_BF16) return fwd_stream_g<Q, WBF16>(sh, W, p, codes, mode, what, st);
+    return fwd_stream_g<Q, WF32>(sh, W, p, codes, mode, what, st);
+}
+
+cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
+                              uq_grads gr, cudaStream_t st) {
+    switch (sh.q) {
+        case 1: return bwd_stream_w<1>(sh, W, p, codes, gup, gr, st);
+        case 2: return bwd_stream_w<2>(sh, W, p, codes, gup, gr, st);
+        case 3: return bwd_stream_w<3>(sh, W, p, codes, gup, gr, st);
+        default: return bwd_stream_w<4>(sh, W, p, codes, gup, gr, st);
+    }
+}
+
+cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode, float* what,
+                              cudaStream_t st) {
+    switch (sh.q) {
+        case 1: return fwd_stream_w<1>(sh, W, p, codes, mode, what, st);
+        case 2: return fwd_stream_w<2>(sh, W, p, codes, mode, what, st);
+        case 3: return fwd_stream_w<3>(sh, W, p, codes, mode, what, st);
+        default: return fwd_stream_w<4>(sh, W, p, codes, mode, what, st);
+    }
+}
+
+cudaError_t stream_error(bool clear, unsigned int* flag) {
+    unsigned int v = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_stream_err, sizeof(v));
+    if (e != cudaSuccess) return e;
+    *flag = v;
+    if (clear && v) {
+        const unsigned int z = 0;
+        e = cudaMemcpyToSymbol(g_stream_err, &z, sizeof(z));
+    }
+    return e;
+}
+
+}  // namespace uq
