@@ -9,10 +9,11 @@
 // the warp computes from shared memory while the copies of the next units
 // are in flight.  Thread blocks are persistent: block b handles row blocks
 // b, b + gridDim.x, ...; within a row block the warps split the row's units
-// as in the non-pipelined kernels, and one block barrier per row block
-// orders the ds_r sum.  Every mbarrier wait is bounded (about one second of
+// as in the non-pipelined kernels.  Every mbarrier wait is bounded (about one second of
 // GPU clock); a wait that runs out sets g_stream_err, which
-// uq_check_device() reports, and the warp stops computing.
+// uq_check_device() reports, and the warp stops computing.  The backward
+// kernel's ds_r partials wait in a shared-memory ring of kRowRing row
+// blocks, summed in warp order after one block barrier per ring.
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
@@ -71,24 +72,52 @@ __device__ __forceinline__ void copy_g2s(uint32_t dst, const void* src, uint32_t
 
 constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
-// Shared-memory stage layout of one work unit.
-template <int Q, typename WT, int G_>
+// Shared memory per warp for its stages, and the resident blocks per SM the
+// register allocation is bounded for (backward; forward).
+#ifndef UQ_BWD_STAGE_BYTES
+#define UQ_BWD_STAGE_BYTES 11520
+#endif
+#ifndef UQ_FWD_STAGE_BYTES
+#define UQ_FWD_STAGE_BYTES 5632
+#endif
+#ifndef UQ_STREAM_BWD_MIN_BLOCKS
+#define UQ_STREAM_BWD_MIN_BLOCKS 2
+#endif
+#ifndef UQ_STREAM_FWD_MIN_BLOCKS
+#define UQ_STREAM_FWD_MIN_BLOCKS 4
+#endif
+constexpr int kMaxStages = 16;
+constexpr int kRowRing = 32;             // row blocks whose ds_r partials wait in shared memory
+
+// Shared-memory stage layout of one work unit.  HAS_X: weights and s are
+// staged; HAS_G: dL/dW^ is staged; HAS_C: code words are staged.  The group
+// parameters (Delta, z_U, z_B, alpha of the unit's NG groups) always are.
+template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET>
 struct Stage {
     static constexpr int LPG = G_ <= 64 ? 4 : 8;
     static constexpr int NG = 32 / LPG;                  // groups per unit
     static constexpr int NV = G_ / (4 * LPG);            // vectors per lane
     static constexpr int UE = NG * G_;                   // elements per unit
     static constexpr int WBYTES = sizeof(typename WT::raw) / 4;
-    static constexpr int SZ_W = UE * WBYTES, SZ_F = UE * 4, SZ_C = UE, SZ_P = NG * 4, SZ_A = NG * Q * 4;
+    static constexpr int SZ_W = HAS_X ? UE * WBYTES : 0;
+    static constexpr int SZ_S = HAS_X ? UE * 4 : 0;
+    static constexpr int SZ_G = HAS_G ? UE * 4 : 0;
+    static constexpr int SZ_C = HAS_C ? UE : 0;
+    static constexpr int SZ_P = NG * 4, SZ_A = NG * Q * 4;
     static constexpr int OFF_W = 0;
     static constexpr int OFF_S = align_up(OFF_W + SZ_W, 16);
-    static constexpr int OFF_G = OFF_S + SZ_F;
-    static constexpr int OFF_C = OFF_G + SZ_F;
+    static constexpr int OFF_G = OFF_S + SZ_S;
+    static constexpr int OFF_C = OFF_G + SZ_G;
     static constexpr int OFF_D = align_up(OFF_C + SZ_C, 16);
     static constexpr int OFF_Z = OFF_D + SZ_P;
     static constexpr int OFF_B = OFF_Z + SZ_P;
     static constexpr int OFF_A = OFF_B + SZ_P;
     static constexpr int BYTES = align_up(OFF_A + SZ_A, 128);
+    static constexpr uint32_t TX = SZ_W + SZ_S + SZ_G + SZ_C + 3 * SZ_P + SZ_A;   // bytes copied per unit
+    // stages per warp within the per-warp shared-memory budget
+    static constexpr int FIT = BUDGET / BYTES;
+    static constexpr int NST = FIT < 2 ? 2 : (FIT > kMaxStages ? kMaxStages : FIT);
+    static constexpr int WARP_BYTES = NST * BYTES;
     static_assert(SZ_P % 16 == 0 && SZ_A % 16 == 0 && SZ_C % 16 == 0, "bulk copy sizes must be multiples of 16");
 };
 
@@ -116,29 +145,29 @@ struct Items {
 // Backward
 // ---------------------------------------------------------------------------
 
-template <int Q, typename WT, int G_, int NST>
-__global__ void __launch_bounds__(kThreads, 2)
+template <int Q, typename WT, int G_>
+__global__ void __launch_bounds__(kThreads, UQ_STREAM_BWD_MIN_BLOCKS)
 bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
                   const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
                   const float* __restrict__ ZB, const uint8_t* __restrict__ CODES, const float* __restrict__ GUP,
                   float* __restrict__ DS, float* __restrict__ DSR, float* __restrict__ DDELTA,
                   float* __restrict__ DZU, float* __restrict__ DZB, float* __restrict__ DALPHA, int64_t out,
                   int n_in, int R, int n_rb) {
-    using St = Stage<Q, WT, G_>;
-    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE;
-    constexpr uint32_t TX = St::SZ_W + 2 * St::SZ_F + St::SZ_C + 3 * St::SZ_P + St::SZ_A;
+    using St = Stage<Q, WT, G_, true, true, true, UQ_BWD_STAGE_BYTES>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
+    constexpr uint32_t TX = St::TX;
     using SR8 = SegReduce<LPG>;
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
-    __shared__ LvTab<Q, NG> tabs[kWarps];
+    __shared__ float2 tabs[kWarps][NG][L];          // (l(c), l(c) - z_U) per group slot and code word
     __shared__ float tau_s[kWarps][NG];
-    __shared__ float red[2][kWarps];
+    __shared__ float red[kRowRing][kWarps];       // per row block and warp: sum of Delta S3
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
     const Items it(U, R, n_rb, warp);
-    unsigned char* wsm = smem + (size_t)warp * NST * St::BYTES;
-    LvTab<Q, NG>& t = tabs[warp];
+    unsigned char* wsm = smem + (size_t)warp * St::WARP_BYTES;
+    float2 (*t)[L] = tabs[warp];
 
     if (lane == 0) {
         for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
@@ -157,8 +186,8 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         tma::fence_async_smem();
         tma::bar_arrive_tx(bar, TX);
         tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
-        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_F, bar);
-        tma::copy_g2s(d + St::OFF_G, GUP + e0, St::SZ_F, bar);
+        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
+        tma::copy_g2s(d + St::OFF_G, GUP + e0, St::SZ_G, bar);
         tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
         tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
@@ -197,7 +226,8 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     float a[Q];
 #pragma unroll
                     for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
-                    t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+                    const float lvc = level_of<Q>(c, a, pb[kk]);
+                    t[kk][c] = make_float2(lvc, lvc - pz[kk]);
                     if (c == 0) {
                         float m = fabsf(a[0]);
 #pragma unroll
@@ -223,14 +253,15 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 #pragma unroll
                     for (int kq = 0; kq < 4; ++kq) {
                         const int c = (cv >> (8 * kq)) & (L - 1);
-                        const float m = t.lv[sub][c];
+                        const float2 mm = t[sub][c];
+                        const float m = mm.x;
                         float uu;
                         const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
                         const bool f = fabsf(__fsub_rn(x, m)) <= tau;
                         const float fu = f ? uu : 0.f;
                         const float gfu = G[kq] * fu;
                         ds[kq] = -__fdividef(dl * gfu, s4[kq]);
-                        acc[0] += G[kq] * ((m - zu) - fu);
+                        acc[0] += G[kq] * (mm.y - fu);
                         acc[1] += f ? 0.f : G[kq];
                         acc[2] += G[kq];
                         acc[3] += gfu;
@@ -258,16 +289,23 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
             if (alive && lane == 0 && i + NST < it.total) issue(i + NST);
         }
         prow = warp_sum(prow);
-        if (lane == 0) red[k & 1][warp] = prow;
-        __syncthreads();
-        if (threadIdx.x < R) {
-            const int64_t r = rb * R + threadIdx.x;
-            if (r < out) {
-                const int WPR = kWarps / R;
-                float s = red[k & 1][threadIdx.x * WPR];
-                for (int w = 1; w < WPR; ++w) s += red[k & 1][threadIdx.x * WPR + w];
-                DSR[r] = -s / __ldg(SR + r);
+        if (lane == 0) red[k % kRowRing][warp] = prow;
+        // ds_r of the last kRowRing row blocks, once the ring is full or at the end
+        if (k % kRowRing == kRowRing - 1 || k == n_mine - 1) {
+            __syncthreads();
+            const int k0 = k - k % kRowRing;
+            const int WPR = kWarps / R;
+            for (int idx = threadIdx.x; idx < (k - k0 + 1) * R; idx += kThreads) {
+                const int kk = k0 + idx / R, rsub = idx % R;
+                const int64_t r = ((int64_t)blockIdx.x + (int64_t)kk * gridDim.x) * R + rsub;
+                if (r < out) {
+                    const float* rr = red[kk % kRowRing];
+                    float s = rr[rsub * WPR];
+                    for (int w = 1; w < WPR; ++w) s += rr[rsub * WPR + w];
+                    DSR[r] = -s / __ldg(SR + r);
+                }
             }
+            __syncthreads();
         }
     }
 }
@@ -276,14 +314,16 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // Forward
 // ---------------------------------------------------------------------------
 
-template <int Q, typename WT, int G_, int NST>
-__global__ void __launch_bounds__(kThreads, 2)
+template <int Q, typename WT, int G_, int MODE>
+__global__ void __launch_bounds__(kThreads, UQ_STREAM_FWD_MIN_BLOCKS)
 fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
                   const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
                   const float* __restrict__ ZB, uint8_t* __restrict__ CODES, float* __restrict__ WHAT,
-                  int64_t out, int n_in, int R, int n_rb, int mode) {
-    using St = Stage<Q, WT, G_>;
-    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE;
+                  int64_t out, int n_in, int R, int n_rb) {
+    constexpr int mode = MODE;
+    constexpr bool need_x = MODE != FWD_KEEP, need_c = MODE != FWD_FULL;
+    using St = Stage<Q, WT, G_, need_x, false, need_c, UQ_FWD_STAGE_BYTES>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ MapTab<Q, NG> tabs[kWarps];
@@ -291,10 +331,9 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
     const Items it(U, R, n_rb, warp);
-    unsigned char* wsm = smem + (size_t)warp * NST * St::BYTES;
+    unsigned char* wsm = smem + (size_t)warp * St::WARP_BYTES;
     MapTab<Q, NG>& t = tabs[warp];
-    const bool need_x = mode != FWD_KEEP, need_c = mode != FWD_FULL;
-    const uint32_t TX = (need_x ? St::SZ_W + St::SZ_F : 0) + (need_c ? St::SZ_C : 0) + 3 * St::SZ_P + St::SZ_A;
+    constexpr uint32_t TX = St::TX;
 
     if (lane == 0) {
         for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
@@ -312,11 +351,11 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
         tma::fence_async_smem();
         tma::bar_arrive_tx(bar, TX);
-        if (need_x) {
+        if constexpr (need_x) {
             tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
-            tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_F, bar);
+            tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
         }
-        if (need_c) tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+        if constexpr (need_c) tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
         tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
@@ -347,13 +386,13 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
             }
             __syncwarp();
-            if (mode == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
-            else if (mode == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            if constexpr (mode == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
+            else if constexpr (mode == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
             const float dl = pd[sub], zu = pz[sub];
             const float sr = need_x ? __ldg(SR + row) : 0.f;
             const int64_t ebase = row * n_in + (int64_t)it.unit_of(i) * UE;
             float srt[L];
-            if (mode == FWD_FULL) {
+            if constexpr (mode == FWD_FULL) {
 #pragma unroll
                 for (int r = 0; r < L; ++r) srt[r] = t.srt[sub][r];
             }
@@ -362,8 +401,9 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 const int el = sub * G_ + 4 * li + 4 * LPG * v;
                 float o[4];
                 uint32_t nc = 0;
-                const uint32_t cv = need_c ? *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el) : 0u;
-                if (mode == FWD_KEEP) {
+                uint32_t cv = 0u;
+                if constexpr (need_c) cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+                if constexpr (mode == FWD_KEEP) {
 #pragma unroll
                     for (int kq = 0; kq < 4; ++kq) {
                         const int c = (cv >> (8 * kq)) & (L - 1);
@@ -373,7 +413,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     float w[4], s4[4];
                     WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
-                    if (mode == FWD_REMAP) {
+                    if constexpr (mode == FWD_REMAP) {
 #pragma unroll
                         for (int kq = 0; kq < 4; ++kq) {
                             const int c = (cv >> (8 * kq)) & (L - 1);
@@ -415,8 +455,6 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // Launchers
 // ---------------------------------------------------------------------------
 
-constexpr int kStreamStages = 2;
-
 static int sm_count() {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 1;
@@ -446,12 +484,12 @@ static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
 template <int Q, typename WT, int G_>
 static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
                                   const float* gup, uq_grads gr, cudaStream_t st) {
-    using St = Stage<Q, WT, G_>;
+    using St = Stage<Q, WT, G_, true, true, true, UQ_BWD_STAGE_BYTES>;
     const int U = sh.n_in / St::UE;
     const int R = rows_per_block(U);
     const int n_rb = (int)((sh.out + R - 1) / R);
-    const size_t dyn = (size_t)kWarps * kStreamStages * St::BYTES;
-    auto kern = bwd_stream_kernel<Q, WT, G_, kStreamStages>;
+    const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
+    auto kern = bwd_stream_kernel<Q, WT, G_>;
     int grid = 0;
     cudaError_t e = grid_for(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
@@ -460,21 +498,29 @@ static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, c
     return cudaGetLastError();
 }
 
-template <int Q, typename WT, int G_>
-static cudaError_t run_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
-                                  float* what, cudaStream_t st) {
-    using St = Stage<Q, WT, G_>;
+template <int Q, typename WT, int G_, int MODE>
+static cudaError_t run_fwd_stream_mode(const Shape& sh, const void* W, uq_params p, uint8_t* codes, float* what,
+                                       cudaStream_t st) {
+    using St = Stage<Q, WT, G_, MODE != FWD_KEEP, false, MODE != FWD_FULL, UQ_FWD_STAGE_BYTES>;
     const int U = sh.n_in / St::UE;
     const int R = rows_per_block(U);
     const int n_rb = (int)((sh.out + R - 1) / R);
-    const size_t dyn = (size_t)kWarps * kStreamStages * St::BYTES;
-    auto kern = fwd_stream_kernel<Q, WT, G_, kStreamStages>;
+    const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
+    auto kern = fwd_stream_kernel<Q, WT, G_, MODE>;
     int grid = 0;
     cudaError_t e = grid_for(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R,
-                                      n_rb, mode);
+                                      n_rb);
     return cudaGetLastError();
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t run_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
+                                  float* what, cudaStream_t st) {
+    if (mode == FWD_KEEP) return run_fwd_stream_mode<Q, WT, G_, FWD_KEEP>(sh, W, p, codes, what, st);
+    if (mode == FWD_REMAP) return run_fwd_stream_mode<Q, WT, G_, FWD_REMAP>(sh, W, p, codes, what, st);
+    return run_fwd_stream_mode<Q, WT, G_, FWD_FULL>(sh, W, p, codes, what, st);
 }
 
 template <int Q, typename WT>

@@ -213,3 +213,30 @@ def test_side_stream_and_error_leaves_outputs_untouched():
     assert ei.value.status == api.UQ_ERR_UNSUPPORTED
     torch.cuda.synchronize()
     assert torch.all(what == 3.0) and torch.equal(cd.cpu(), torch.from_numpy(codes0))
+
+
+def test_device_check_reports_no_timeouts_after_normal_work():
+    """The pipelined kernels bound every wait; after ordinary calls no wait ran
+    out and uq_check_device reports OK (and synchronises the stream)."""
+    q, g, out, n_in = 3, 128, 64, 2048
+    raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=21)
+    what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+    gr = C.gpu_bwd(raw, P, codes, Gup, q, g)
+    api.uq_check_device()
+    assert api.uq_last_error() == ""
+
+
+@pytest.mark.parametrize("n_in,g", [(512, 128), (2048, 64), (768, 32), (1536, 128), (384, 128)])
+def test_pipelined_and_plain_paths_agree_across_shapes(n_in, g):
+    """Rows that split into whole 512-element units (256 for g = 32) take the
+    pipelined kernels, others the per-row kernels; both match the oracle,
+    including short rows packed several to a block and a ragged last block."""
+    q, out = 3, 21
+    raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=n_in + g)
+    what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(what, codes, r_what, r_codes, f"n_in={n_in} g={g}")
+    gr = C.gpu_bwd(raw, P, codes, Gup, q, g)
+    ref, mass = C.oracle_bwd(W, P, r_codes, Gup, g)
+    C.assert_grads_close(gr, ref, mass, f"n_in={n_in} g={g}")
