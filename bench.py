@@ -128,7 +128,7 @@ def measured_peaks():
 
 def kernel_hash():
     h = hashlib.sha256()
-    for f in ("uq_bwd.cu", "uq_common.cuh"):
+    for f in ("uq_stream.cu", "uq_common.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2506_03781_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -356,7 +356,7 @@ def run_gpu(args):
                        "l2": "inputs larger than L2 (about 1.5 GB moved per step vs 129 MB L2)",
                        "step_bytes_avg": step_bytes / args.steps,
                        "hbm_gbs_step": step_bytes / secs / 1e9 * world},
-            "roofline": {"bound": "hbm", "kernel": "uq_bwd", "achieved": achieved, "peak": peak,
+            "roofline": {"bound": "hbm", "kernel": "bwd_stream_kernel", "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak,
                          "traffic": recorded_traffic(wl.name, q),
                          "algorithmic_bytes": bwd_bytes, "avg_ms": bwd_avg_s * 1e3,
