@@ -305,3 +305,66 @@ class HostStep:
             host_out["codes"].copy_(self.dev["codes"], non_blocking=True)
             for k in GRAD_NAMES:
                 host_out[k].copy_(self.grads[k], non_blocking=True)
+
+
+class HostPipeline:
+    """Overlapped quantizer steps on HOST buffers, through the C ABI.
+
+    ``submit`` queues one step: the host-to-device copies of its inputs on an
+    upload stream, ``uq_quantize_fwd`` + ``uq_quantize_bwd`` on a compute
+    stream and the device-to-host copies of its results on a download
+    stream, ordered by CUDA events.  ``depth`` device buffer sets are used in
+    turn, so a step's uploads overlap the previous steps' compute and
+    downloads (the two copy directions run concurrently).  Steps submitted
+    back to back must be independent -- e.g. different weight matrices of a
+    model -- because a step's host inputs are read when its upload starts.
+    Host tensors should be pinned; ``synchronize`` waits for every step.
+    """
+
+    def __init__(self, out, n_in, q, g, w_dtype=torch.bfloat16, device="cuda", depth=2):
+        self.steps = [HostStep(out, n_in, q, g, w_dtype, device, stream=None) for _ in range(depth)]
+        dev = torch.device(device)
+        self.up = torch.cuda.Stream(dev)
+        self.comp = torch.cuda.Stream(dev)
+        self.down = torch.cuda.Stream(dev)
+        self.ev = [{k: torch.cuda.Event() for k in ("up", "comp", "down")} for _ in range(depth)]
+        self.n = 0
+
+    def empty_host(self, pinned=True):
+        return self.steps[0].empty_host(pinned)
+
+    def bytes_in(self, host_in):
+        return self.steps[0].bytes_in(host_in)
+
+    def bytes_out(self, host_out):
+        return self.steps[0].bytes_out(host_out)
+
+    def submit(self, host_in, host_out, step, p_period=2, map_mode=MAP_LOCAL_PERIODIC):
+        k = self.n % len(self.steps)
+        hs, ev = self.steps[k], self.ev[k]
+        dev = {**hs.dev, **hs.params}
+        # inputs of this buffer set are free once the compute that read them is done
+        self.up.wait_event(ev["comp"])
+        with torch.cuda.stream(self.up):
+            for name in HostStep.IN_KEYS:
+                dev[name].copy_(host_in[name], non_blocking=True)
+        ev["up"].record(self.up)
+        # outputs of this buffer set are free once their download is done
+        self.comp.wait_event(ev["up"])
+        self.comp.wait_event(ev["down"])
+        uq_quantize_fwd(hs.dev["W"], hs.q, hs.g, hs.params, hs.dev["codes"], hs.dev["W_hat"], map_mode, step,
+                        p_period, stream=self.comp)
+        uq_quantize_bwd(hs.dev["W"], hs.q, hs.g, hs.params, hs.dev["codes"], hs.dev["dL_dWhat"], hs.grads,
+                        stream=self.comp)
+        ev["comp"].record(self.comp)
+        self.down.wait_event(ev["comp"])
+        with torch.cuda.stream(self.down):
+            host_out["W_hat"].copy_(hs.dev["W_hat"], non_blocking=True)
+            host_out["codes"].copy_(hs.dev["codes"], non_blocking=True)
+            for name in GRAD_NAMES:
+                host_out[name].copy_(hs.grads[name], non_blocking=True)
+        ev["down"].record(self.down)
+        self.n += 1
+
+    def synchronize(self):
+        self.down.synchronize()

@@ -24,10 +24,7 @@ namespace uq {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kVec = 4;                     // elements per lane per warp-step
-constexpr int kStep = 32 * kVec;            // 128 elements per warp-step
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kSlots = 4;                   // group tables per warp and batch
 
 // Weight-storage adaptors: 4 consecutive weights per lane.
 struct WF32 {
@@ -72,83 +69,6 @@ __device__ __forceinline__ float level_of(int c, const float a[Q], float zb) {
     return __fadd_rn(acc, zb);
 }
 
-// Per-warp group tables: levels by code word, sorted levels, code of each
-// rank, rank of each code, and for the local mapping the (lower, own, upper)
-// neighbour levels with the neighbours' code words packed in .w.
-template <int Q>
-struct GroupTables {
-    static constexpr int L = 1 << Q;
-    float lv[kSlots][L];
-    float srt[kSlots][L];
-    float4 nb[kSlots][L];
-    float tau[kSlots];
-    uint8_t cor[kSlots][L];
-    uint8_t rk[kSlots][L];
-};
-
-// Builds the tables of up to kSlots groups (slot k -> group grp_of_slot(k),
-// valid if ok_of_slot(k)).  Whole warp; ends with __syncwarp().
-// Levels come from (alpha, z_B) by level_of; the rank of code c is the
-// number of codes whose level is smaller, or equal with a smaller code word
-// (the stable ascending order).
-template <int Q, bool NEED_SORT, bool NEED_NB, typename GrpFn, typename OkFn>
-__device__ __forceinline__ void build_tables(GroupTables<Q>& t, int lane, const float* __restrict__ alpha,
-                                             const float* __restrict__ zb, GrpFn grp_of_slot, OkFn ok_of_slot) {
-    constexpr int L = 1 << Q;
-    constexpr int E = kSlots * L;
-#pragma unroll
-    for (int e = lane; e < E; e += 32) {
-        const int k = e / L, c = e % L;
-        float lvv = 0.f;
-        if (ok_of_slot(k)) {
-            const int64_t grp = grp_of_slot(k);
-            float a[Q];
-#pragma unroll
-            for (int j = 0; j < Q; ++j) a[j] = __ldg(alpha + grp * Q + j);
-            lvv = level_of<Q>(c, a, __ldg(zb + grp));
-            if (c == 0) {
-                float m = fabsf(a[0]);
-#pragma unroll
-                for (int j = 1; j < Q; ++j) m = fminf(m, fabsf(a[j]));
-                t.tau[k] = m;
-            }
-        } else if (c == 0) {
-            t.tau[k] = 0.f;
-        }
-        t.lv[k][c] = lvv;
-    }
-    __syncwarp();
-    if constexpr (NEED_SORT) {
-#pragma unroll
-        for (int e = lane; e < E; e += 32) {
-            const int k = e / L, c = e % L;
-            const float v = t.lv[k][c];
-            int r = 0;
-#pragma unroll
-            for (int c2 = 0; c2 < L; ++c2) {
-                const float v2 = t.lv[k][c2];
-                r += (v2 < v) || (v2 == v && c2 < c);
-            }
-            t.srt[k][r] = v;
-            t.cor[k][r] = static_cast<uint8_t>(c);
-            t.rk[k][c] = static_cast<uint8_t>(r);
-        }
-        __syncwarp();
-    }
-    if constexpr (NEED_NB) {
-#pragma unroll
-        for (int e = lane; e < E; e += 32) {
-            const int k = e / L, c = e % L;
-            const int r = t.rk[k][c];
-            const int rl = r > 0 ? r - 1 : 0;
-            const int rh = r < L - 1 ? r + 1 : L - 1;
-            const uint32_t packed = uint32_t(t.cor[k][rl]) | (uint32_t(t.cor[k][rh]) << 8);
-            t.nb[k][c] = make_float4(t.srt[k][rl], t.lv[k][c], t.srt[k][rh], __uint_as_float(packed));
-        }
-        __syncwarp();
-    }
-}
-
 // Full mapping M_B over the sorted levels held in registers: argmin over
 // ranks of |x - l|, first (lowest) rank wins ties.  Returns the rank; m is
 // the chosen level.
@@ -163,34 +83,6 @@ __device__ __forceinline__ int nearest_rank(float x, const float srt[L], float& 
         if (d < best) { best = d; br = r; m = srt[r]; }
     }
     return br;
-}
-
-// Segmented reduce-scatter of 8 partial sums over SEGL consecutive lanes
-// (SEGL = 8, 16 or 32).  Three butterfly levels halve the number of live
-// values (8 -> 4 -> 2 -> 1) while exchanging the other half with the
-// partner lane; the remaining levels sum the single value.  On return the
-// lane holds the segment-wide total of slot `slot`; lanes whose index is a
-// multiple of SEGL/8 hold distinct slots 0..7.  Fixed order: deterministic.
-template <int SEGL>
-__device__ __forceinline__ float seg_reduce8(float v[8], int lane, int& slot) {
-    int base = 0;
-#pragma unroll
-    for (int lvl = 0; lvl < 3; ++lvl) {
-        const int off = SEGL >> (lvl + 1);
-        const int h = 4 >> lvl;
-        const bool up = (lane & off) != 0;
-#pragma unroll
-        for (int i = 0; i < h; ++i) {
-            const float send = up ? v[i] : v[i + h];
-            const float keep = up ? v[i + h] : v[i];
-            v[i] = keep + __shfl_xor_sync(kFull, send, off);
-        }
-        base += up ? h : 0;
-    }
-#pragma unroll
-    for (int off = SEGL >> 4; off >= 1; off >>= 1) v[0] += __shfl_xor_sync(kFull, v[0], off);
-    slot = base;
-    return v[0];
 }
 
 __device__ __forceinline__ float warp_sum(float v) {

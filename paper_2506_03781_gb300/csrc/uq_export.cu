@@ -1,162 +1,128 @@
 // Export: unification theorem (Theorem 1) and bit-plane packing of the
-// final binary codes (Algorithm 1, lines 10-11), one thread block per row.
+// final binary codes (Algorithm 1, lines 10-11).
 //
 // alpha* = Delta alpha, z_B* = Delta (z_B - z_U) per group.  The codes are
 // the stored ones (REUSE) or the nearest level of Theta_B* to each original
-// weight (Eq. 4).  Packing: a lane holds 4 consecutive code words; for each
-// 32-column word of a warp-step, one shuffle gives every lane the code of
-// its column and one __ballot_sync per bit j yields the 32-bit word of
-// plane j.  HBM traffic per element: 1 (or 2 for Eq. 4 with bf16 W) read,
-// q/8 written, plus (q+1)*4/g each way for the group parameters.
+// weight (Eq. 4).  One thread owns 32 consecutive columns of a row (one
+// 32-bit word of every bit-plane): it reads their 32 code bytes with two
+// 16-byte loads and gathers bit j of four bytes at a time with the
+// carry-free product ((x >> j) & 0x01010101) * 0x01020408, whose top byte
+// holds the four bits in order.  Consecutive threads write consecutive
+// words.  HBM traffic per element: 1 (codes) or 2-4 (weights) read, q/8
+// written, plus the group parameters.
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
 namespace uq {
 
-template <int Q, typename WT, int GPS, bool EQ4>
+__device__ __forceinline__ uint32_t gather_bit(uint32_t four_codes, int j) {
+    return (((four_codes >> j) & 0x01010101u) * 0x01020408u) >> 24;
+}
+
+template <int Q, typename WT, bool EQ4>
 __global__ void __launch_bounds__(kThreads)
 export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const float* __restrict__ ZU,
               const float* __restrict__ ALPHA, const float* __restrict__ ZB, const uint8_t* __restrict__ CODES,
               uint32_t* __restrict__ PLANES, float* __restrict__ ASTAR, float* __restrict__ ZSTAR, int64_t out,
               int n_in, int g) {
     constexpr int L = 1 << Q;
-    constexpr int WB = kSlots / GPS;
-    constexpr int SH = GPS == 4 ? 3 : (GPS == 2 ? 4 : 5);
-    constexpr uint32_t kMask = (uint32_t(L - 1) * 0x01010101u);
-    __shared__ GroupTables<Q> tabs[kWarps];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    GroupTables<Q>& t = tabs[warp];
-    const int64_t row = blockIdx.x;
-    const int n_ws = (n_in + kStep - 1) / kStep;
-    const int Gr = n_in / g;
+    constexpr uint32_t kMask = uint32_t(L - 1) * 0x01010101u;
     const int words = n_in / 32;
-    const int64_t eoff = row * (int64_t)n_in;
-    const int64_t goff = row * (int64_t)Gr;
+    const int Gr = n_in / g;
+    const int64_t nthr = (int64_t)gridDim.x * blockDim.x;
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
 
-    // Theorem 1 for every group of the row.
-    for (int gi = threadIdx.x; gi < Gr; gi += kThreads) {
-        const int64_t grp = goff + gi;
+    // Theorem 1 for every group.
+    for (int64_t grp = tid; grp < out * Gr; grp += nthr) {
         const float d = __ldg(DELTA + grp);
 #pragma unroll
         for (int j = 0; j < Q; ++j) ASTAR[grp * Q + j] = __fmul_rn(d, __ldg(ALPHA + grp * Q + j));
         ZSTAR[grp] = __fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp)));
     }
 
-    for (int base = warp; base < n_ws; base += kWarps * WB) {
-        uint32_t cw[WB];
-        typename WT::raw wraw[WB];
-        bool ok[WB];
-        int col[WB];
+    for (int64_t ch = tid; ch < out * words; ch += nthr) {
+        const int64_t row = ch / words;
+        const int wcol = (int)(ch - row * words);
+        const int64_t e0 = row * n_in + (int64_t)wcol * 32;
+        uint32_t cw[8];
+        if constexpr (!EQ4) {
+            const uint4 a = __ldg(reinterpret_cast<const uint4*>(CODES + e0));
+            const uint4 b = __ldg(reinterpret_cast<const uint4*>(CODES + e0 + 16));
+            cw[0] = a.x & kMask; cw[1] = a.y & kMask; cw[2] = a.z & kMask; cw[3] = a.w & kMask;
+            cw[4] = b.x & kMask; cw[5] = b.y & kMask; cw[6] = b.z & kMask; cw[7] = b.w & kMask;
+        } else {
+            // Levels of Theta_B* of this chunk's group (the fp32 values written above).
+            const int64_t grp = row * Gr + (wcol * 32) / g;
+            const float d = __ldg(DELTA + grp);
+            float a[Q];
 #pragma unroll
-        for (int b = 0; b < WB; ++b) {
-            const int ws = base + b * kWarps;
-            col[b] = ws * kStep + lane * kVec;
-            ok[b] = ws < n_ws && col[b] < n_in;
-            cw[b] = 0;
-            if (ok[b]) {
-                if constexpr (EQ4) wraw[b] = WT::load(W, eoff + col[b]);
-                else cw[b] = __ldg(reinterpret_cast<const unsigned int*>(CODES + eoff + col[b])) & kMask;
-            }
-        }
-        if constexpr (EQ4) {
-            // Levels of Theta_B*: the same fp32 alpha*, z_B* as written above.
-            auto ok_of_slot = [&](int k) -> bool {
-                const int ws = base + (k / GPS) * kWarps;
-                return ws < n_ws && (ws * kStep) / g + (k % GPS) < Gr;
-            };
-            __syncwarp();
-            constexpr int E = kSlots * L;
+            for (int j = 0; j < Q; ++j) a[j] = __fmul_rn(d, __ldg(ALPHA + grp * Q + j));
+            const float zs = __fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp)));
+            float lv[L];
+            int rk[L];
 #pragma unroll
-            for (int e = lane; e < E; e += 32) {
-                const int k = e / L, c = e % L;
-                float lvv = 0.f;
-                if (ok_of_slot(k)) {
-                    const int64_t grp = goff + ((base + (k / GPS) * kWarps) * kStep) / g + (k % GPS);
-                    const float d = __ldg(DELTA + grp);
-                    float a[Q];
+            for (int c = 0; c < L; ++c) lv[c] = level_of<Q>(c, a, zs);
 #pragma unroll
-                    for (int j = 0; j < Q; ++j) a[j] = __fmul_rn(d, __ldg(ALPHA + grp * Q + j));
-                    lvv = level_of<Q>(c, a, __fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp))));
-                }
-                t.lv[k][c] = lvv;
-            }
-            __syncwarp();
-#pragma unroll
-            for (int e = lane; e < E; e += 32) {
-                const int k = e / L, c = e % L;
-                const float v = t.lv[k][c];
+            for (int c = 0; c < L; ++c) {
                 int r = 0;
 #pragma unroll
-                for (int c2 = 0; c2 < L; ++c2) {
-                    const float v2 = t.lv[k][c2];
-                    r += (v2 < v) || (v2 == v && c2 < c);
-                }
-                t.srt[k][r] = v;
-                t.cor[k][r] = static_cast<uint8_t>(c);
+                for (int c2 = 0; c2 < L; ++c2) r += (lv[c2] < lv[c]) || (lv[c2] == lv[c] && c2 < c);
+                rk[c] = r;
             }
-            __syncwarp();
 #pragma unroll
-            for (int b = 0; b < WB; ++b) {
-                if (!ok[b]) continue;
-                const int k = b * GPS + (lane >> SH);
-                float srt[L], w[4];
+            for (int v = 0; v < 8; ++v) {
+                float w[4];
+                WT::unpack(WT::load(W, e0 + 4 * v), w);
+                uint32_t packed = 0;
 #pragma unroll
-                for (int r = 0; r < L; ++r) srt[r] = t.srt[k][r];
-                WT::unpack(wraw[b], w);
+                for (int k = 0; k < 4; ++k) {
+                    // nearest level, ties to the lower rank (same result as a scan of the sorted levels)
+                    float best = fabsf(__fsub_rn(w[k], lv[0]));
+                    int bc = 0, br = rk[0];
 #pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    float m;
-                    const int r = nearest_rank<L>(w[v], srt, m);
-                    cw[b] |= uint32_t(t.cor[k][r]) << (8 * v);
+                    for (int c = 1; c < L; ++c) {
+                        const float dd = fabsf(__fsub_rn(w[k], lv[c]));
+                        if (dd < best || (dd == best && rk[c] < br)) { best = dd; bc = c; br = rk[c]; }
+                    }
+                    packed |= uint32_t(bc) << (8 * k);
                 }
+                cw[v] = packed;
             }
         }
 #pragma unroll
-        for (int b = 0; b < WB; ++b) {
-            const int ws = base + b * kWarps;
-            if (ws >= n_ws) break;                           // warp-uniform
-            uint32_t mine = 0;
+        for (int j = 0; j < Q; ++j) {
+            uint32_t word = 0;
 #pragma unroll
-            for (int tw = 0; tw < 4; ++tw) {
-                // column 32*tw + lane of this warp-step lives in lane 8*tw + lane/4, byte lane%4
-                const uint32_t v = (__shfl_sync(kFull, cw[b], 8 * tw + (lane >> 2)) >> (8 * (lane & 3))) & 0xffu;
-#pragma unroll
-                for (int j = 0; j < Q; ++j) {
-                    const uint32_t word = __ballot_sync(kFull, (v >> j) & 1u);
-                    if (lane == j * 4 + tw) mine = word;
-                }
-            }
-            if (lane < 4 * Q) {
-                const int j = lane >> 2, tw = lane & 3;
-                const int wcol = ws * kStep + tw * 32;
-                if (wcol < n_in) PLANES[((int64_t)j * out + row) * words + ws * 4 + tw] = mine;
-            }
+            for (int v = 0; v < 8; ++v) word |= gather_bit(cw[v], j) << (4 * v);
+            PLANES[((int64_t)j * out + row) * words + wcol] = word;
         }
     }
 }
 
-template <int Q, typename WT, int GPS, bool EQ4>
-static cudaError_t run_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, uint32_t* planes,
-                              float* astar, float* zstar, cudaStream_t st) {
-    export_kernel<Q, WT, GPS, EQ4><<<dim3((unsigned)sh.out), kThreads, 0, st>>>(
-        W, p.delta, p.zu, p.alpha, p.zb, codes, planes, astar, zstar, sh.out, sh.n_in, sh.g);
-    return cudaGetLastError();
+static int export_grid(int64_t work) {
+    int dev = 0, sms = 1;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (work + kThreads - 1) / kThreads;
+    const int64_t cap = (int64_t)sms * 8;
+    return (int)(want < cap ? (want < 1 ? 1 : want) : cap);
 }
 
 template <int Q, typename WT, bool EQ4>
-static cudaError_t export_g(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, uint32_t* planes,
-                            float* astar, float* zstar, cudaStream_t st) {
-    if (sh.g == 32) return run_export<Q, WT, 4, EQ4>(sh, W, p, codes, planes, astar, zstar, st);
-    if (sh.g == 64) return run_export<Q, WT, 2, EQ4>(sh, W, p, codes, planes, astar, zstar, st);
-    return run_export<Q, WT, 1, EQ4>(sh, W, p, codes, planes, astar, zstar, st);
+static cudaError_t run_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, uint32_t* planes,
+                              float* astar, float* zstar, cudaStream_t st) {
+    const int grid = export_grid(sh.out * (int64_t)(sh.n_in / 32));
+    export_kernel<Q, WT, EQ4><<<grid, kThreads, 0, st>>>(W, p.delta, p.zu, p.alpha, p.zb, codes, planes, astar,
+                                                         zstar, sh.out, sh.n_in, sh.g);
+    return cudaGetLastError();
 }
 
 template <int Q>
 static cudaError_t export_q(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
                             uint32_t* planes, float* astar, float* zstar, cudaStream_t st) {
-    if (mode == UQ_EXPORT_REUSE_CODES) return export_g<Q, WF32, false>(sh, W, p, codes, planes, astar, zstar, st);
-    if (sh.wdtype == UQ_W_BF16) return export_g<Q, WBF16, true>(sh, W, p, codes, planes, astar, zstar, st);
-    return export_g<Q, WF32, true>(sh, W, p, codes, planes, astar, zstar, st);
+    if (mode == UQ_EXPORT_REUSE_CODES) return run_export<Q, WF32, false>(sh, W, p, codes, planes, astar, zstar, st);
+    if (sh.wdtype == UQ_W_BF16) return run_export<Q, WBF16, true>(sh, W, p, codes, planes, astar, zstar, st);
+    return run_export<Q, WF32, true>(sh, W, p, codes, planes, astar, zstar, st);
 }
 
 cudaError_t launch_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,

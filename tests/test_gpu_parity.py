@@ -240,3 +240,40 @@ def test_pipelined_and_plain_paths_agree_across_shapes(n_in, g):
     gr = C.gpu_bwd(raw, P, codes, Gup, q, g)
     ref, mass = C.oracle_bwd(W, P, r_codes, Gup, g)
     C.assert_grads_close(gr, ref, mass, f"n_in={n_in} g={g}")
+
+
+def test_host_buffer_apis_match_the_oracle():
+    """HostStep and HostPipeline (pinned host buffers in, results back on the
+    host) give the oracle's results; two independent problems are submitted
+    alternately through the overlapped pipeline."""
+    q, g, out, n_in = 3, 128, 48, 1024
+    probs = []
+    for seed in (31, 32):
+        raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=seed)
+        r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                         O.MAP_LOCAL_PERIODIC, 0, 2)
+        ref, mass = C.oracle_bwd(W, P, r_codes, Gup, g)
+        probs.append((raw, P, codes0, Gup, r_what, r_codes, ref, mass))
+    hp = api.HostPipeline(out, n_in, q, g, torch.bfloat16, C.dev(), depth=2)
+    bufs = []
+    for raw, P, codes0, Gup, *_ in probs:
+        hin, hout = hp.empty_host(pinned=True)
+        hin["W"].copy_(torch.from_numpy(raw.view(np.int16)).view(torch.bfloat16))
+        for k in api.PARAM_NAMES:
+            hin[k].copy_(torch.from_numpy(P[k]))
+        hin["codes"].copy_(torch.from_numpy(codes0))
+        hin["dL_dWhat"].copy_(torch.from_numpy(Gup))
+        bufs.append((hin, hout))
+    for rep in range(3):
+        for (hin, hout) in bufs:
+            hp.submit(hin, hout, 0, 2)
+    hp.synchronize()
+    for (hin, hout), (raw, P, codes0, Gup, r_what, r_codes, ref, mass) in zip(bufs, probs):
+        C.assert_fwd_equal(hout["W_hat"].numpy(), hout["codes"].numpy(), r_what, r_codes, "pipeline")
+        C.assert_grads_close({k: hout[k].numpy() for k in api.GRAD_NAMES}, ref, mass, "pipeline")
+    hs = api.HostStep(out, n_in, q, g, torch.bfloat16, C.dev())
+    hin, hout = bufs[0][0], hs.empty_host(pinned=True)[1]
+    hs.run(hin, hout, 0, 2)
+    hs.stream.synchronize()
+    raw, P, codes0, Gup, r_what, r_codes, ref, mass = probs[0]
+    C.assert_fwd_equal(hout["W_hat"].numpy(), hout["codes"].numpy(), r_what, r_codes, "hoststep")
