@@ -121,10 +121,12 @@ struct Stage {
     static_assert(SZ_P % 16 == 0 && SZ_A % 16 == 0 && SZ_C % 16 == 0, "bulk copy sizes must be multiples of 16");
 };
 
-// Work-item bookkeeping shared by the two kernels: item i of a warp is unit
-// wr + WPR * (i % n_w) of row (blockIdx.x + (i / n_w) * gridDim.x) * R + row_sub.
+// Work items of one warp: for its row blocks k = 0, 1, ... (block rows
+// (blockIdx.x + k * gridDim.x) * R + row_sub) the units wr, wr + WPR, ...
+// (n_w per row block).  Positions advance with Cursor::next, without
+// integer division.
 struct Items {
-    int R, WPR, row_sub, wr, n_w;
+    int R, WPR, row_sub, wr, n_w, n_blocks;
     long long total;
     __device__ Items(int U, int Rr, int n_rb, int warp) {
         R = Rr;
@@ -132,13 +134,28 @@ struct Items {
         row_sub = warp / WPR;
         wr = warp % WPR;
         n_w = wr < U ? (U - wr + WPR - 1) / WPR : 0;
-        const int mine = (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
-        total = (long long)mine * n_w;
+        n_blocks = (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+        total = (long long)n_blocks * n_w;
     }
-    __device__ int64_t row_of(long long i) const {
-        return ((int64_t)blockIdx.x + (i / n_w) * (int64_t)gridDim.x) * R + row_sub;
+    __device__ int64_t row(int k) const { return ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * R + row_sub; }
+    __device__ int unit(int j) const { return wr + WPR * j; }
+};
+
+struct Cursor {
+    int k = 0, j = 0;                        // row block, unit slot
+    __device__ void next(int n_w) {
+        if (++j == n_w) { j = 0; ++k; }
     }
-    __device__ int unit_of(long long i) const { return wr + WPR * (int)(i % n_w); }
+};
+
+// Stage ring position: stage index and the mbarrier phase parity of its next completion.
+template <int NST>
+struct Ring {
+    int s = 0;
+    uint32_t parity = 0;
+    __device__ void next() {
+        if (++s == NST) { s = 0; parity ^= 1u; }
+    }
 };
 
 // ---------------------------------------------------------------------------
@@ -175,13 +192,12 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     }
     __syncthreads();
 
-    auto issue = [&](long long i) {                       // lane 0 only
-        const int s = (int)(i % NST);
+    auto issue = [&](const Cursor& c, int s) {           // lane 0 only
         const uint32_t bar = tma::smem_addr(&bars[warp][s]);
-        const int64_t row = it.row_of(i);
+        const int64_t row = it.row(c.k);
         if (row >= out) { tma::bar_arrive(bar); return; }
-        const int64_t e0 = row * n_in + (int64_t)it.unit_of(i) * UE;
-        const int64_t g0 = row * Gr + (int64_t)it.unit_of(i) * NG;
+        const int64_t e0 = row * n_in + (int64_t)it.unit(c.j) * UE;
+        const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * NG;
         const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
         tma::fence_async_smem();
         tma::bar_arrive_tx(bar, TX);
@@ -194,22 +210,27 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
     };
-    if (lane == 0)
-        for (long long i = 0; i < NST && i < it.total; ++i) issue(i);
+    Cursor ic;                                            // next item to issue
+    long long issued = 0;
+    if (lane == 0) {
+        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+            issue(ic, s);
+            ic.next(it.n_w);
+        }
+    }
 
     bool alive = true;
-    long long i = 0;
-    const int n_mine = it.n_w > 0 ? (int)(it.total / it.n_w)
-                                  : (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+    Ring<NST> ring;
+    const int n_mine = it.n_blocks;
     for (int k = 0; k < n_mine; ++k) {
         const int64_t rb = (int64_t)blockIdx.x + (int64_t)k * gridDim.x;
         const int64_t row = rb * R + it.row_sub;
         const bool row_ok = row < out;
         const float sr = row_ok ? __ldg(SR + row) : 1.f;
         float prow = 0.f;
-        for (int j = 0; j < it.n_w; ++j, ++i) {
-            const int s = (int)(i % NST);
-            if (alive && !tma::bar_wait(tma::smem_addr(&bars[warp][s]), (uint32_t)((i / NST) & 1))) {
+        for (int j = 0; j < it.n_w; ++j) {
+            const int s = ring.s;
+            if (alive && !tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity)) {
                 alive = false;
                 if (lane == 0) atomicOr(&g_stream_err, 1u);
             }
@@ -237,7 +258,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 }
                 __syncwarp();
                 const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub];
-                const int unit = it.unit_of(i);
+                const int unit = it.unit(j);
                 const int64_t ebase = row * n_in + (int64_t)unit * UE;
                 float acc[8];
 #pragma unroll
@@ -286,7 +307,12 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 }
             }
             __syncwarp();                                // stage s and the tables are free again
-            if (alive && lane == 0 && i + NST < it.total) issue(i + NST);
+            if (alive && lane == 0 && issued < it.total) {
+                issue(ic, s);
+                ic.next(it.n_w);
+                ++issued;
+            }
+            ring.next();
         }
         prow = warp_sum(prow);
         if (lane == 0) red[k % kRowRing][warp] = prow;
@@ -341,13 +367,12 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     }
     __syncwarp();
 
-    auto issue = [&](long long i) {
-        const int s = (int)(i % NST);
+    auto issue = [&](const Cursor& c, int s) {           // lane 0 only
         const uint32_t bar = tma::smem_addr(&bars[warp][s]);
-        const int64_t row = it.row_of(i);
+        const int64_t row = it.row(c.k);
         if (row >= out) { tma::bar_arrive(bar); return; }
-        const int64_t e0 = row * n_in + (int64_t)it.unit_of(i) * UE;
-        const int64_t g0 = row * Gr + (int64_t)it.unit_of(i) * NG;
+        const int64_t e0 = row * n_in + (int64_t)it.unit(c.j) * UE;
+        const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * NG;
         const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
         tma::fence_async_smem();
         tma::bar_arrive_tx(bar, TX);
@@ -361,16 +386,24 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
     };
-    if (lane == 0)
-        for (long long i = 0; i < NST && i < it.total; ++i) issue(i);
+    Cursor ic;
+    long long issued = 0;
+    if (lane == 0) {
+        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+            issue(ic, s);
+            ic.next(it.n_w);
+        }
+    }
 
+    Ring<NST> ring;
+    Cursor cc;                                            // item being computed
     for (long long i = 0; i < it.total; ++i) {
-        const int s = (int)(i % NST);
-        if (!tma::bar_wait(tma::smem_addr(&bars[warp][s]), (uint32_t)((i / NST) & 1))) {
+        const int s = ring.s;
+        if (!tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity)) {
             if (lane == 0) atomicOr(&g_stream_err, 1u);
             return;                                      // no block barrier in this kernel
         }
-        const int64_t row = it.row_of(i);
+        const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
             const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
@@ -390,7 +423,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
             else if constexpr (mode == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
             const float dl = pd[sub], zu = pz[sub];
             const float sr = need_x ? __ldg(SR + row) : 0.f;
-            const int64_t ebase = row * n_in + (int64_t)it.unit_of(i) * UE;
+            const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
             float srt[L];
             if constexpr (mode == FWD_FULL) {
 #pragma unroll
@@ -447,7 +480,13 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
             }
         }
         __syncwarp();
-        if (lane == 0 && i + NST < it.total) issue(i + NST);
+        if (lane == 0 && issued < it.total) {
+            issue(ic, s);
+            ic.next(it.n_w);
+            ++issued;
+        }
+        ring.next();
+        cc.next(it.n_w);
     }
 }
 
