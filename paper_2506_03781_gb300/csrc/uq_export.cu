@@ -40,9 +40,13 @@ export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const
         ZSTAR[grp] = __fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp)));
     }
 
+    // (row, wcol) of chunk ch = row * words + wcol, advanced by nthr chunks
+    // per iteration without dividing inside the loop.
+    const int64_t step_rows = nthr / words;
+    const int step_cols = (int)(nthr - step_rows * words);
+    int64_t row = tid / words;
+    int wcol = (int)(tid - row * words);
     for (int64_t ch = tid; ch < out * words; ch += nthr) {
-        const int64_t row = ch / words;
-        const int wcol = (int)(ch - row * words);
         const int64_t e0 = row * n_in + (int64_t)wcol * 32;
         uint32_t cw[8];
         if constexpr (!EQ4) {
@@ -96,6 +100,9 @@ export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const
             for (int v = 0; v < 8; ++v) word |= gather_bit(cw[v], j) << (4 * v);
             PLANES[((int64_t)j * out + row) * words + wcol] = word;
         }
+        row += step_rows;
+        wcol += step_cols;
+        if (wcol >= words) { wcol -= words; ++row; }
     }
 }
 
