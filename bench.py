@@ -195,6 +195,73 @@ def time_oracle_step(wl, q, rows, budget_s):
 # GPU run
 # ---------------------------------------------------------------------------
 
+def time_matrices(wl, q, steps, warmup, dev, with_export=False, seed=0, graph=False):
+    """Times `steps` optimisation steps over every matrix of a workload, all
+    launches back to back on one stream: per matrix the forward (local
+    mapping, p from the workload: remap and keep steps alternate) and the
+    backward, plus the bit-plane export when `with_export`.  Parameters come
+    from the GPU unified initialization, jittered once.  With `graph` the
+    launches of a remap step and of a keep step are captured once as two CUDA
+    graphs and replayed.  Returns (ms per step, total weights)."""
+    import torch
+    from paper_2506_03781_gb300 import api, synth
+    g = wl.g
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 * wl.seed + q + 7 * seed)
+    mats = []
+    for idx, m in enumerate(wl.matrices):
+        raw, _ = synth.workload_weights(wl, idx)
+        Wd = api.weights_tensor(raw, dev)
+        p = api.empty_params(m.out, m.n_in, q, g, dev)
+        codes = torch.empty(m.out, m.n_in, dtype=torch.uint8, device=dev)
+        api.uq_init_params(Wd, q, g, p, codes, G=wl.G, T=wl.T)
+        for k in ("delta", "s", "sr", "alpha"):
+            p[k].mul_(1.0 + wl.init_eps * torch.randn(p[k].shape, generator=gen, device=dev))
+        G = torch.randn(m.out, m.n_in, generator=gen, device=dev) * float(np.sqrt(wl.grad_var))
+        qz = api.Quantizer(Wd, q, g, p, codes, torch.empty(m.out, m.n_in, device=dev), G,
+                           api.empty_grads(m.out, m.n_in, q, g, dev))
+        ex = None
+        if with_export:
+            ex = (torch.empty(q, m.out, m.n_in // 32, dtype=torch.int32, device=dev),
+                  torch.empty(m.out, m.n_in // g, q, device=dev), torch.empty(m.out, m.n_in // g, device=dev))
+        mats.append((qz, ex))
+
+    def step(t):
+        for qz, ex in mats:
+            qz.fwd(t, wl.p)
+            qz.bwd()
+            if ex is not None:
+                qz.export(*ex)
+
+    for t in range(warmup):
+        step(t)
+    torch.cuda.synchronize()
+    graphs = None
+    if graph:
+        side = torch.cuda.Stream(dev)
+        graphs = []
+        for t in (0, 1):                        # a remap step, a keep step
+            cg = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(cg, stream=side):
+                step(t)
+            graphs.append(cg)
+        torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(steps):
+        if graphs is not None:
+            graphs[(warmup + t) % wl.p != 0].replay()
+        else:
+            step(warmup + t)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    n = sum(m.out * m.n_in for m in wl.matrices)
+    del mats, graphs
+    torch.cuda.empty_cache()
+    return e0.elapsed_time(e1) / steps, n
+
+
 def run_gpu(args):
     import torch
     from paper_2506_03781_gb300 import api, roofline, synth
@@ -332,6 +399,16 @@ def run_gpu(args):
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
     e2e_value = weak_scaling_value(N, e2e_steps, world, e2e_ms / 1e3)
 
+    # bit-width sweep of the same matrix (the workload is specified for q in {2, 3, 4})
+    sweep = {}
+    if not args.no_sweep:
+        for qq in wl.qs:
+            if qq == q:
+                sweep[f"q{qq}"] = {"weights_per_s": value / world, "ms_per_step": ms_max / args.steps}
+                continue
+            ms_q, n_q = time_matrices(wl, qq, min(args.steps, 50), 3, dev)
+            sweep[f"q{qq}"] = {"weights_per_s": n_q / (ms_q / 1e3), "ms_per_step": ms_q}
+
     result = None
     if rank == 0:
         cpu = None
@@ -379,6 +456,7 @@ def run_gpu(args):
                     "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps,
                     "api": "paper_2506_03781_gb300.api.HostPipeline (pinned host buffers, uploads/compute/"
                            "downloads of consecutive steps overlapped)"},
+            "q_sweep": sweep,
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
@@ -387,6 +465,28 @@ def run_gpu(args):
     if world > 1:
         torch.distributed.destroy_process_group()
     return result
+
+
+def run_workloads(args):
+    """Times the other workloads: the Llama-3-8B block (seven matrices, q = 2,
+    g = 64, fwd + bwd + export as one launch sequence on one stream) and the
+    Llama-2-70B MLP matrices (q = 3, g = 128, fwd + bwd + export).  One JSON
+    line per workload."""
+    import torch
+    from paper_2506_03781_gb300 import synth
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    lines = []
+    for name in ("llama3_8b_block_bf16", "llama2_70b_mlp_bf16", "attn4k_bf16", "mat1k_f32"):
+        wl = synth.WORKLOADS[name]
+        for graph in (False, True):
+            ms, n = time_matrices(wl, wl.q, args.steps, args.warmup, dev, with_export=True, graph=graph)
+            line = {"workload": name, "q": wl.q, "g": wl.g, "weights": n, "steps": args.steps,
+                    "cuda_graph": graph, "ms_per_step": ms, "weights_per_s": n / (ms / 1e3),
+                    "step": "per matrix: fwd (local mapping, remap/keep alternating) + bwd + bit-plane export"}
+            print(json.dumps(line))
+            lines.append(line)
+    return lines
 
 
 def run_reference(args):
@@ -430,10 +530,14 @@ def main(argv=None):
     ap.add_argument("--q", type=int, default=3)
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the q sweep of the headline matrix")
+    ap.add_argument("--workloads", action="store_true", help="time the other workloads instead")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)          # at least 3 untimed warm-up steps
     if args.impl == "reference":
         return run_reference(args)
+    if args.workloads:
+        return run_workloads(args)
     return run_gpu(args)
 
 

@@ -147,11 +147,7 @@ def _raise(status):
 def _dims(W, g):
     if W.dim() != 2:
         raise ValueError("W must be 2-D [out, in]")
-    out, n_in = W.shape
-    if g <= 0 or n_in % g:
-        # let the library produce the error message for bad g
-        return out, n_in
-    return out, n_in
+    return W.shape[0], W.shape[1]
 
 
 # ---------------------------------------------------------------------------
@@ -368,3 +364,54 @@ class HostPipeline:
 
     def synchronize(self):
         self.down.synchronize()
+
+
+class Quantizer:
+    """Pre-validated buffers of one weight matrix, for repeated steps.
+
+    Checks every tensor once at construction (shapes, dtypes, device,
+    contiguity, the same checks as the functions above) and keeps the C
+    argument structures, so ``fwd``/``bwd``/``export`` are single C calls.
+    That matters for small matrices, whose kernels are shorter than the
+    per-call marshalling, and for capturing a whole step in a CUDA graph.
+    ``stream`` (a torch.cuda.Stream or raw handle) defaults to the current
+    stream at call time.
+    """
+
+    def __init__(self, W, q, g, params, codes, W_hat, dL_dWhat, grads):
+        self.W, self.q, self.g = W, q, g
+        self.out, self.n_in = _dims(W, g)
+        self.wd = _wdtype(W)
+        dev = W.device
+        self.device = dev
+        self.keep = (params, codes, W_hat, dL_dWhat, grads)       # keep the tensors alive
+        self.p = _params(params, self.out, self.n_in, q, g, dev)
+        self.codes = _check(codes, "codes", (self.out, self.n_in), torch.uint8, dev)
+        self.what = _check(W_hat, "W_hat", (self.out, self.n_in), torch.float32, dev)
+        self.G = _check(dL_dWhat, "dL_dWhat", (self.out, self.n_in), torch.float32, dev)
+        Gr = self.n_in // g
+        shapes = {"ddelta": (self.out, Gr), "dzu": (self.out, Gr), "ds": (self.out, self.n_in),
+                  "dsr": (self.out,), "dalpha": (self.out, Gr, q), "dzb": (self.out, Gr)}
+        self.gr = uq_grads(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev)
+                              for n in GRAD_NAMES})
+        self.wptr = W.data_ptr()
+        self.L = lib()
+
+    def _st(self, stream):
+        return _stream(stream, self.device)
+
+    def fwd(self, step, p_period=2, map_mode=MAP_LOCAL_PERIODIC, stream=None):
+        _raise(self.L.uq_quantize_fwd(self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes,
+                                      map_mode, step, p_period, self.what, self._st(stream)))
+
+    def bwd(self, stream=None):
+        _raise(self.L.uq_quantize_bwd(self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes,
+                                      self.G, self.gr, self._st(stream)))
+
+    def export(self, bitplanes, alpha_star, zb_star, mode=EXPORT_REUSE_CODES, stream=None):
+        Gr = self.n_in // self.g
+        _raise(self.L.uq_export_bcq(
+            self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes, mode,
+            _check(bitplanes, "bitplanes", (self.q, self.out, self.n_in // 32), torch.int32, self.device),
+            _check(alpha_star, "alpha_star", (self.out, Gr, self.q), torch.float32, self.device),
+            _check(zb_star, "zb_star", (self.out, Gr), torch.float32, self.device), self._st(stream)))

@@ -107,9 +107,7 @@ export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const
 }
 
 static int export_grid(int64_t work) {
-    int dev = 0, sms = 1;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int sms = sm_count();
     const int64_t want = (work + kThreads - 1) / kThreads;
     const int64_t cap = (int64_t)sms * 8;
     return (int)(want < cap ? (want < 1 ? 1 : want) : cap);

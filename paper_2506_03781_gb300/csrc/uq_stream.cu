@@ -494,10 +494,15 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // Launchers
 // ---------------------------------------------------------------------------
 
-static int sm_count() {
+constexpr int kMaxDevices = 64;
+
+int sm_count() {
+    static int cached[kMaxDevices] = {0};
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (dev >= 0 && dev < kMaxDevices && cached[dev] > 0) return cached[dev];
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return 1;
+    if (dev >= 0 && dev < kMaxDevices) cached[dev] = n;
     return n;
 }
 
@@ -507,14 +512,24 @@ bool stream_path_ok(const Shape& sh) {
     return sh.n_in % ue == 0;
 }
 
-template <typename KERN>
+// Persistent grid: min(row blocks, SMs x resident blocks per SM).  The
+// shared-memory attribute and the occupancy of a kernel instantiation are
+// set and queried once per device (KERN is a distinct type per call site).
+template <typename Tag, typename KERN>
 static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
-    int per_sm = 0;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    static int per_sm_cache[kMaxDevices] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
+    int per_sm = (dev >= 0 && dev < kMaxDevices) ? per_sm_cache[dev] : 0;
+    if (per_sm == 0) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) per_sm = 1;
+        if (dev >= 0 && dev < kMaxDevices) per_sm_cache[dev] = per_sm;
+    }
     const long long cap = (long long)sm_count() * per_sm;
     grid = (int)(n_rb < cap ? n_rb : cap);
     return cudaSuccess;
@@ -530,7 +545,7 @@ static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, c
     const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
     auto kern = bwd_stream_kernel<Q, WT, G_>;
     int grid = 0;
-    cudaError_t e = grid_for(kern, dyn, n_rb, grid);
+    cudaError_t e = grid_for<St>(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr,
                                       gr.ddelta, gr.dzu, gr.dzb, gr.dalpha, sh.out, sh.n_in, R, n_rb);
@@ -547,7 +562,8 @@ static cudaError_t run_fwd_stream_mode(const Shape& sh, const void* W, uq_params
     const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
     auto kern = fwd_stream_kernel<Q, WT, G_, MODE>;
     int grid = 0;
-    cudaError_t e = grid_for(kern, dyn, n_rb, grid);
+    cudaError_t e = grid_for<Stage<Q, WT, G_, MODE != FWD_KEEP, false, MODE != FWD_FULL, UQ_FWD_STAGE_BYTES>>(
+        kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R,
                                       n_rb);

@@ -277,3 +277,44 @@ def test_host_buffer_apis_match_the_oracle():
     hs.stream.synchronize()
     raw, P, codes0, Gup, r_what, r_codes, ref, mass = probs[0]
     C.assert_fwd_equal(hout["W_hat"].numpy(), hout["codes"].numpy(), r_what, r_codes, "hoststep")
+
+
+def test_quantizer_object_and_cuda_graph_capture():
+    """The pre-validated Quantizer gives the same bits as the function API, and
+    a step captured in a CUDA graph and replayed gives the same bits as eager
+    calls (the launch path makes no call that breaks stream capture)."""
+    q, g, out, n_in = 3, 128, 32, 1024
+    raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=41)
+    d = C.dev()
+
+    def make():
+        Wd = api.weights_tensor(raw, d)
+        pd = C.to_dev(P)
+        cd = torch.from_numpy(codes0).to(d)
+        qz = api.Quantizer(Wd, q, g, pd, cd, torch.empty(out, n_in, device=d), torch.from_numpy(Gup).to(d),
+                           api.empty_grads(out, n_in, q, g, d))
+        return qz, cd
+
+    qz, cd = make()
+    qz.fwd(0, 2)
+    qz.bwd()
+    eager = (C.host(qz.keep[2]).copy(), C.host(cd).copy(), {k: C.host(v).copy() for k, v in qz.keep[4].items()})
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(eager[0], eager[1], r_what, r_codes, "quantizer")
+    qz2, cd2 = make()
+    qz2.fwd(1, 2)                                   # warm the launch path before capture
+    torch.cuda.synchronize()
+    cd2.copy_(torch.from_numpy(codes0))
+    side = torch.cuda.Stream(d)
+    cg = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(cg, stream=side):
+        qz2.fwd(0, 2)
+        qz2.bwd()
+    cd2.copy_(torch.from_numpy(codes0))
+    torch.cuda.synchronize()
+    cg.replay()
+    torch.cuda.synchronize()
+    assert np.array_equal(C.host(qz2.keep[2]), eager[0]) and np.array_equal(C.host(cd2), eager[1])
+    for k in eager[2]:
+        assert np.array_equal(C.host(qz2.keep[4][k]), eager[2][k]), k
