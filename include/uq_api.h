@@ -198,6 +198,17 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
  */
 uq_status uq_check_device(void* stream);
 
+/*
+ * uq_selftest_wait_timeout -- exercises the bounded-wait path without any
+ * fault: launches one warp that waits on a shared-memory mbarrier nothing
+ * arrives at; after about 2^24 GPU clock cycles (~8 ms) the wait gives up,
+ * sets the same device indicator as a pipelined kernel would, and the warp
+ * returns.  The next uq_check_device() then returns UQ_ERR_CUDA (and clears
+ * the indicator); the context stays usable.  For tests of the failure path.
+ * The paper has no counterpart.
+ */
+uq_status uq_selftest_wait_timeout(void* stream);
+
 /* Message for the last non-OK status returned on the calling thread (never
  * NULL; "" if none).  Owned by the library, valid until the next call on
  * the same thread. */

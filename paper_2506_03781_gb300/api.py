@@ -29,7 +29,7 @@ EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
 ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq",
-                "uq_check_device", "uq_last_error", "uq_abi_version")
+                "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
 
 class UQError(RuntimeError):
@@ -70,6 +70,8 @@ def lib() -> ctypes.CDLL:
         L.uq_last_error.restype = ctypes.c_char_p
         L.uq_check_device.argtypes = [vp]
         L.uq_check_device.restype = ctypes.c_int
+        L.uq_selftest_wait_timeout.argtypes = [vp]
+        L.uq_selftest_wait_timeout.restype = ctypes.c_int
         L.uq_abi_version.argtypes = []
         L.uq_abi_version.restype = ctypes.c_int
         _lib = L
@@ -82,6 +84,12 @@ def uq_last_error() -> str:
 
 def uq_abi_version() -> int:
     return lib().uq_abi_version()
+
+
+def uq_selftest_wait_timeout(stream=None, device=None):
+    """Launches the bounded-wait self-test (a wait that runs out after ~8 ms)."""
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else device
+    _raise(lib().uq_selftest_wait_timeout(_stream(stream, dev)))
 
 
 def uq_check_device(stream=None, device=None):

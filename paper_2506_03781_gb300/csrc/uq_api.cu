@@ -158,8 +158,13 @@ uq_status uq_check_device(void* stream) {
     unsigned int flag = 0;
     e = uq::stream_error(true, &flag);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
-    if (flag) return fail(UQ_ERR_CUDA, "a pipelined kernel gave up waiting for its own data copies (bounded wait ran out)");
+    if (flag) return fail(UQ_ERR_CUDA, "a bounded wait ran out on the device (flag %u): a kernel gave up waiting "
+                                       "for its own data copies", flag);
     return ok();
+}
+
+uq_status uq_selftest_wait_timeout(void* stream) {
+    return cuda_status(uq::launch_wait_selftest((cudaStream_t)stream), "uq_selftest_wait_timeout");
 }
 
 }  // extern "C"

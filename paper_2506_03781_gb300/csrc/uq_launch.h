@@ -34,6 +34,8 @@ cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8
                               float* what, cudaStream_t st);
 cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
                               const float* gup, uq_grads gr, cudaStream_t st);
+// Launches the bounded-wait self-test (one warp, a wait that runs out).
+cudaError_t launch_wait_selftest(cudaStream_t st);
 // Streaming multiprocessors of the current device (cached per device).
 int sm_count();
 // Reads (and optionally clears) the flag a pipelined kernel sets when a

@@ -21,6 +21,11 @@ namespace uq {
 
 __device__ unsigned int g_stream_err = 0;
 
+#ifndef UQ_WAIT_HINT_NS
+#define UQ_WAIT_HINT_NS 20000
+#endif
+constexpr uint32_t kWaitHintNs = UQ_WAIT_HINT_NS;   // suspend-time hint of one try_wait
+
 namespace tma {
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -49,12 +54,26 @@ __device__ __forceinline__ bool bar_try_wait(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Bounded wait: gives up after ~2^31 GPU clock cycles (about one second).
-__device__ __forceinline__ bool bar_wait(uint32_t bar, uint32_t parity) {
+// try_wait with a suspend-time hint: the warp is parked by the hardware
+// until the phase completes or about `ns` nanoseconds pass, instead of
+// spinning through issue slots.
+__device__ __forceinline__ bool bar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: gives up after `limit` GPU clock cycles (default 2^31, about one second).
+__device__ __forceinline__ bool bar_wait(uint32_t bar, uint32_t parity, long long limit = 1ll << 31) {
     if (bar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
-    while (!bar_try_wait(bar, parity)) {
-        if (clock64() - t0 > (1ll << 31)) return false;
+    while (!bar_try_wait_sleep(bar, parity, kWaitHintNs)) {
+        if (clock64() - t0 > limit) return false;
     }
     return true;
 }
@@ -626,6 +645,26 @@ cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8
         case 3: return fwd_stream_w<3>(sh, W, p, codes, mode, what, st);
         default: return fwd_stream_w<4>(sh, W, p, codes, mode, what, st);
     }
+}
+
+// Self-test of the bounded wait: one warp waits on an mbarrier that nothing
+// ever arrives at; the wait runs out after `limit` cycles and sets the same
+// device flag a pipelined kernel sets, then the warp returns.
+__global__ void wait_selftest_kernel(long long limit) {
+    __shared__ __align__(8) unsigned long long bar;
+    const uint32_t b = tma::smem_addr(&bar);
+    if (threadIdx.x == 0) {
+        tma::bar_init(b, 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+    const bool done = tma::bar_wait(b, 0u, limit);
+    if (!done && threadIdx.x == 0) atomicOr(&g_stream_err, 2u);
+}
+
+cudaError_t launch_wait_selftest(cudaStream_t st) {
+    wait_selftest_kernel<<<1, 32, 0, st>>>(1ll << 24);     // ~8 ms at 2 GHz
+    return cudaGetLastError();
 }
 
 cudaError_t stream_error(bool clear, unsigned int* flag) {

@@ -318,3 +318,22 @@ def test_quantizer_object_and_cuda_graph_capture():
     assert np.array_equal(C.host(qz2.keep[2]), eager[0]) and np.array_equal(C.host(cd2), eager[1])
     for k in eager[2]:
         assert np.array_equal(C.host(qz2.keep[4][k]), eager[2][k]), k
+
+
+def test_bounded_wait_runs_out_reports_and_context_survives():
+    """Failure path of the pipelined kernels without any fault: a wait on an
+    mbarrier nothing arrives at gives up (bounded), the host reads the status
+    through uq_check_device, the indicator is cleared, and normal work on the
+    same context still matches the oracle."""
+    api.uq_check_device()                               # start clean
+    api.uq_selftest_wait_timeout()
+    with pytest.raises(api.UQError) as ei:
+        api.uq_check_device()
+    assert ei.value.status == api.UQ_ERR_CUDA and "bounded wait" in str(ei.value)
+    api.uq_check_device()                               # cleared
+    q, g, out, n_in = 3, 128, 16, 1024
+    raw, W, P, codes0, _ = C.make_inputs(out, n_in, q, g, seed=51)
+    what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(what, codes, r_what, r_codes, "after timeout")
