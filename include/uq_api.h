@@ -37,8 +37,7 @@
  *   bit-planes [q, out, in/32] uint32: bit b of planes[j][r][t] is c_{j+1}
  *                                 of column 32 t + b (1 <=> +1)
  * Shapes.  1 <= q <= 4; g in {32, 64} or g a multiple of 128; in a multiple
- *   of g; out >= 1; in <= 196608 (the backward pass keeps one row's group
- *   partial sums on chip for g > 128).
+ *   of g; 1 <= out <= 2^31 - 1; in <= 2^24.
  * Alignment.  Every pointer must be 16-byte aligned.
  * Errors.  Arguments are checked before anything is launched; on error the
  *   call returns a non-zero uq_status, launches nothing, writes nothing, and

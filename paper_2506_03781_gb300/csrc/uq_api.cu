@@ -24,7 +24,7 @@ uq_status ok() {
     return UQ_OK;
 }
 
-constexpr int64_t kMaxIn = 196608;   // one row's per-warp-step partials fit in shared memory
+constexpr int64_t kMaxIn = int64_t(1) << 24;   // row lengths whose 32-bit per-row offsets stay exact
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

@@ -81,7 +81,7 @@ def _grads(api, **over):
     (dict(q=0), "UNSUPPORTED"), (dict(q=5), "UNSUPPORTED"),
     (dict(g=48), "ARG"), (dict(g=16), "ARG"), (dict(g=96, n_in=384), "UNSUPPORTED"),
     (dict(n_in=200), "ARG"), (dict(out=0), "ARG"), (dict(n_in=0), "ARG"),
-    (dict(n_in=196608 * 2, g=128), "UNSUPPORTED"),
+    (dict(n_in=(1 << 24) + 128, g=128), "UNSUPPORTED"),
     (dict(wd=7), "ARG"), (dict(map_mode=3), "ARG"), (dict(p_period=0), "ARG"), (dict(step=-1), "ARG"),
     (dict(W=0), "ARG"), (dict(W=FAKE + 8), "ALIGN"), (dict(what=0), "ARG"), (dict(codes=FAKE + 4), "ALIGN"),
     (dict(params=dict(delta=0)), "ARG"), (dict(params=dict(alpha=FAKE + 2)), "ALIGN"),

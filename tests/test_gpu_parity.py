@@ -337,3 +337,59 @@ def test_bounded_wait_runs_out_reports_and_context_survives():
     r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
                                      O.MAP_LOCAL_PERIODIC, 0, 2)
     C.assert_fwd_equal(what, codes, r_what, r_codes, "after timeout")
+
+
+@pytest.mark.parametrize("g,n_in", [(512, 2048), (1024, 3072), (2048, 2048), (640, 1280)])
+def test_large_groups_all_entry_points(g, n_in):
+    """Groups of more than 128 elements, including one group per row
+    (channel-wise, g = in): forward (all modes), backward, export and
+    initialization on the general path."""
+    q, out = 3, 9
+    raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=g + n_in, init_G=4, init_T=2)
+    for mode, step in ((api.MAP_FULL, 0), (api.MAP_LOCAL_PERIODIC, 0), (api.MAP_LOCAL_PERIODIC, 1)):
+        what, codes = C.gpu_fwd(raw, P, codes0 if mode else None, q, g, mode, step, 2)
+        r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"],
+                                         codes0 if mode else None, g, mode, step, 2)
+        C.assert_fwd_equal(what, codes, r_what, r_codes, f"g={g} mode={mode} step={step}")
+    gr = C.gpu_bwd(raw, P, codes0, Gup, q, g)
+    ref, mass = C.oracle_bwd(W, P, codes0, Gup, g)
+    C.assert_grads_close(gr, ref, mass, f"g={g}")
+    planes, a_s, z_s = C.gpu_export(raw, P, codes0, q, g, api.EXPORT_REUSE_CODES)
+    r_planes, r_as, r_zs, _ = O.export_bcq(W, P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g)
+    assert np.array_equal(planes, r_planes) and np.array_equal(a_s, r_as) and np.array_equal(z_s, r_zs)
+    Wd = api.weights_tensor(raw, C.dev())
+    p = api.empty_params(out, n_in, q, g, C.dev())
+    codes = torch.empty(out, n_in, dtype=torch.uint8, device=C.dev())
+    api.uq_init_params(Wd, q, g, p, codes, G=4, T=2)
+    ref_i = O.unified_init(W, q, g, G=4, T=2)
+    same = (C.host(p["delta"]) == ref_i["delta"]) & (C.host(p["zu"]) == ref_i["zu"]) & \
+        (C.host(p["alpha"]) == ref_i["alpha"]).all(-1)
+    assert same.mean() >= 0.9, same.mean()
+
+
+def test_maximum_row_length():
+    """The longest supported row (in = 2^24) on both paths: g = 128 takes the
+    pipelined kernels, g = 256 the general ones.  Parameters are a jittered
+    uniform level grid (no initialization needed at this size)."""
+    q, out, n_in = 2, 1, 1 << 24
+    rng = np.random.default_rng(8)
+    W32 = (rng.standard_normal((out, n_in)) * 0.02).astype(np.float32)
+    raw, W = synth.bf16_round(W32)
+    Gup = synth.upstream_grad(out, n_in, 1e-4, 8)
+    for g in (128, 256):
+        Gr = n_in // g
+        P = {"delta": rng.uniform(0.008, 0.012, (out, Gr)).astype(np.float32),
+             "zu": rng.uniform(1.3, 1.7, (out, Gr)).astype(np.float32),
+             "s": rng.uniform(0.95, 1.05, (out, n_in)).astype(np.float32),
+             "sr": np.ones(out, np.float32),
+             "alpha": (np.array([1.0, 0.5]) * rng.uniform(0.9, 1.1, (out, Gr, q))).astype(np.float32),
+             "zb": np.full((out, Gr), 1.5, np.float32)}
+        _, codes0 = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], None, g, O.MAP_FULL)
+        P["delta"] = (P["delta"] * np.float32(1.01)).astype(np.float32)
+        what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+        r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                         O.MAP_LOCAL_PERIODIC, 0, 2)
+        C.assert_fwd_equal(what, codes, r_what, r_codes, f"max row g={g}")
+        gr = C.gpu_bwd(raw, P, r_codes, Gup, q, g)
+        ref, mass = C.oracle_bwd(W, P, r_codes, Gup, g)
+        C.assert_grads_close(gr, ref, mass, f"max row g={g}")
