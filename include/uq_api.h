@@ -44,8 +44,9 @@
  *   uq_last_error() describes the problem.  UQ_ERR_CUDA reports a failed
  *   launch (cudaGetLastError after the launch).  No entry point aborts,
  *   exits or traps the device.
- * Determinism.  No atomics are used; a call repeated on the same inputs
- *   gives bitwise-identical outputs.
+ * Determinism.  No output is accumulated with atomics (the only atomic is
+ *   the OR into the library's timeout flag); a call repeated on the same
+ *   inputs gives bitwise-identical outputs.
  * Numerics.  Every value that decides an integer (x, the levels, the
  *   distances, the filter test) is computed in IEEE fp32 with the operation
  *   order written at each entry point, no FMA contraction; gradients are
