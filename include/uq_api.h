@@ -13,7 +13,7 @@
  * estimator with gradient filtering (App. C.1).  After training, Theorem 1
  * folds D_R into the BCQ parameters (alpha* = Delta alpha,
  * z_B* = Delta (z_B - z_U)) and the binary codes are exported as bit-planes
- * (Algorithm 1, lines 10-11; Eq. 4).
+ * (the last two steps of Algorithm 1; Eq. 4).
  *
  * Conventions common to every entry point
  * ---------------------------------------
@@ -172,8 +172,8 @@ uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
                           uq_grads grads, void* stream);
 
 /*
- * uq_export_bcq -- Theorem 1 and the final binary codes (Algorithm 1,
- * lines 10-11).
+ * uq_export_bcq -- Theorem 1 and the final binary codes (the last two
+ * steps of Algorithm 1).
  *
  * alpha_star[r, k, j] = Delta * alpha_j and zb_star[r, k] = Delta * (z_B - z_U)
  * (fp32, z_B - z_U first).  The code matrix is the stored codes

@@ -321,7 +321,7 @@ def pack_bitplanes(codes, q):
 
 
 def export_bcq(W, delta, zu, alpha, zb, codes, g, mode=EXPORT_REUSE_CODES):
-    """Algorithm 1 lines 10-11: Theta_B* by Theorem 1, then the code matrix.
+    """The last two steps of Algorithm 1: Theta_B* by Theorem 1, then the code matrix.
 
     mode EXPORT_REUSE_CODES keeps the codes of the last quantizer step (for
     which Theorem 1 makes R_B(C; Theta_B*) equal the quantizer output);

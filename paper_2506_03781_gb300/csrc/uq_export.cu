@@ -1,5 +1,5 @@
 // Export: unification theorem (Theorem 1) and bit-plane packing of the
-// final binary codes (Algorithm 1, lines 10-11).
+// final binary codes (the last two steps of Algorithm 1).
 //
 // alpha* = Delta alpha, z_B* = Delta (z_B - z_U) per group.  The codes are
 // the stored ones (REUSE) or the nearest level of Theta_B* to each original

@@ -132,7 +132,7 @@ def test_unified_init_keeps_the_best_candidate(clip):
     gamma = i.astype(F32) / F32(G)
     d_ref = gamma * (w.max(-1) - w.min(-1)) / F32((1 << q) - 1)
     assert np.allclose(res["delta"].reshape(-1), d_ref, rtol=1e-6)
-    # s = 1, s_r = 1, z_B untouched for G > 1 (Alg. 2 line 2, Alg. 3 line 5)
+    # s = 1, s_r = 1, z_B untouched for G > 1 (Algorithm 2 sets s and s_r to 1; Algorithm 3 moves z_B only when G = 1)
     assert np.all(res["s"] == 1) and np.all(res["sr"] == 1)
     assert np.all(res["zb"] == GOLD["z_B_initial"]["k3"])
     # initial codes are the full mapping under the kept parameters
