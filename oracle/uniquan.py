@@ -42,6 +42,7 @@ __all__ = [
     "signs", "levels", "sorted_levels",
     "transform_F", "map_full", "map_local", "reconstruct", "detransform",
     "quantize_fwd", "quantize_bwd", "bwd_l1_mass",
+    "LR_F", "LR_B", "sgd_update", "train_step",
     "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
     "clip_params", "greedy_init", "general_alternating", "unified_init",
     "rtn",
@@ -277,6 +278,51 @@ def bwd_l1_mass(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
         dalpha=np.repeat(mass_gbar[..., None], q, axis=-1),
         dsr=np.abs(gbar * fu).sum(axis=(1, 2)) / np.abs(t["sr"]),
     )
+
+
+# ---------------------------------------------------------------------------
+# One optimisation step around the quantizer (the inner loop of Algorithm 1)
+# ---------------------------------------------------------------------------
+
+LR_F = 0.005     # learning rate of Theta_F = {Delta, z_U, s, s_r} (hyperparameter table, App. C.1)
+LR_B = 0.0005    # learning rate of Theta_B = {alpha, z_B} (same table)
+
+
+def sgd_update(s, sr, delta, zu, alpha, zb, grads, lr_F=LR_F, lr_B=LR_B):
+    """Plain SGD on Theta_IF = Theta_F u Theta_B.
+
+    FlexRound trains Theta_F by stochastic gradient descent (Sec. 3.1);
+    Algorithm 1 updates Theta_IF once per data point (batch size 1) with one
+    learning rate for Theta_F and one for Theta_B (hyperparameter table,
+    App. C.1):  theta <- theta - eta * dL/dtheta.  Evaluated in fp64 from
+    the fp64 gradients of quantize_bwd, stored as fp32.
+    """
+    def upd(theta, grad, lr):
+        return (np.asarray(theta, F64) - lr * np.asarray(grad, F64)).astype(F32)
+
+    return dict(
+        s=upd(s, grads["ds"], lr_F), sr=upd(sr, grads["dsr"], lr_F),
+        delta=upd(delta, grads["ddelta"], lr_F), zu=upd(zu, grads["dzu"], lr_F),
+        alpha=upd(alpha, grads["dalpha"], lr_B), zb=upd(zb, grads["dzb"], lr_B),
+    )
+
+
+def train_step(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, step, lr_F=LR_F, lr_B=LR_B,
+               mode=MAP_LOCAL_PERIODIC, p=2):
+    """One pass of Algorithm 1's inner loop as the quantizer sees it.
+
+    `codes` are the codes the forward of step `step` produced and Gup is
+    dL/dW^ of that forward.  The step back-propagates Gup (quantize_bwd),
+    updates Theta_IF (sgd_update) and quantizes W again for step `step + 1`
+    with the updated parameters (quantize_fwd; under M*_B that forward
+    remaps only when (step + 1) % p == 0).
+    Returns (dict of the updated fp32 parameters, codes and W^ of step + 1).
+    """
+    grads = quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g)
+    new = sgd_update(s, sr, delta, zu, alpha, zb, grads, lr_F, lr_B)
+    what, codes1 = quantize_fwd(W, new["s"], new["sr"], new["delta"], new["zu"], new["alpha"], new["zb"],
+                                codes, g, mode, step + 1, p)
+    return new, codes1, what
 
 
 # ---------------------------------------------------------------------------
