@@ -172,6 +172,35 @@ uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
                           uq_grads grads, void* stream);
 
 /*
+ * uq_train_step -- one optimisation step of Algorithm 1's inner loop, fused
+ * into one kernel: the backward of step `step` (exactly the gradients
+ * uq_quantize_bwd defines, not written out), the SGD update of every
+ * parameter in place (FlexRound trains Theta_F by SGD, Sec. 3.1; one
+ * learning rate for Theta_F = {Delta, z_U, s, s_r} and one for
+ * Theta_B = {alpha, z_B}, hyperparameter table of App. C.1: 0.005 and
+ * 0.0005), then the forward of step + 1 (as uq_quantize_fwd with step + 1)
+ * with the updated parameters.
+ *
+ * codes: in, the codes the forward of `step` produced; out, the codes of
+ *   step + 1 (under UQ_MAP_LOCAL_PERIODIC rewritten only when
+ *   (step + 1) % p_period == 0).
+ * dL_dWhat: [out, in] fp32, the gradient of that forward's W_hat.
+ * params: read, then overwritten with theta - lr * grad, evaluated in fp32
+ *   as fl(theta - fl(lr * grad)); each gradient is formed as in
+ *   uq_quantize_bwd (ds_r from the row's partial sums in a fixed order).
+ * W_hat: [out, in] fp32, written with W^ of step + 1.
+ * Shapes: g in {32, 64, 128}, in a multiple of 512 (256 for g = 32) and at
+ *   most 32768 (16384 for g = 32); other shapes return UQ_ERR_UNSUPPORTED
+ *   (the separate entry points cover them).  step in [0, 2^63 - 1),
+ *   p_period >= 1.  Outputs must not overlap the inputs other than the
+ *   in/out codes and params.  Deterministic: the same inputs give the same
+ *   bits.  The paper has no fused kernel; the step itself is its own.
+ */
+uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                        uq_params params, uint8_t* codes, const float* dL_dWhat, float lr_F, float lr_B,
+                        uq_map map, int64_t step, int p_period, float* W_hat, void* stream);
+
+/*
  * uq_export_bcq -- Theorem 1 and the final binary codes (the last two
  * steps of Algorithm 1).
  *

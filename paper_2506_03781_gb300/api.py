@@ -24,11 +24,12 @@ UQ_OK, UQ_ERR_ARG, UQ_ERR_UNSUPPORTED, UQ_ERR_ALIGN, UQ_ERR_CUDA = range(5)
 W_F32, W_BF16 = 0, 1
 CLIP_FIXED_MIN, CLIP_FIXED_MAX, CLIP_BALANCED = 0, 1, 2
 MAP_FULL, MAP_LOCAL_PERIODIC = 0, 1
+LR_THETA_F, LR_THETA_B = 0.005, 0.0005     # learning rates of the hyperparameter table (App. C.1)
 EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
-ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq",
+ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
                 "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
 
@@ -64,6 +65,9 @@ def lib() -> ctypes.CDLL:
         L.uq_quantize_fwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, vp]
         L.uq_export_bcq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
+        f32 = ctypes.c_float
+        L.uq_train_step.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, f32, f32, i32, i64, i32, vp,
+                                    vp]
         for name in ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq"):
             getattr(L, name).restype = ctypes.c_int
         L.uq_last_error.argtypes = []
@@ -206,6 +210,22 @@ def uq_quantize_bwd(W, q, g, params, codes, dL_dWhat, grads, stream=None):
         W.data_ptr(), _wdtype(W), out, n_in, q, g, _params(params, out, n_in, q, g, dev),
         _check(codes, "codes", (out, n_in), torch.uint8, dev),
         _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), gp, _stream(stream, dev))
+    _raise(st)
+
+
+def uq_train_step(W, q, g, params, codes, dL_dWhat, W_hat, step, lr_F=LR_THETA_F, lr_B=LR_THETA_B,
+                  map_mode=MAP_LOCAL_PERIODIC, p_period=2, stream=None):
+    """Fused step: backward of ``step``, SGD update of ``params`` in place, forward of ``step + 1``.
+
+    ``codes`` holds the codes of the forward of ``step`` on entry and those
+    of ``step + 1`` on return; ``W_hat`` receives W^ of ``step + 1``."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    st = lib().uq_train_step(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), float(lr_F), float(lr_B), map_mode, step,
+        p_period, _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
     _raise(st)
 
 
@@ -415,6 +435,13 @@ class Quantizer:
     def bwd(self, stream=None):
         _raise(self.L.uq_quantize_bwd(self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes,
                                       self.G, self.gr, self._st(stream)))
+
+    def train_step(self, step, lr_F=LR_THETA_F, lr_B=LR_THETA_B, p_period=2, map_mode=MAP_LOCAL_PERIODIC,
+                   stream=None):
+        """Fused backward of ``step`` + SGD update + forward of ``step + 1`` (uq_train_step)."""
+        _raise(self.L.uq_train_step(self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes,
+                                    self.G, float(lr_F), float(lr_B), map_mode, step, p_period, self.what,
+                                    self._st(stream)))
 
     def export(self, bitplanes, alpha_star, zb_star, mode=EXPORT_REUSE_CODES, stream=None):
         Gr = self.n_in // self.g

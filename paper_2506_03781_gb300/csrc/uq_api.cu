@@ -4,6 +4,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <cstdint>
 
 #include "uq_launch.h"
 
@@ -131,6 +132,35 @@ uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
     return cuda_status(uq::launch_bwd(sh, W, p, codes, dL_dWhat, gr, (cudaStream_t)stream), "uq_quantize_bwd");
 }
 
+uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                        uint8_t* codes, const float* dL_dWhat, float lr_F, float lr_B, uq_map map, int64_t step,
+                        int p_period, float* W_hat, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (map != UQ_MAP_FULL && map != UQ_MAP_LOCAL_PERIODIC) return fail(UQ_ERR_ARG, "unknown mapping %d", (int)map);
+    if (p_period < 1) return fail(UQ_ERR_ARG, "p_period=%d must be >= 1", p_period);
+    if (step < 0 || step == INT64_MAX) return fail(UQ_ERR_ARG, "step=%lld must be in [0, 2^63 - 1)", (long long)step);
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::step_path_ok(sh))
+        return fail(UQ_ERR_UNSUPPORTED,
+                    "the fused step handles g in {32, 64, 128} with in a multiple of %d and at most %d (g=%d in=%lld); "
+                    "use uq_quantize_bwd and uq_quantize_fwd",
+                    g == 32 ? 256 : 512, g == 32 ? 16384 : 32768, g, (long long)in);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.s, "params.s"));
+    UQ_TRY(check_ptr(p.sr, "params.sr"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(W_hat, "W_hat"));
+    const int64_t next = step + 1;
+    const int mode = map == UQ_MAP_FULL ? uq::FWD_FULL : (next % p_period == 0 ? uq::FWD_REMAP : uq::FWD_KEEP);
+    return cuda_status(uq::launch_step(sh, W, p, codes, dL_dWhat, lr_F, lr_B, mode, W_hat, (cudaStream_t)stream),
+                       "uq_train_step");
+}
+
 uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
                         const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes, float* alpha_star,
                         float* zb_star, void* stream) {
@@ -155,9 +185,11 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
 uq_status uq_check_device(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
-    unsigned int flag = 0;
+    unsigned int flag = 0, flag_step = 0;
     e = uq::stream_error(true, &flag);
+    if (e == cudaSuccess) e = uq::step_error(true, &flag_step);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
+    flag |= flag_step << 4;
     if (flag) return fail(UQ_ERR_CUDA, "a bounded wait ran out on the device (flag %u): a kernel gave up waiting "
                                        "for its own data copies", flag);
     return ok();

@@ -34,6 +34,14 @@ cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8
                               float* what, cudaStream_t st);
 cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
                               const float* gup, uq_grads gr, cudaStream_t st);
+// Fused optimisation step (uq_step.cu): backward of step t, SGD update,
+// forward of step t + 1 in `mode` (a FWD_* value).  step_path_ok tells
+// whether the shape is one the fused kernel handles.
+bool step_path_ok(const Shape& sh);
+cudaError_t launch_step(const Shape& sh, const void* W, uq_params p, uint8_t* codes, const float* gup, float lr_f,
+                        float lr_b, int mode, float* what, cudaStream_t st);
+// Reads (and optionally clears) the fused step kernel's bounded-wait flag.
+cudaError_t step_error(bool clear, unsigned int* flag);
 // Launches the bounded-wait self-test (one warp, a wait that runs out).
 cudaError_t launch_wait_selftest(cudaStream_t st);
 // Streaming multiprocessors of the current device (cached per device).

@@ -16,80 +16,11 @@
 // blocks, summed in warp order after one block barrier per ring.
 #include "uq_common.cuh"
 #include "uq_launch.h"
+#include "uq_pipe.cuh"
 
 namespace uq {
 
 __device__ unsigned int g_stream_err = 0;
-
-#ifndef UQ_WAIT_HINT_NS
-#define UQ_WAIT_HINT_NS 20000
-#endif
-constexpr uint32_t kWaitHintNs = UQ_WAIT_HINT_NS;   // suspend-time hint of one try_wait
-
-namespace tma {
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void bar_init_fence() {
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void bar_arrive_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void bar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool bar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// try_wait with a suspend-time hint: the warp is parked by the hardware
-// until the phase completes or about `ns` nanoseconds pass, instead of
-// spinning through issue slots.
-__device__ __forceinline__ bool bar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t ns) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity), "r"(ns)
-        : "memory");
-    return ok != 0;
-}
-// Bounded wait: gives up after `limit` GPU clock cycles (default 2^31, about one second).
-__device__ __forceinline__ bool bar_wait(uint32_t bar, uint32_t parity, long long limit = 1ll << 31) {
-    if (bar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (!bar_try_wait_sleep(bar, parity, kWaitHintNs)) {
-        if (clock64() - t0 > limit) return false;
-    }
-    return true;
-}
-__device__ __forceinline__ void fence_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-// Global -> shared bulk copy; bytes a multiple of 16, both addresses 16-byte aligned.
-__device__ __forceinline__ void copy_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
-
-}  // namespace tma
-
-constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
 // Shared memory per warp for its stages, and the resident blocks per SM the
 // register allocation is bounded for (backward; forward).
@@ -105,40 +36,7 @@ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 #ifndef UQ_STREAM_FWD_MIN_BLOCKS
 #define UQ_STREAM_FWD_MIN_BLOCKS 4
 #endif
-constexpr int kMaxStages = 16;
 constexpr int kRowRing = 32;             // row blocks whose ds_r partials wait in shared memory
-
-// Shared-memory stage layout of one work unit.  HAS_X: weights and s are
-// staged; HAS_G: dL/dW^ is staged; HAS_C: code words are staged.  The group
-// parameters (Delta, z_U, z_B, alpha of the unit's NG groups) always are.
-template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET>
-struct Stage {
-    static constexpr int LPG = G_ <= 64 ? 4 : 8;
-    static constexpr int NG = 32 / LPG;                  // groups per unit
-    static constexpr int NV = G_ / (4 * LPG);            // vectors per lane
-    static constexpr int UE = NG * G_;                   // elements per unit
-    static constexpr int WBYTES = sizeof(typename WT::raw) / 4;
-    static constexpr int SZ_W = HAS_X ? UE * WBYTES : 0;
-    static constexpr int SZ_S = HAS_X ? UE * 4 : 0;
-    static constexpr int SZ_G = HAS_G ? UE * 4 : 0;
-    static constexpr int SZ_C = HAS_C ? UE : 0;
-    static constexpr int SZ_P = NG * 4, SZ_A = NG * Q * 4;
-    static constexpr int OFF_W = 0;
-    static constexpr int OFF_S = align_up(OFF_W + SZ_W, 16);
-    static constexpr int OFF_G = OFF_S + SZ_S;
-    static constexpr int OFF_C = OFF_G + SZ_G;
-    static constexpr int OFF_D = align_up(OFF_C + SZ_C, 16);
-    static constexpr int OFF_Z = OFF_D + SZ_P;
-    static constexpr int OFF_B = OFF_Z + SZ_P;
-    static constexpr int OFF_A = OFF_B + SZ_P;
-    static constexpr int BYTES = align_up(OFF_A + SZ_A, 128);
-    static constexpr uint32_t TX = SZ_W + SZ_S + SZ_G + SZ_C + 3 * SZ_P + SZ_A;   // bytes copied per unit
-    // stages per warp within the per-warp shared-memory budget
-    static constexpr int FIT = BUDGET / BYTES;
-    static constexpr int NST = FIT < 2 ? 2 : (FIT > kMaxStages ? kMaxStages : FIT);
-    static constexpr int WARP_BYTES = NST * BYTES;
-    static_assert(SZ_P % 16 == 0 && SZ_A % 16 == 0 && SZ_C % 16 == 0, "bulk copy sizes must be multiples of 16");
-};
 
 // Work items of one warp: for its row blocks k = 0, 1, ... (block rows
 // (blockIdx.x + k * gridDim.x) * R + row_sub) the units wr, wr + WPR, ...
@@ -167,15 +65,15 @@ struct Cursor {
     }
 };
 
-// Stage ring position: stage index and the mbarrier phase parity of its next completion.
+
+// After a wait ran out: waits (bounded again) for the copies of items
+// [waited, issued) of a warp's stage ring, so that none lands in shared
+// memory after the block has exited.  Lane 0 only.
 template <int NST>
-struct Ring {
-    int s = 0;
-    uint32_t parity = 0;
-    __device__ void next() {
-        if (++s == NST) { s = 0; parity ^= 1u; }
-    }
-};
+__device__ void drain(unsigned long long (&bars)[NST], long long waited, long long issued) {
+    for (long long i = waited; i < issued; ++i)
+        tma::bar_wait(tma::smem_addr(&bars[i % NST]), (uint32_t)((i / NST) & 1));
+}
 
 // ---------------------------------------------------------------------------
 // Backward
@@ -239,6 +137,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     }
 
     bool alive = true;
+    long long waited = 0;                                 // items whose copies have landed
     Ring<NST> ring;
     const int n_mine = it.n_blocks;
     for (int k = 0; k < n_mine; ++k) {
@@ -249,9 +148,14 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         float prow = 0.f;
         for (int j = 0; j < it.n_w; ++j) {
             const int s = ring.s;
-            if (alive && !tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity)) {
-                alive = false;
-                if (lane == 0) atomicOr(&g_stream_err, 1u);
+            if (alive) {
+                // one verdict for the whole warp (lanes poll the mbarrier separately)
+                if (__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
+                    ++waited;
+                } else {
+                    alive = false;
+                    if (lane == 0) atomicOr(&g_stream_err, 1u);
+                }
             }
             if (alive && row_ok) {
                 const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -353,6 +257,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
             __syncthreads();
         }
     }
+    if (!alive && lane == 0) drain(bars[warp], waited, issued);
 }
 
 // ---------------------------------------------------------------------------
@@ -418,8 +323,11 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     Cursor cc;                                            // item being computed
     for (long long i = 0; i < it.total; ++i) {
         const int s = ring.s;
-        if (!tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity)) {
-            if (lane == 0) atomicOr(&g_stream_err, 1u);
+        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
+            if (lane == 0) {
+                atomicOr(&g_stream_err, 1u);
+                drain(bars[warp], i, issued);
+            }
             return;                                      // no block barrier in this kernel
         }
         const int64_t row = it.row(cc.k);

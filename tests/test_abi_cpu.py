@@ -137,6 +137,40 @@ def test_export_and_init_validation(libpath):
     assert L.uq_init_params(FAKE, 1, 8, 256, 3, 128, 30, 15, 0, _params(api, s=0), FAKE, None) == api.UQ_ERR_ARG
 
 
+@cpu_only
+@pytest.mark.parametrize("case,expect", [
+    (dict(q=5), "UNSUPPORTED"), (dict(n_in=200), "ARG"), (dict(map_mode=2), "ARG"), (dict(p_period=0), "ARG"),
+    (dict(step=-1), "ARG"), (dict(step=(1 << 63) - 1), "ARG"),
+    # shapes the fused kernel does not take: group sizes outside {32, 64, 128}, ragged units, rows over 64 units
+    (dict(g=256, n_in=512), "UNSUPPORTED"), (dict(n_in=384), "UNSUPPORTED"), (dict(g=32, n_in=384), "UNSUPPORTED"),
+    (dict(n_in=32768 + 512), "UNSUPPORTED"), (dict(g=32, n_in=16384 + 256), "UNSUPPORTED"),
+    (dict(W=0), "ARG"), (dict(gup=0), "ARG"), (dict(gup=FAKE + 4), "ALIGN"), (dict(what=0), "ARG"),
+    (dict(codes=0), "ARG"), (dict(params=dict(sr=0)), "ARG"), (dict(params=dict(s=FAKE + 8)), "ALIGN"),
+])
+def test_train_step_validation(libpath, case, expect):
+    from paper_2506_03781_gb300 import api
+    a = dict(W=FAKE, wd=api.W_BF16, out=8, n_in=512, q=3, g=128, codes=FAKE + 0x9000, gup=FAKE + 0xB000,
+             map_mode=1, step=0, p_period=2, what=FAKE + 0xA000)
+    a.update({k: v for k, v in case.items() if k != "params"})
+    p = _params(api, **case.get("params", {}))
+    st = api.lib().uq_train_step(a["W"], a["wd"], a["out"], a["n_in"], a["q"], a["g"], p, a["codes"], a["gup"],
+                                 0.005, 0.0005, a["map_mode"], a["step"], a["p_period"], a["what"], None)
+    assert st == getattr(api, "UQ_ERR_" + expect), (st, api.uq_last_error())
+    assert api.uq_last_error() != ""
+
+
+@cpu_only
+@pytest.mark.parametrize("g,n_in", [(128, 512), (128, 32768), (64, 32768), (32, 16384), (32, 256)])
+def test_train_step_accepts_the_fused_shapes(libpath, g, n_in):
+    """Shapes at the limits of the fused kernel pass validation (on this
+    GPU-less machine the launch itself then fails with UQ_ERR_CUDA)."""
+    from paper_2506_03781_gb300 import api
+    st = api.lib().uq_train_step(FAKE, api.W_BF16, 8, n_in, 3, g, _params(api), FAKE + 0x9000, FAKE + 0xB000,
+                                 0.005, 0.0005, 1, 0, 2, FAKE + 0xA000, None)
+    assert st == api.UQ_ERR_CUDA, api.uq_last_error()
+    assert "uq_train_step" in api.uq_last_error()
+
+
 def test_binding_rejects_host_tensors_before_calling(libpath):
     import torch
     from paper_2506_03781_gb300 import api
