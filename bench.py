@@ -128,7 +128,7 @@ def measured_peaks():
 
 def kernel_hash():
     h = hashlib.sha256()
-    for f in ("uq_stream.cu", "uq_common.cuh"):
+    for f in ("uq_stream.cu", "uq_common.cuh", "uq_pipe.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2506_03781_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -262,6 +262,35 @@ def time_matrices(wl, q, steps, warmup, dev, with_export=False, seed=0, graph=Fa
     return e0.elapsed_time(e1) / steps, n
 
 
+def time_train_step(Wd, q, g, P0, codes0, Gup, p, steps, stream, dev):
+    """CUDA-event times of the fused step (uq_train_step) over `steps` calls
+    after 3 warm-up calls, on copies of the parameters and codes (updated in
+    place from call to call, as in training).  Returns avg ms over all calls,
+    over the calls whose forward remaps and over those that keep the codes."""
+    import torch
+    from paper_2506_03781_gb300 import api
+    P = {k: v.clone() for k, v in P0.items()}
+    codes = codes0.clone()
+    what = torch.empty(codes.shape, dtype=torch.float32, device=dev)
+    qz = api.Quantizer(Wd, q, g, P, codes, what, Gup, api.empty_grads(codes.shape[0], codes.shape[1], q, g, dev))
+    for t in range(3):
+        qz.train_step(t, p_period=p, stream=stream)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for t in range(steps):
+        ev[t][0].record(stream)
+        qz.train_step(3 + t, p_period=p, stream=stream)
+        ev[t][1].record(stream)
+    torch.cuda.synchronize()
+    api.uq_check_device(stream)
+    ms = [a.elapsed_time(b) for a, b in ev]
+    remap = [m for t, m in enumerate(ms) if (3 + t + 1) % p == 0]
+    keep = [m for t, m in enumerate(ms) if (3 + t + 1) % p != 0]
+    return {"avg_ms": statistics.mean(ms), "steps": steps,
+            "remap": statistics.mean(remap) if remap else float("nan"),
+            "keep": statistics.mean(keep) if keep else float("nan")}
+
+
 def run_gpu(args):
     import torch
     from paper_2506_03781_gb300 import api, roofline, synth
@@ -373,6 +402,17 @@ def run_gpu(args):
     exp_ms = ex[0].elapsed_time(ex[1])
     exp_bytes = roofline.bytes_per_launch("export_reuse", out, n_in, q, g, wbytes)
 
+    # fused optimisation step (backward of t + SGD update + forward of t + 1)
+    # on its own copy of the parameters, updated in place step after step
+    train = time_train_step(Wd, q, g, ring[0], codes, Gup, wl.p, min(args.steps, 100), stream, dev)
+    train_bytes = {k: roofline.bytes_per_launch(k, out, n_in, q, g, wbytes) for k in ("step_remap", "step_keep")}
+    for k in ("remap", "keep"):
+        ms_k = train[k]
+        train[k] = {"avg_ms": ms_k, "gbs": train_bytes["step_" + k] / 1e6 / ms_k,
+                    "frac": train_bytes["step_" + k] / 1e6 / ms_k / peak}
+    train["weights_per_s"] = N / (train["avg_ms"] / 1e3)
+    train["algorithmic_bytes_avg"] = (train_bytes["step_remap"] + train_bytes["step_keep"]) / 2
+
     # end-to-end through the public host-buffer API: every step uploads its
     # inputs from pinned host memory, runs fwd+bwd and downloads its results;
     # consecutive steps (independent, like successive weight matrices)
@@ -456,6 +496,7 @@ def run_gpu(args):
                     "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps,
                     "api": "paper_2506_03781_gb300.api.HostPipeline (pinned host buffers, uploads/compute/"
                            "downloads of consecutive steps overlapped)"},
+            "train_step": train,
             "q_sweep": sweep,
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,

@@ -4,6 +4,9 @@ Per element: weights (2 B bf16 / 4 B fp32), s (4 B), code word (1 B),
 w^ / dL/dw^ / ds (4 B each).  Per group: the parameters Delta, z_U, z_B and
 alpha_1..q ((3 + q) * 4 B) read once, and the same number of gradient
 values written by the backward.  Per row: s_r (4 B) read, ds_r written.
+The fused optimisation step reads W, s, codes and dL/dw^ once and writes the
+updated s, w^ of the next step and (on remap steps) its codes; every group
+parameter and s_r is read and rewritten.
 """
 
 from __future__ import annotations
@@ -21,6 +24,10 @@ def bytes_per_launch(kind: str, out: int, n_in: int, q: int, g: int, wbytes: int
         return n * (wbytes + 4 + 4 + 1) + gp + out * 4
     if kind == "bwd":              # read W, s, codes, dL/dw^; write ds; group/row grads
         return n * (wbytes + 4 + 1 + 4 + 4) + 2 * gp + 2 * out * 4
+    if kind in ("step_remap", "step_full"):  # read W, s, codes, dL/dw^; write s', w^, codes; params in/out
+        return n * (wbytes + 4 + 1 + 4 + 4 + 4 + 1) + 2 * gp + 2 * out * 4
+    if kind == "step_keep":        # as step_remap, codes not rewritten
+        return n * (wbytes + 4 + 1 + 4 + 4 + 4) + 2 * gp + 2 * out * 4
     if kind == "export_reuse":     # read codes; write planes, alpha*, z*
         return n * 1 + q * n // 8 + gp + groups * (q + 1) * 4
     if kind == "export_eq4":       # read W; write planes, alpha*, z*
