@@ -44,6 +44,7 @@ __all__ = [
     "quantize_fwd", "quantize_bwd", "bwd_l1_mass",
     "LR_F", "LR_B", "sgd_update", "train_step",
     "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
+    "bcq_dequantize", "bcq_gemv",
     "clip_params", "greedy_init", "general_alternating", "unified_init",
     "rtn",
 ]
@@ -382,6 +383,45 @@ def export_bcq(W, delta, zu, alpha, zb, codes, g, mode=EXPORT_REUSE_CODES):
     else:
         c = np.asarray(codes, np.uint8)
     return pack_bitplanes(c, q), a_star, z_star, c
+
+
+# ---------------------------------------------------------------------------
+# Deployment: the BCQ product from the exported format
+# ---------------------------------------------------------------------------
+
+def bcq_dequantize(planes, alpha_star, zb_star, g, rows=slice(None)):
+    """R_B(C; Theta_B*) = C alpha* + z_B* (Sec. 2.3) read back from the
+    exported format: bit b of planes[j, r, t] is c_{j+1} = +1 for column
+    32 t + b (App. F.1 stores one bit per code and weight).  fp64, [rows, in].
+    """
+    planes = np.asarray(planes, np.uint32)[:, rows]
+    q, out, words = planes.shape
+    n_in = words * 32
+    bits = (planes[..., None] >> np.arange(32, dtype=np.uint32)) & 1          # [q, out, words, 32]
+    c = np.where(bits.reshape(q, out, n_in) == 1, 1.0, -1.0)                 # c_{j+1} per element
+    a = np.repeat(np.asarray(alpha_star, F64)[rows], g, axis=1)             # [out, in, q]
+    z = np.repeat(np.asarray(zb_star, F64)[rows], g, axis=1)                # [out, in]
+    return np.einsum("jri,rij->ri", c, a) + z
+
+
+def bcq_gemv(planes, alpha_star, zb_star, x, g, row_block=256):
+    """y = W~ x for every row x of `x` [batch, in], with W~ = C alpha* + z_B*
+    the exported BCQ weights: the product a BCQ inference kernel computes
+    (Sec. 2.3; the deployment format of App. F.1).  fp64, [batch, out].
+
+    Each output is the fp64 sum over the row of W~_ri x_i (numpy's sum along
+    the contiguous axis, the same for every row); the rows of W~ are
+    dequantized `row_block` at a time only to bound the memory.
+    """
+    x = np.atleast_2d(np.asarray(x, F64))
+    out = np.shape(planes)[1]
+    y = np.empty((x.shape[0], out), F64)
+    for r0 in range(0, out, row_block):
+        rows = slice(r0, min(out, r0 + row_block))
+        Wt = bcq_dequantize(planes, alpha_star, zb_star, g, rows)
+        for b in range(x.shape[0]):
+            y[b, rows] = (Wt * x[b][None, :]).sum(-1)
+    return y
 
 
 # ---------------------------------------------------------------------------
