@@ -291,6 +291,58 @@ def time_train_step(Wd, q, g, P0, codes0, Gup, p, steps, stream, dev):
             "keep": statistics.mean(keep) if keep else float("nan")}
 
 
+def time_gemv(q, g, dev, stream, peak, shapes=((14336, 4096), (8192, 28672)), reps=60):
+    """CUDA-event time of the BCQ product from the exported format
+    (uq_bcq_gemv, one bf16 token: the split kernel and the tile sum) per
+    call, on random bit-planes, alpha*, z* of each shape; the calls cycle
+    through enough copies of the inputs to exceed twice the L2, so every call
+    reads them from HBM.  `reps` calls are replayed from one CUDA graph."""
+    import math
+    import torch
+    from paper_2506_03781_gb300 import api, roofline
+    res = {}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(77)
+    for out, n_in in shapes:
+        nbytes = roofline.bytes_per_launch("gemv", out, n_in, q, g, 2)
+        copies = max(2, math.ceil(2 * 129e6 / nbytes))
+        ring = []
+        for _ in range(copies):
+            planes = torch.randint(-2 ** 31, 2 ** 31 - 1, (q, out, n_in // 32), generator=gen, device=dev,
+                                   dtype=torch.int32)
+            a_s = torch.randn(out, n_in // g, q, generator=gen, device=dev) * 0.01
+            z_s = torch.randn(out, n_in // g, generator=gen, device=dev) * 0.003
+            x = torch.randn(1, n_in, generator=gen, device=dev).to(torch.bfloat16)
+            ring.append((planes, a_s, z_s, x, torch.empty(1, out, device=dev)))
+        ws = api.bcq_gemv_workspace(out, n_in, 1, dev)
+        for i in range(3):
+            api.uq_bcq_gemv(*ring[i % copies], g, workspace=ws, stream=stream)
+        torch.cuda.synchronize()
+        # the calls are captured once in a CUDA graph so that the replay measures
+        # device time, not the per-call argument checking of the Python binding
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=side):
+            for i in range(reps):
+                api.uq_bcq_gemv(*ring[i % copies], g, workspace=ws, stream=side)
+        graph.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        graph.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / reps
+        del graph
+        res[f"{out}x{n_in}"] = {"us": us, "gbs": nbytes / us / 1e3, "frac": nbytes / us / 1e3 / peak,
+                                "weights_per_s": out * n_in / (us * 1e-6), "algorithmic_bytes": nbytes,
+                                "input_copies": copies}
+        del ring
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_gpu(args):
     import torch
     from paper_2506_03781_gb300 import api, roofline, synth
@@ -413,6 +465,9 @@ def run_gpu(args):
     train["weights_per_s"] = N / (train["avg_ms"] / 1e3)
     train["algorithmic_bytes_avg"] = (train_bytes["step_remap"] + train_bytes["step_keep"]) / 2
 
+    # deployment: the BCQ product from the exported format (one bf16 token)
+    gemv = time_gemv(q, g, dev, stream, peak)
+
     # end-to-end through the public host-buffer API: every step uploads its
     # inputs from pinned host memory, runs fwd+bwd and downloads its results;
     # consecutive steps (independent, like successive weight matrices)
@@ -497,6 +552,7 @@ def run_gpu(args):
                     "api": "paper_2506_03781_gb300.api.HostPipeline (pinned host buffers, uploads/compute/"
                            "downloads of consecutive steps overlapped)"},
             "train_step": train,
+            "bcq_gemv": gemv,
             "q_sweep": sweep,
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,

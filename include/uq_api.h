@@ -217,6 +217,36 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                         uint32_t* bitplanes, float* alpha_star, float* zb_star, void* stream);
 
 /*
+ * uq_bcq_gemv -- the BCQ matrix-vector product of deployment, computed from
+ * the exported format alone: y[b, r] = sum_i W~[r, i] x[b, i] with
+ * W~[r, i] = sum_j alpha_star[r, k, j] c_j + zb_star[r, k], k = i / g, and
+ * c_j = +1 where bit (i % 32) of bitplanes[j, r, i / 32] is set, else -1
+ * (R_B(C; Theta_B*) of Sec. 2.3; by Theorem 1 this is the quantizer's W^,
+ * so no Delta or z_U is needed at inference; bit-plane storage of App. F.1).
+ *
+ * bitplanes [q, out, in/32] uint32, alpha_star [out, in/g, q] and
+ * zb_star [out, in/g] fp32 as uq_export_bcq writes them; x [batch, in]
+ * (xdtype fp32 or bf16), y [batch, out] fp32, both row-major.  The columns
+ * are split into tiles of 512; each tile's contribution is formed from
+ * per-8-column partial sums of x (one table lookup per plane byte) and
+ * written to `workspace` (caller-owned device memory of at least
+ * uq_bcq_gemv_workspace_bytes(out, in, batch) bytes, overwritten), then the
+ * tiles are summed in order into y.  fp32 throughout, fixed order:
+ * deterministic, and within a small multiple of the fp32 unit roundoff of
+ * sum_i (sum_j |alpha*_j| + |z*|) |x_i| of the exact product.  Shapes as
+ * uq_quantize_fwd; 1 <= batch <= 64 (each token re-reads the planes).
+ * Reads every input, writes y and the workspace.  A too small workspace is
+ * UQ_ERR_ARG.
+ */
+uq_status uq_bcq_gemv(const uint32_t* bitplanes, const float* alpha_star, const float* zb_star, int64_t out,
+                      int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch, float* y,
+                      float* workspace, int64_t workspace_bytes, void* stream);
+
+/* Bytes of workspace uq_bcq_gemv needs for this shape (ceil(in/512) * batch
+ * * out floats), or -1 if the shape or batch is invalid.  Host only. */
+int64_t uq_bcq_gemv_workspace_bytes(int64_t out, int64_t in, int batch);
+
+/*
  * uq_check_device -- waits for `stream` to finish, then reports whether a
  * pipelined kernel of this library gave up waiting for its own data copies
  * since the last check (every wait on an mbarrier is bounded to about one

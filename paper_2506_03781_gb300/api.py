@@ -29,7 +29,8 @@ EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
-ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
+ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq", "uq_bcq_gemv",
+                "uq_bcq_gemv_workspace_bytes",
                 "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
 
@@ -65,6 +66,9 @@ def lib() -> ctypes.CDLL:
         L.uq_quantize_fwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, vp]
         L.uq_export_bcq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
+        L.uq_bcq_gemv.argtypes = [vp, vp, vp, i64, i64, i32, i32, vp, i32, i32, vp, vp, i64, vp]
+        L.uq_bcq_gemv_workspace_bytes.argtypes = [i64, i64, i32]
+        L.uq_bcq_gemv_workspace_bytes.restype = i64
         f32 = ctypes.c_float
         L.uq_train_step.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, f32, f32, i32, i64, i32, vp,
                                     vp]
@@ -245,6 +249,46 @@ def uq_export_bcq(W, q, g, params, codes, bitplanes, alpha_star, zb_star, mode=E
         cptr, mode, _check(bitplanes, "bitplanes", (q, out, n_in // 32), torch.int32, dev),
         _check(alpha_star, "alpha_star", (out, Gr, q), torch.float32, dev),
         _check(zb_star, "zb_star", (out, Gr), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_bcq_gemv_workspace_bytes(out, n_in, batch=1) -> int:
+    """Bytes of device workspace uq_bcq_gemv needs (-1 for an invalid shape)."""
+    return int(lib().uq_bcq_gemv_workspace_bytes(out, n_in, batch))
+
+
+def bcq_gemv_workspace(out, n_in, batch=1, device="cuda"):
+    """A workspace tensor large enough for uq_bcq_gemv on this shape."""
+    nbytes = uq_bcq_gemv_workspace_bytes(out, n_in, batch)
+    if nbytes < 0:
+        raise ValueError(f"invalid shape for the BCQ product: out={out} in={n_in} batch={batch}")
+    return torch.empty(max(nbytes // 4, 4), dtype=torch.float32, device=device)
+
+
+def uq_bcq_gemv(bitplanes, alpha_star, zb_star, x, y, g, workspace=None, stream=None):
+    """BCQ product y = W~ x from the exported format (``bitplanes`` int32 [q, out, in/32],
+    ``alpha_star`` [out, in/g, q], ``zb_star`` [out, in/g]); x [batch, in] fp32/bf16, y [batch, out] fp32.
+    ``workspace``: a float32 device tensor of at least uq_bcq_gemv_workspace_bytes bytes
+    (allocated here when None)."""
+    if bitplanes.dim() != 3 or x.dim() != 2:
+        raise ValueError("bitplanes must be [q, out, in/32] and x [batch, in]")
+    q, out, words = bitplanes.shape
+    batch, n_in = x.shape
+    if n_in != 32 * words:
+        raise ValueError(f"x has {n_in} columns, the planes {32 * words}")
+    dev = x.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    if workspace is None:
+        workspace = bcq_gemv_workspace(out, n_in, batch, dev)
+    if workspace.dtype != torch.float32 or workspace.device != dev or not workspace.is_contiguous():
+        raise ValueError("workspace must be a contiguous float32 tensor on the device of x")
+    st = lib().uq_bcq_gemv(
+        _check(bitplanes, "bitplanes", (q, out, words), torch.int32, dev),
+        _check(alpha_star, "alpha_star", (out, Gr, q), torch.float32, dev),
+        _check(zb_star, "zb_star", (out, Gr), torch.float32, dev), out, n_in, q, g,
+        _check(x, "x", (batch, n_in), x.dtype, dev), _wdtype(x), batch,
+        _check(y, "y", (batch, out), torch.float32, dev), workspace.data_ptr(), workspace.numel() * 4,
+        _stream(stream, dev))
     _raise(st)
 
 

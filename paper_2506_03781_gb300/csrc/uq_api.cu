@@ -182,6 +182,31 @@ uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                        "uq_export_bcq");
 }
 
+int64_t uq_bcq_gemv_workspace_bytes(int64_t out, int64_t in, int batch) {
+    if (out < 1 || in < 32 || in % 32 != 0 || in > kMaxIn || batch < 1 || batch > 64) return -1;
+    return uq::gemv_workspace_floats(out, in, batch) * (int64_t)sizeof(float);
+}
+
+uq_status uq_bcq_gemv(const uint32_t* bitplanes, const float* alpha_star, const float* zb_star, int64_t out,
+                      int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch, float* y, float* workspace,
+                      int64_t workspace_bytes, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, xdtype));
+    if (batch < 1 || batch > 64) return fail(UQ_ERR_ARG, "batch=%d must be in 1..64", batch);
+    UQ_TRY(check_ptr(bitplanes, "bitplanes"));
+    UQ_TRY(check_ptr(alpha_star, "alpha_star"));
+    UQ_TRY(check_ptr(zb_star, "zb_star"));
+    UQ_TRY(check_ptr(x, "x"));
+    UQ_TRY(check_ptr(y, "y"));
+    UQ_TRY(check_ptr(workspace, "workspace"));
+    const int64_t need = uq_bcq_gemv_workspace_bytes(out, in, batch);
+    if (workspace_bytes < need)
+        return fail(UQ_ERR_ARG, "workspace of %lld bytes; this product needs %lld (uq_bcq_gemv_workspace_bytes)",
+                    (long long)workspace_bytes, (long long)need);
+    return cuda_status(uq::launch_gemv(bitplanes, alpha_star, zb_star, out, (int)in, q, g, x, (int)xdtype, batch, y,
+                                       workspace, (cudaStream_t)stream),
+                       "uq_bcq_gemv");
+}
+
 uq_status uq_check_device(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));

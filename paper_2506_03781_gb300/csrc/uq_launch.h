@@ -42,6 +42,11 @@ cudaError_t launch_step(const Shape& sh, const void* W, uq_params p, uint8_t* co
                         float lr_b, int mode, float* what, cudaStream_t st);
 // Reads (and optionally clears) the fused step kernel's bounded-wait flag.
 cudaError_t step_error(bool clear, unsigned int* flag);
+// BCQ matrix-vector product from the exported bit-planes (uq_gemv.cu); `work`
+// holds gemv_workspace_floats(out, in, batch) floats of per-tile partials.
+int64_t gemv_workspace_floats(int64_t out, int64_t n_in, int batch);
+cudaError_t launch_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in, int q,
+                        int g, const void* x, int xdtype, int batch, float* y, float* work, cudaStream_t st);
 // Launches the bounded-wait self-test (one warp, a wait that runs out).
 cudaError_t launch_wait_selftest(cudaStream_t st);
 // Streaming multiprocessors of the current device (cached per device).

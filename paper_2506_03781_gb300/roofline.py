@@ -28,6 +28,8 @@ def bytes_per_launch(kind: str, out: int, n_in: int, q: int, g: int, wbytes: int
         return n * (wbytes + 4 + 1 + 4 + 4 + 4 + 1) + 2 * gp + 2 * out * 4
     if kind == "step_keep":        # as step_remap, codes not rewritten
         return n * (wbytes + 4 + 1 + 4 + 4 + 4) + 2 * gp + 2 * out * 4
+    if kind == "gemv":             # read planes, alpha*, z*, one token x (wbytes per value); write y
+        return q * n // 8 + groups * (q + 1) * 4 + n_in * wbytes + out * 4
     if kind == "export_reuse":     # read codes; write planes, alpha*, z*
         return n * 1 + q * n // 8 + gp + groups * (q + 1) * 4
     if kind == "export_eq4":       # read W; write planes, alpha*, z*

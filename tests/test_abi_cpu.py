@@ -171,6 +171,35 @@ def test_train_step_accepts_the_fused_shapes(libpath, g, n_in):
     assert "uq_train_step" in api.uq_last_error()
 
 
+@cpu_only
+@pytest.mark.parametrize("case,expect", [
+    (dict(q=0), "UNSUPPORTED"), (dict(g=48), "ARG"), (dict(n_in=200), "ARG"), (dict(out=0), "ARG"),
+    (dict(batch=0), "ARG"), (dict(batch=65), "ARG"), (dict(xd=5), "ARG"),
+    (dict(planes=0), "ARG"), (dict(planes=FAKE + 4), "ALIGN"), (dict(a=0), "ARG"), (dict(z=FAKE + 8), "ALIGN"),
+    (dict(x=0), "ARG"), (dict(y=0), "ARG"), (dict(y=FAKE + 12), "ALIGN"),
+    (dict(work=0), "ARG"), (dict(work=FAKE + 4), "ALIGN"), (dict(wbytes=8 * 4 - 4), "ARG"),
+])
+def test_bcq_gemv_validation(libpath, case, expect):
+    from paper_2506_03781_gb300 import api
+    a = dict(planes=FAKE, a=FAKE + 0x1000, z=FAKE + 0x2000, out=8, n_in=512, q=3, g=128, x=FAKE + 0x3000,
+             xd=api.W_BF16, batch=1, y=FAKE + 0x4000, work=FAKE + 0x5000, wbytes=1 << 20)
+    a.update(case)
+    st = api.lib().uq_bcq_gemv(a["planes"], a["a"], a["z"], a["out"], a["n_in"], a["q"], a["g"], a["x"], a["xd"],
+                               a["batch"], a["y"], a["work"], a["wbytes"], None)
+    assert st == getattr(api, "UQ_ERR_" + expect), (st, api.uq_last_error())
+    assert api.uq_last_error() != ""
+
+
+def test_bcq_gemv_workspace_size(libpath):
+    from paper_2506_03781_gb300 import api
+    # one float per 512-column tile, token and row
+    assert api.uq_bcq_gemv_workspace_bytes(8, 512, 1) == 8 * 4
+    assert api.uq_bcq_gemv_workspace_bytes(8192, 28672, 1) == 56 * 8192 * 4
+    assert api.uq_bcq_gemv_workspace_bytes(100, 4096 + 96, 3) == 9 * 3 * 100 * 4
+    for bad in ((0, 512, 1), (8, 500, 1), (8, 512, 0), (8, 512, 65)):
+        assert api.uq_bcq_gemv_workspace_bytes(*bad) == -1
+
+
 def test_binding_rejects_host_tensors_before_calling(libpath):
     import torch
     from paper_2506_03781_gb300 import api
