@@ -247,6 +247,35 @@ uq_status uq_bcq_gemv(const uint32_t* bitplanes, const float* alpha_star, const 
 int64_t uq_bcq_gemv_workspace_bytes(int64_t out, int64_t in, int batch);
 
 /*
+ * uq_bcq_gemv_noalloc -- the same product as uq_bcq_gemv (same arguments
+ * minus the workspace, same results bit for bit), for callers that cannot
+ * allocate device memory: code that runs where every byte of the GPU is
+ * owned by someone else's allocator, or where an allocation call is not
+ * allowed at all (it may block the whole device, or the host runtime simply
+ * gives the caller no way to reach it).  The paper has no counterpart; this
+ * is a convenience of the library.
+ *
+ * Instead of a workspace it uses scratch built into the library: 4 MiB
+ * (1,048,576 floats) in a static device array, which every GPU that loads
+ * the library holds until the process exits.  A shape whose partials need
+ * more (ceil(in/512) * batch * out floats, e.g. more than 2 tokens of an
+ * 8192 x 28672 matrix) is rejected with UQ_ERR_UNSUPPORTED before anything
+ * is launched.  Nothing is allocated and nothing is freed: no cudaMalloc,
+ * no cudaFree, no library routine that allocates.
+ *
+ * The first call on a device looks up the scratch's device address (once,
+ * with that device current) and caches it; make that first call before any
+ * stream capture.  All calls share the one scratch array and it keeps the
+ * last call's contents: each call overwrites every word it reads before
+ * reading it, so nothing needs clearing, but two calls whose work overlaps
+ * on the GPU (for instance on two streams) race on it and may give wrong
+ * results.  Order such calls on one stream.
+ */
+uq_status uq_bcq_gemv_noalloc(const uint32_t* bitplanes, const float* alpha_star, const float* zb_star,
+                              int64_t out, int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch,
+                              float* y, void* stream);
+
+/*
  * uq_check_device -- waits for `stream` to finish, then reports whether a
  * pipelined kernel of this library gave up waiting for its own data copies
  * since the last check (every wait on an mbarrier is bounded to about one

@@ -30,7 +30,7 @@ EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
 ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq", "uq_bcq_gemv",
-                "uq_bcq_gemv_workspace_bytes",
+                "uq_bcq_gemv_workspace_bytes", "uq_bcq_gemv_noalloc",
                 "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
 
@@ -69,6 +69,7 @@ def lib() -> ctypes.CDLL:
         L.uq_bcq_gemv.argtypes = [vp, vp, vp, i64, i64, i32, i32, vp, i32, i32, vp, vp, i64, vp]
         L.uq_bcq_gemv_workspace_bytes.argtypes = [i64, i64, i32]
         L.uq_bcq_gemv_workspace_bytes.restype = i64
+        L.uq_bcq_gemv_noalloc.argtypes = [vp, vp, vp, i64, i64, i32, i32, vp, i32, i32, vp, vp]
         f32 = ctypes.c_float
         L.uq_train_step.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, f32, f32, i32, i64, i32, vp,
                                     vp]
@@ -289,6 +290,28 @@ def uq_bcq_gemv(bitplanes, alpha_star, zb_star, x, y, g, workspace=None, stream=
         _check(x, "x", (batch, n_in), x.dtype, dev), _wdtype(x), batch,
         _check(y, "y", (batch, out), torch.float32, dev), workspace.data_ptr(), workspace.numel() * 4,
         _stream(stream, dev))
+    _raise(st)
+
+
+def uq_bcq_gemv_noalloc(bitplanes, alpha_star, zb_star, x, y, g, stream=None):
+    """The BCQ product of uq_bcq_gemv without a workspace: for callers that
+    cannot allocate device memory, it uses 4 MiB of scratch built into the
+    library (shared by all calls; calls that overlap on the GPU race on it).
+    Larger shapes raise UQError (UQ_ERR_UNSUPPORTED)."""
+    if bitplanes.dim() != 3 or x.dim() != 2:
+        raise ValueError("bitplanes must be [q, out, in/32] and x [batch, in]")
+    q, out, words = bitplanes.shape
+    batch, n_in = x.shape
+    if n_in != 32 * words:
+        raise ValueError(f"x has {n_in} columns, the planes {32 * words}")
+    dev = x.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    st = lib().uq_bcq_gemv_noalloc(
+        _check(bitplanes, "bitplanes", (q, out, words), torch.int32, dev),
+        _check(alpha_star, "alpha_star", (out, Gr, q), torch.float32, dev),
+        _check(zb_star, "zb_star", (out, Gr), torch.float32, dev), out, n_in, q, g,
+        _check(x, "x", (batch, n_in), x.dtype, dev), _wdtype(x), batch,
+        _check(y, "y", (batch, out), torch.float32, dev), _stream(stream, dev))
     _raise(st)
 
 

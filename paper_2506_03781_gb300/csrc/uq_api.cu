@@ -207,6 +207,31 @@ uq_status uq_bcq_gemv(const uint32_t* bitplanes, const float* alpha_star, const 
                        "uq_bcq_gemv");
 }
 
+uq_status uq_bcq_gemv_noalloc(const uint32_t* bitplanes, const float* alpha_star, const float* zb_star,
+                              int64_t out, int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch,
+                              float* y, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, xdtype));
+    if (batch < 1 || batch > 64) return fail(UQ_ERR_ARG, "batch=%d must be in 1..64", batch);
+    UQ_TRY(check_ptr(bitplanes, "bitplanes"));
+    UQ_TRY(check_ptr(alpha_star, "alpha_star"));
+    UQ_TRY(check_ptr(zb_star, "zb_star"));
+    UQ_TRY(check_ptr(x, "x"));
+    UQ_TRY(check_ptr(y, "y"));
+    const int64_t need = uq::gemv_workspace_floats(out, in, batch);
+    const int64_t have = uq::gemv_static_workspace_floats();
+    if (need > have)
+        return fail(UQ_ERR_UNSUPPORTED,
+                    "this product needs %lld floats of scratch (ceil(in/512) * batch * out); the built-in scratch "
+                    "holds %lld: pass a workspace to uq_bcq_gemv instead",
+                    (long long)need, (long long)have);
+    float* work = nullptr;
+    const cudaError_t e = uq::gemv_static_workspace(&work);
+    if (e != cudaSuccess) return cuda_status(e, "uq_bcq_gemv_noalloc: looking up the built-in scratch");
+    return cuda_status(uq::launch_gemv(bitplanes, alpha_star, zb_star, out, (int)in, q, g, x, (int)xdtype, batch, y,
+                                       work, (cudaStream_t)stream),
+                       "uq_bcq_gemv_noalloc");
+}
+
 uq_status uq_check_device(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));

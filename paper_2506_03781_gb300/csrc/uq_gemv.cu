@@ -21,6 +21,8 @@
 // SegReduce) leaves one row's tile partial on each of 8 lanes, which store it
 // to the caller's workspace [tile][token][row].  A second kernel sums the
 // partials of a row in tile order.  Deterministic; no atomics.
+#include <atomic>
+
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
@@ -225,6 +227,39 @@ bcq_gemv_reduce_kernel(const float* __restrict__ PART, float* __restrict__ Y, in
 
 int64_t gemv_workspace_floats(int64_t out, int64_t n_in, int batch) {
     return ((n_in + kTileCols - 1) / kTileCols) * (int64_t)batch * out;
+}
+
+// Built-in scratch for uq_bcq_gemv_noalloc: the per-tile partials of one call,
+// for callers that cannot allocate device memory themselves.  4 MiB, held by
+// every GPU that loads the library until the process exits; shared by all
+// calls (a call overwrites every word it later reads, so nothing has to be
+// cleared between calls, but two calls in flight at once race on it).
+constexpr int64_t kStaticWorkFloats = int64_t(1) << 20;
+static __device__ __align__(256) float g_gemv_static_work[kStaticWorkFloats];
+
+int64_t gemv_static_workspace_floats() { return kStaticWorkFloats; }
+
+// Device address of g_gemv_static_work on the current device.  The name is
+// only a host-side stand-in in host code, so the address is looked up once
+// per device with that device current, and cached.
+cudaError_t gemv_static_workspace(float** work) {
+    static std::atomic<float*> cached[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) {
+        float* p = cached[dev].load(std::memory_order_acquire);
+        if (p != nullptr) {
+            *work = p;
+            return cudaSuccess;
+        }
+    }
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_gemv_static_work);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) cached[dev].store(static_cast<float*>(p), std::memory_order_release);
+    *work = static_cast<float*>(p);
+    return cudaSuccess;
 }
 
 template <int Q, typename XT, int NGT>

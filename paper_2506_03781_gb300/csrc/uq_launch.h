@@ -45,6 +45,10 @@ cudaError_t step_error(bool clear, unsigned int* flag);
 // BCQ matrix-vector product from the exported bit-planes (uq_gemv.cu); `work`
 // holds gemv_workspace_floats(out, in, batch) floats of per-tile partials.
 int64_t gemv_workspace_floats(int64_t out, int64_t n_in, int batch);
+// The library's own scratch for the product (uq_bcq_gemv_noalloc): its size in
+// floats, and its device address on the current device (looked up once per device).
+int64_t gemv_static_workspace_floats();
+cudaError_t gemv_static_workspace(float** work);
 cudaError_t launch_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in, int q,
                         int g, const void* x, int xdtype, int batch, float* y, float* work, cudaStream_t st);
 // Launches the bounded-wait self-test (one warp, a wait that runs out).
