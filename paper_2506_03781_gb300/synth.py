@@ -212,3 +212,58 @@ def jitter(params: dict, factors: dict) -> dict:
     for k, f in factors.items():
         outp[k] = (np.asarray(params[k], F32) * f).astype(F32)
     return outp
+
+
+# ---------------------------------------------------------------------------
+# Synthetic Transformer block for the reconstruction loop (Algorithm 1)
+# ---------------------------------------------------------------------------
+
+@dataclass
+class BlockShape:
+    """Shape of a Llama-style decoder block: RMSNorm, grouped-query
+    attention with rotary position embedding, RMSNorm, SwiGLU MLP.  Only the
+    seven linear weights are quantized (norm weights are one)."""
+    name: str
+    d: int               # hidden size
+    heads: int
+    kv_heads: int
+    head_dim: int
+    mlp: int
+    seq: int             # tokens per sample
+    theta: float = 500000.0
+    eps: float = 1e-5
+
+    def matrices(self, std: float = 0.02):
+        """The seven linear weights as (name, out, in) Matrix records."""
+        qd, kd = self.heads * self.head_dim, self.kv_heads * self.head_dim
+        mk = lambda n, o, i: Matrix(n, o, i, "t4", std)
+        return [mk("q_proj", qd, self.d), mk("k_proj", kd, self.d), mk("v_proj", kd, self.d),
+                mk("o_proj", self.d, qd), mk("gate_proj", self.mlp, self.d), mk("up_proj", self.mlp, self.d),
+                mk("down_proj", self.d, self.mlp)]
+
+
+BLOCKS = {
+    # Llama-3-8B block, one calibration sample of 2048 tokens (Sec. 4.1)
+    "llama3_8b": BlockShape("llama3_8b", d=4096, heads=32, kv_heads=8, head_dim=128, mlp=14336, seq=2048),
+    # small blocks of the same structure, for tests
+    "tiny": BlockShape("tiny", d=128, heads=4, kv_heads=2, head_dim=32, mlp=256, seq=16),
+    "small": BlockShape("small", d=512, heads=8, kv_heads=2, head_dim=64, mlp=1024, seq=64),
+}
+
+
+def block_weights(shape: BlockShape, seed):
+    """fp32 values of the seven weights, bf16-rounded (stored raw bits, values)."""
+    out = {}
+    for i, m in enumerate(shape.matrices()):
+        out[m.name] = bf16_round(matrix_weights(m, (seed, i)))
+    return out
+
+
+def block_inputs(shape: BlockShape, n: int, seed, perturb: float = 0.0):
+    """n samples X [seq, d] ~ N(0, 1) (the block's input hidden states) and
+    X^ = X (1 + perturb N(0, 1)), standing for the input of the quantized
+    block after quantized predecessors (Algorithm 1's X^).  fp32."""
+    rng = _rng(seed, 11)
+    X = rng.standard_normal((n, shape.seq, shape.d)).astype(F32)
+    Xh = (X * (1.0 + perturb * rng.standard_normal(X.shape))).astype(F32)
+    return X, Xh
