@@ -343,6 +343,70 @@ def time_gemv(q, g, dev, stream, peak, shapes=((14336, 4096), (8192, 28672)), re
     return res
 
 
+def time_block_step(dev, steps=20, warmup=3, samples=4):
+    """Algorithm 1 on a Llama-3-8B-shaped block (seq 2048, bf16 block
+    compute, the block workload's q and g): ms per optimisation step (block
+    forward + backward in torch, then uq_train_step for the seven weights),
+    the quantizer's share of it, and the share of codes a remap step moves."""
+    import time
+    import torch
+    from paper_2506_03781_gb300 import api, synth
+    from paper_2506_03781_gb300.recon import NAMES, BlockReconstructor
+    wl = synth.WORKLOADS["llama3_8b_block_bf16"]
+    shape = synth.BLOCKS["llama3_8b"]
+    Wb = synth.block_weights(shape, wl.seed)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    rec = BlockReconstructor(shape, {n: Wb[n][0] for n in NAMES}, wl.q, wl.g, device=dev, G=wl.G, T=wl.T)
+    torch.cuda.synchronize()
+    init_s = time.perf_counter() - t0
+    X, Xh = synth.block_inputs(shape, samples, wl.seed, perturb=0.01)
+    Xd = [torch.from_numpy(x).to(dev) for x in X]
+    Xhd = [torch.from_numpy(x).to(dev) for x in Xh]
+    Y = rec.targets(Xd)
+    losses = []
+    for i in range(warmup):
+        losses.append(rec.step(Y[i % samples], Xhd[i % samples]))
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        losses.append(rec.step(Y[i % samples], Xhd[i % samples]))
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    # the quantizer alone: the seven fused steps of one optimisation step
+    q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    q0.record(stream)
+    for i in range(steps):
+        for n in NAMES:
+            rec.qz[n].train_step(rec.t, rec.lr_F, rec.lr_B, rec.p, rec.map_mode)
+        rec.t += 1
+    q1.record(stream)
+    torch.cuda.synchronize()
+    qms = q0.elapsed_time(q1) / steps
+    # codes moved by remap steps (the forward of t + 1 remaps when (t + 1) % p == 0)
+    moved = []
+    for i in range(4):
+        before = {n: rec.codes[n].clone() for n in NAMES}
+        remap = (rec.t + 1) % rec.p == 0
+        rec.step(Y[i % samples], Xhd[i % samples])
+        if remap:
+            ch = sum(int((rec.codes[n] != before[n]).sum()) for n in NAMES)
+            moved.append(ch / sum(rec.codes[n].numel() for n in NAMES))
+    api.uq_check_device(stream)
+    n_w = sum(rec.codes[n].numel() for n in NAMES)
+    res = {"block": shape.name, "seq": shape.seq, "q": wl.q, "g": wl.g, "weights": n_w, "steps": steps,
+           "ms_per_step": ms, "quantizer_ms_per_step": qms, "quantizer_share": qms / ms,
+           "codes_moved_per_remap_step": statistics.mean(moved) if moved else None,
+           "loss_first": float(losses[0]), "loss_last": float(losses[-1]), "init_s": init_s,
+           "paper_step_s_a100_derived": 0.25}
+    del rec, Y, Xd, Xhd
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_gpu(args):
     import torch
     from paper_2506_03781_gb300 import api, roofline, synth
@@ -468,6 +532,9 @@ def run_gpu(args):
     # deployment: the BCQ product from the exported format (one bf16 token)
     gemv = time_gemv(q, g, dev, stream, peak)
 
+    # Algorithm 1 on a Llama-3-8B-shaped block (the quantizer inside the loop)
+    block = None if args.no_block else time_block_step(dev)
+
     # end-to-end through the public host-buffer API: every step uploads its
     # inputs from pinned host memory, runs fwd+bwd and downloads its results;
     # consecutive steps (independent, like successive weight matrices)
@@ -553,6 +620,7 @@ def run_gpu(args):
                            "downloads of consecutive steps overlapped)"},
             "train_step": train,
             "bcq_gemv": gemv,
+            "block_step": block,
             "q_sweep": sweep,
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,
@@ -628,6 +696,7 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle CPU work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true", help="skip the q sweep of the headline matrix")
+    ap.add_argument("--no-block", action="store_true", help="skip the block reconstruction loop timing")
     ap.add_argument("--workloads", action="store_true", help="time the other workloads instead")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)          # at least 3 untimed warm-up steps

@@ -473,7 +473,7 @@ class Quantizer:
     stream at call time.
     """
 
-    def __init__(self, W, q, g, params, codes, W_hat, dL_dWhat, grads):
+    def __init__(self, W, q, g, params, codes, W_hat, dL_dWhat, grads=None):
         self.W, self.q, self.g = W, q, g
         self.out, self.n_in = _dims(W, g)
         self.wd = _wdtype(W)
@@ -487,8 +487,9 @@ class Quantizer:
         Gr = self.n_in // g
         shapes = {"ddelta": (self.out, Gr), "dzu": (self.out, Gr), "ds": (self.out, self.n_in),
                   "dsr": (self.out,), "dalpha": (self.out, Gr, q), "dzb": (self.out, Gr)}
-        self.gr = uq_grads(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev)
-                              for n in GRAD_NAMES})
+        # grads may be None when only the fused train_step is used (it writes no gradients)
+        self.gr = None if grads is None else uq_grads(
+            **{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev) for n in GRAD_NAMES})
         self.wptr = W.data_ptr()
         self.L = lib()
 
@@ -500,6 +501,8 @@ class Quantizer:
                                       map_mode, step, p_period, self.what, self._st(stream)))
 
     def bwd(self, stream=None):
+        if self.gr is None:
+            raise ValueError("this Quantizer was built without gradient buffers")
         _raise(self.L.uq_quantize_bwd(self.wptr, self.wd, self.out, self.n_in, self.q, self.g, self.p, self.codes,
                                       self.G, self.gr, self._st(stream)))
 

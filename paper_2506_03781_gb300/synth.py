@@ -246,7 +246,7 @@ BLOCKS = {
     # Llama-3-8B block, one calibration sample of 2048 tokens (Sec. 4.1)
     "llama3_8b": BlockShape("llama3_8b", d=4096, heads=32, kv_heads=8, head_dim=128, mlp=14336, seq=2048),
     # small blocks of the same structure, for tests
-    "tiny": BlockShape("tiny", d=128, heads=4, kv_heads=2, head_dim=32, mlp=256, seq=16),
+    "tiny": BlockShape("tiny", d=256, heads=4, kv_heads=2, head_dim=64, mlp=512, seq=16),
     "small": BlockShape("small", d=512, heads=8, kv_heads=2, head_dim=64, mlp=1024, seq=64),
 }
 

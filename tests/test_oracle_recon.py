@@ -11,8 +11,8 @@ the quantizer).
 * the loss of W^ = W on X^ = X is zero;
 * one step of the loop is train_step applied per weight to the gradient of
   the loss of the current W^ (composition, against the pieces called
-  separately), and with the paper's learning rates the step lowers the loss
-  on a tiny block.
+  separately), and with the codes held the paper's learning rates lower the
+  loss at every step (plain gradient descent on the block output error).
 """
 
 import math
@@ -128,10 +128,14 @@ def test_step_is_train_step_of_the_loss_gradient_and_lowers_the_loss():
         P1, c1, w1 = O.train_step(W[n], P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], c, G[n], g, 0)
         assert all(np.array_equal(new[n][0][k], P1[k]) for k in P1)
         assert np.array_equal(new[n][1], c1) and np.array_equal(new[n][2], w1)
-    # a few steps on the same sample lower its loss
+    # With the codes held (no remap: p larger than the number of steps) W^ is
+    # a smooth function of Delta, z_U, alpha, z_B, and the steps are plain
+    # gradient descent on it: the loss of the sample goes down at every step.
+    # (Remap steps move codes and may raise it: the mapping is not descended.)
     st, losses = state, []
-    for t in range(6):
-        st, l = R.recon_step(st, W, Ys[0], Xh[0], shape, g, t)
+    for t in range(5):
+        st, l = R.recon_step(st, W, Ys[0], Xh[0], shape, g, t, p=1000)
         losses.append(l)
     after, _ = R.loss_and_grads(Ys[0], Xh[0], {n: st[n][2] for n in R.NAMES}, shape)
-    assert after < losses[0], (losses, after)
+    losses.append(after)
+    assert all(b < a for a, b in zip(losses, losses[1:])), losses
