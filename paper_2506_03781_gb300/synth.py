@@ -215,7 +215,7 @@ def jitter(params: dict, factors: dict) -> dict:
 
 
 # ---------------------------------------------------------------------------
-# Synthetic Transformer block for the reconstruction loop (Algorithm 1)
+# Synthetic decoder block for the reconstruction loop (Algorithm 1)
 # ---------------------------------------------------------------------------
 
 @dataclass
