@@ -43,6 +43,7 @@ __all__ = [
     "transform_F", "map_full", "map_local", "reconstruct", "detransform",
     "quantize_fwd", "quantize_bwd", "bwd_l1_mass",
     "LR_F", "LR_B", "sgd_update", "train_step",
+    "omni_params", "quantize_fwd_omni", "quantize_bwd_omni", "bwd_l1_mass_omni", "export_bcq_omni",
     "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
     "bcq_dequantize", "bcq_gemv",
     "clip_params", "greedy_init", "general_alternating", "unified_init",
@@ -279,6 +280,128 @@ def bwd_l1_mass(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
         dalpha=np.repeat(mass_gbar[..., None], q, axis=-1),
         dsr=np.abs(gbar * fu).sum(axis=(1, 2)) / np.abs(t["sr"]),
     )
+
+
+# ---------------------------------------------------------------------------
+# OmniQuant unified into BCQ (App. E, extensibility): T_O / D_O
+# ---------------------------------------------------------------------------
+
+def omni_params(W, beta, gamma, q, g):
+    """OmniQuant's learnable clipping as UniQuan's transformation parameters.
+
+    Per group, with w_m and w_M the smallest and largest weight:
+      Delta_O = (gamma w_M - beta w_m) / (2^q - 1),
+      z_O     = -round(beta w_m / Delta_O)   (round half to even).
+    fp32: each product rounded, then the difference, then the division.
+    Returns (Delta_O, z_O), fp32 [out, in/g].
+    """
+    out, n_in = np.shape(W)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    wm, wM = Wg.min(-1), Wg.max(-1)
+    beta, gamma = np.asarray(beta, F32), np.asarray(gamma, F32)
+    num = (gamma * wM).astype(F32) - (beta * wm).astype(F32)
+    delta = (num.astype(F32) / F32((1 << q) - 1)).astype(F32)
+    zo = -np.rint(((beta * wm).astype(F32) / delta).astype(F32)).astype(F32)
+    return delta.astype(F32), zo.astype(F32)
+
+
+def quantize_fwd_omni(W, beta, gamma, alpha, zb, codes, g, mode=MAP_LOCAL_PERIODIC, step=0, p=2):
+    """UniQuan with OmniQuant's maps: D_O(M*_B(T_O(w))) (or M_B with MAP_FULL).
+
+    T_O(w) = w / Delta_O + z_O,  D_O(w~) = Delta_O (w~ - z_O)  (fp32, this
+    op order); the mapping and its tie rules are those of quantize_fwd.
+    Returns (w_hat fp32 [out, in], codes uint8 [out, in]).
+    """
+    out, n_in = np.shape(W)
+    q = np.shape(alpha)[-1]
+    delta, zo = omni_params(W, beta, gamma, q, g)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    lv = levels(alpha, zb)
+    srt, cor, roc = sorted_levels(lv)
+    x = ((Wg / delta[..., None]).astype(F32) + zo[..., None]).astype(F32)
+    if mode == MAP_FULL:
+        new = map_full(x, srt, cor)
+    elif step % p == 0:
+        new = map_local(x, _grouped(codes, out, g).astype(np.int64), srt, cor, roc)
+    else:
+        new = _grouped(codes, out, g).astype(np.int64)
+    what = detransform(reconstruct(new, lv), delta, zo)
+    return what.reshape(out, n_in).astype(F32), new.reshape(out, n_in).astype(np.uint8)
+
+
+def _bwd_terms_omni(W, beta, gamma, alpha, zb, codes, Gup, g):
+    out, n_in = np.shape(W)
+    q = np.shape(alpha)[-1]
+    delta, zo = omni_params(W, beta, gamma, q, g)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    cg = _grouped(codes, out, g).astype(np.int64)
+    x32 = ((Wg / delta[..., None]).astype(F32) + zo[..., None]).astype(F32)
+    m32 = reconstruct(cg, levels(alpha, zb))
+    tau = np.min(np.abs(np.asarray(alpha, F32)), axis=-1)
+    f = np.abs(x32 - m32) <= tau[..., None]
+    d64, z64 = delta.astype(F64), zo.astype(F64)
+    u = Wg.astype(F64) / d64[..., None]
+    C = signs(q, F64)[cg]
+    m64 = (C * np.asarray(alpha, F64)[..., None, :]).sum(-1) + np.asarray(zb, F64)[..., None]
+    G = _grouped(np.asarray(Gup, F64), out, g)
+    fu = np.where(f, u, 0.0)
+    wm, wM = Wg.min(-1).astype(F64), Wg.max(-1).astype(F64)
+    return dict(f=f, u=u, m=m64, C=C, G=G, fu=fu, d=d64, z=z64, wm=wm, wM=wM,
+                beta=np.asarray(beta, F64), L1=float((1 << q) - 1))
+
+
+def quantize_bwd_omni(W, beta, gamma, alpha, zb, codes, Gup, g):
+    """Gradients of L w.r.t. (beta, gamma, alpha, z_B) given G = dL/dW^.
+
+    w^ = Delta_O (w~ - z_O) with w~ = c . alpha + z_B (codes fixed), the
+    straight-through path of x = w / Delta_O + z_O filtered as in App. C.1
+    (tau = min_j |alpha_j|), and the rounding in z_O passed straight through
+    (as OmniQuant trains its zero point).  With u = w / Delta_O:
+      A = dL/dDelta_O (z_O held) = sum G ((m - z_O) - f u)
+      B = dL/dz_O                = -Delta_O sum G (1 - f)
+      dDelta/dbeta = -w_m / (2^q - 1),   dDelta/dgamma = w_M / (2^q - 1)
+      dz/dbeta = -(w_m / Delta - beta w_m dDelta/dbeta / Delta^2)
+      dz/dgamma = beta w_m dDelta/dgamma / Delta^2
+      dbeta = A dDelta/dbeta + B dz/dbeta,  dgamma = A dDelta/dgamma + B dz/dgamma
+      dalpha_j = Delta sum G c_j,  dz_B = Delta sum G.
+    Decisions in fp32, values and sums in fp64 (dict of fp64 arrays).
+    """
+    t = _bwd_terms_omni(W, beta, gamma, alpha, zb, codes, Gup, g)
+    d, z, G = t["d"], t["z"], t["G"]
+    A = (G * ((t["m"] - z[..., None]) - t["fu"])).sum(-1)
+    B = -d * (G * (1.0 - t["f"].astype(F64))).sum(-1)
+    dDb, dDg = -t["wm"] / t["L1"], t["wM"] / t["L1"]
+    dzb_ = -(t["wm"] / d - t["beta"] * t["wm"] * dDb / (d * d))
+    dzg_ = t["beta"] * t["wm"] * dDg / (d * d)
+    return dict(
+        dbeta=A * dDb + B * dzb_, dgamma=A * dDg + B * dzg_,
+        dalpha=(d[..., None, None] * G[..., None] * t["C"]).sum(-2), dzb=d * G.sum(-1),
+    )
+
+
+def bwd_l1_mass_omni(W, beta, gamma, alpha, zb, codes, Gup, g):
+    """L1 mass of each reduction of quantize_bwd_omni (fp64), for tolerances."""
+    t = _bwd_terms_omni(W, beta, gamma, alpha, zb, codes, Gup, g)
+    d, z, G = t["d"], t["z"], t["G"]
+    mA = np.abs(G * ((t["m"] - z[..., None]) - t["fu"])).sum(-1)
+    mB = np.abs(d) * np.abs(G * (1.0 - t["f"].astype(F64))).sum(-1)
+    dDb, dDg = -t["wm"] / t["L1"], t["wM"] / t["L1"]
+    dzb_ = -(t["wm"] / d - t["beta"] * t["wm"] * dDb / (d * d))
+    dzg_ = t["beta"] * t["wm"] * dDg / (d * d)
+    q = np.shape(alpha)[-1]
+    mG = np.abs(d) * np.abs(G).sum(-1)
+    return dict(dbeta=mA * np.abs(dDb) + mB * np.abs(dzb_), dgamma=mA * np.abs(dDg) + mB * np.abs(dzg_),
+                dalpha=np.repeat(mG[..., None], q, axis=-1), dzb=mG)
+
+
+def export_bcq_omni(W, beta, gamma, alpha, zb, codes, g):
+    """Theorem 1 for the OmniQuant maps: D_O has the same form as D_R, so
+    alpha* = Delta_O alpha and z_B* = Delta_O (z_B - z_O); the stored codes.
+    Returns (planes, alpha*, z_B*)."""
+    q = np.shape(alpha)[-1]
+    delta, zo = omni_params(W, beta, gamma, q, g)
+    a_star, z_star = unify(delta, zo, alpha, zb)
+    return pack_bitplanes(codes, q), a_star, z_star
 
 
 # ---------------------------------------------------------------------------
