@@ -103,6 +103,23 @@ typedef struct {
     float* dzb;
 } uq_grads;
 
+/* UniQuan with OmniQuant's transformation (App. E, extensibility): per
+ * group the learnable clipping factors beta, gamma of T_O / D_O, and the
+ * BCQ parameters alpha, z_B.  All [out, in/g] (alpha [out, in/g, q]). */
+typedef struct {
+    float* beta;
+    float* gamma;
+    float* alpha;
+    float* zb;
+} uq_params_omni;
+
+typedef struct {
+    float* dbeta;
+    float* dgamma;
+    float* dalpha;
+    float* dzb;
+} uq_grads_omni;
+
 /*
  * uq_init_params -- unified initialization (Algorithm 2 with the general
  * alternating update of Algorithm 3 and the clipping strategies of App. E.2).
@@ -199,6 +216,52 @@ uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
 uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
                         uq_params params, uint8_t* codes, const float* dL_dWhat, float lr_F, float lr_B,
                         uq_map map, int64_t step, int p_period, float* W_hat, void* stream);
+
+/*
+ * uq_quantize_fwd_omni -- the UniQuan quantizer with OmniQuant's maps
+ * (App. E, extensibility) in place of FlexRound's:
+ *   T_O(w) = w / Delta_O + z_O,  D_O(w~) = Delta_O (w~ - z_O),
+ *   Delta_O = (gamma w_M - beta w_m) / (2^q - 1),  z_O = -round(beta w_m / Delta_O)
+ * with w_m, w_M the smallest and largest weight of the group.  fp32 order:
+ * num = gamma * w_M - beta * w_m (each product rounded), Delta_O = num /
+ * (2^q - 1), z_O = -rint((beta * w_m) / Delta_O) (half to even),
+ * x = w / Delta_O + z_O, W_hat = Delta_O * (l(c) - z_O).  The mapping, the
+ * level order and every tie rule are those of uq_quantize_fwd (map, step,
+ * p_period likewise; W is read on every call, also on keep steps).
+ * g in {32, 64, 128, 256, 512}, else UQ_ERR_UNSUPPORTED.  Delta_O must come
+ * out positive (gamma w_M > beta w_m); the caller keeps it so.
+ */
+uq_status uq_quantize_fwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                               uq_params_omni params, uint8_t* codes, uq_map map, int64_t step, int p_period,
+                               float* W_hat, void* stream);
+
+/*
+ * uq_quantize_bwd_omni -- gradients through uq_quantize_fwd_omni with the
+ * straight-through estimator and the gradient filter of App. C.1
+ * (tau = min_j |alpha_j|, f = |x - l(c)| <= tau), and the rounding in z_O
+ * passed straight through.  With u = w / Delta_O and per group
+ *   A = sum G ((l(c) - z_O) - f u),  B = -Delta_O sum G (1 - f):
+ *   dbeta  = A (-w_m / (2^q-1)) + B dz/dbeta,
+ *   dgamma = A ( w_M / (2^q-1)) + B dz/dgamma,
+ *   dz/dbeta = -(w_m / Delta_O - beta w_m (dDelta/dbeta) / Delta_O^2),
+ *   dz/dgamma = beta w_m (dDelta/dgamma) / Delta_O^2,
+ *   dalpha_j = Delta_O sum G c_j,  dz_B = Delta_O sum G.
+ * Every grads pointer is written (overwritten).  Group sums are reduced
+ * inside the group's lanes; fp32; deterministic.  Shapes as the forward.
+ */
+uq_status uq_quantize_bwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                               uq_params_omni params, const uint8_t* codes, const float* dL_dWhat,
+                               uq_grads_omni grads, void* stream);
+
+/*
+ * uq_omni_scales -- Delta_O and z_O of every group (the fp32 values the
+ * forward uses), written to delta [out, in/g] and zo [out, in/g].  With them
+ * the export of the OmniQuant-unified quantizer is uq_export_bcq with
+ * params.delta = delta and params.zu = zo (D_O has D_R's form, so Theorem 1
+ * gives alpha* = Delta_O alpha, z_B* = Delta_O (z_B - z_O)).
+ */
+uq_status uq_omni_scales(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                         const float* beta, const float* gamma, float* delta, float* zo, void* stream);
 
 /*
  * uq_export_bcq -- Theorem 1 and the final binary codes (the last two

@@ -28,8 +28,11 @@ LR_THETA_F, LR_THETA_B = 0.005, 0.0005     # learning rates of the hyperparamete
 EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
+OMNI_PARAM_NAMES = ("beta", "gamma", "alpha", "zb")
+OMNI_GRAD_NAMES = ("dbeta", "dgamma", "dalpha", "dzb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
-ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq", "uq_bcq_gemv",
+ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
+                "uq_quantize_fwd_omni", "uq_quantize_bwd_omni", "uq_omni_scales", "uq_bcq_gemv",
                 "uq_bcq_gemv_workspace_bytes", "uq_bcq_gemv_noalloc",
                 "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
@@ -50,6 +53,14 @@ class uq_grads(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in GRAD_NAMES]
 
 
+class uq_params_omni(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in OMNI_PARAM_NAMES]
+
+
+class uq_grads_omni(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in OMNI_GRAD_NAMES]
+
+
 _lib = None
 
 
@@ -66,6 +77,9 @@ def lib() -> ctypes.CDLL:
         L.uq_quantize_fwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, vp]
         L.uq_export_bcq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
+        L.uq_quantize_fwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, i32, i64, i32, vp, vp]
+        L.uq_quantize_bwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, vp, uq_grads_omni, vp]
+        L.uq_omni_scales.argtypes = [vp, i32, i64, i64, i32, i32, vp, vp, vp, vp, vp]
         L.uq_bcq_gemv.argtypes = [vp, vp, vp, i64, i64, i32, i32, vp, i32, i32, vp, vp, i64, vp]
         L.uq_bcq_gemv_workspace_bytes.argtypes = [i64, i64, i32]
         L.uq_bcq_gemv_workspace_bytes.restype = i64
@@ -250,6 +264,52 @@ def uq_export_bcq(W, q, g, params, codes, bitplanes, alpha_star, zb_star, mode=E
         cptr, mode, _check(bitplanes, "bitplanes", (q, out, n_in // 32), torch.int32, dev),
         _check(alpha_star, "alpha_star", (out, Gr, q), torch.float32, dev),
         _check(zb_star, "zb_star", (out, Gr), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def _omni_params(p, out, n_in, q, g, device):
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"beta": (out, Gr), "gamma": (out, Gr), "alpha": (out, Gr, q), "zb": (out, Gr)}
+    return uq_params_omni(**{n: _check(p[n], f"params['{n}']", shapes[n], torch.float32, device)
+                             for n in OMNI_PARAM_NAMES})
+
+
+def uq_quantize_fwd_omni(W, q, g, params, codes, W_hat, map_mode=MAP_LOCAL_PERIODIC, step=0, p_period=2,
+                         stream=None):
+    """UniQuan with OmniQuant's T_O / D_O (params: beta, gamma, alpha, zb) into ``W_hat``."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    st = lib().uq_quantize_fwd_omni(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _omni_params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev), map_mode, step, p_period,
+        _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_quantize_bwd_omni(W, q, g, params, codes, dL_dWhat, grads, stream=None):
+    """Gradients w.r.t. beta, gamma, alpha, zb of the OmniQuant-unified quantizer."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"dbeta": (out, Gr), "dgamma": (out, Gr), "dalpha": (out, Gr, q), "dzb": (out, Gr)}
+    gp = uq_grads_omni(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev)
+                          for n in OMNI_GRAD_NAMES})
+    st = lib().uq_quantize_bwd_omni(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _omni_params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), gp, _stream(stream, dev))
+    _raise(st)
+
+
+def uq_omni_scales(W, q, g, beta, gamma, delta, zo, stream=None):
+    """Delta_O and z_O of every group (for uq_export_bcq with delta/zu = delta/zo)."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    st = lib().uq_omni_scales(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _check(beta, "beta", (out, Gr), torch.float32, dev),
+        _check(gamma, "gamma", (out, Gr), torch.float32, dev), _check(delta, "delta", (out, Gr), torch.float32, dev),
+        _check(zo, "zo", (out, Gr), torch.float32, dev), _stream(stream, dev))
     _raise(st)
 
 

@@ -161,6 +161,59 @@ uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                        "uq_train_step");
 }
 
+uq_status uq_quantize_fwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                               uq_params_omni p, uint8_t* codes, uq_map map, int64_t step, int p_period,
+                               float* W_hat, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::omni_ok(sh)) return fail(UQ_ERR_UNSUPPORTED, "g=%d: the OmniQuant maps take g in {32, 64, 128, 256, 512}", g);
+    if (map != UQ_MAP_FULL && map != UQ_MAP_LOCAL_PERIODIC) return fail(UQ_ERR_ARG, "unknown mapping %d", (int)map);
+    if (p_period < 1) return fail(UQ_ERR_ARG, "p_period=%d must be >= 1", p_period);
+    if (step < 0) return fail(UQ_ERR_ARG, "step=%lld must be >= 0", (long long)step);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.beta, "params.beta"));
+    UQ_TRY(check_ptr(p.gamma, "params.gamma"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(W_hat, "W_hat"));
+    const int mode = map == UQ_MAP_FULL ? uq::FWD_FULL : (step % p_period == 0 ? uq::FWD_REMAP : uq::FWD_KEEP);
+    return cuda_status(uq::launch_omni_fwd(sh, W, p, codes, mode, W_hat, (cudaStream_t)stream), "uq_quantize_fwd_omni");
+}
+
+uq_status uq_quantize_bwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                               uq_params_omni p, const uint8_t* codes, const float* dL_dWhat, uq_grads_omni gr,
+                               void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::omni_ok(sh)) return fail(UQ_ERR_UNSUPPORTED, "g=%d: the OmniQuant maps take g in {32, 64, 128, 256, 512}", g);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.beta, "params.beta"));
+    UQ_TRY(check_ptr(p.gamma, "params.gamma"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(gr.dbeta, "grads.dbeta"));
+    UQ_TRY(check_ptr(gr.dgamma, "grads.dgamma"));
+    UQ_TRY(check_ptr(gr.dalpha, "grads.dalpha"));
+    UQ_TRY(check_ptr(gr.dzb, "grads.dzb"));
+    return cuda_status(uq::launch_omni_bwd(sh, W, p, codes, dL_dWhat, gr, (cudaStream_t)stream), "uq_quantize_bwd_omni");
+}
+
+uq_status uq_omni_scales(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, const float* beta,
+                         const float* gamma, float* delta, float* zo, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::omni_ok(sh)) return fail(UQ_ERR_UNSUPPORTED, "g=%d: the OmniQuant maps take g in {32, 64, 128, 256, 512}", g);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(beta, "beta"));
+    UQ_TRY(check_ptr(gamma, "gamma"));
+    UQ_TRY(check_ptr(delta, "delta"));
+    UQ_TRY(check_ptr(zo, "zo"));
+    return cuda_status(uq::launch_omni_scales(sh, W, beta, gamma, delta, zo, (cudaStream_t)stream), "uq_omni_scales");
+}
+
 uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
                         const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes, float* alpha_star,
                         float* zb_star, void* stream) {

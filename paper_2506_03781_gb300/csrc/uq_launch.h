@@ -51,6 +51,14 @@ int64_t gemv_static_workspace_floats();
 cudaError_t gemv_static_workspace(float** work);
 cudaError_t launch_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in, int q,
                         int g, const void* x, int xdtype, int batch, float* y, float* work, cudaStream_t st);
+// UniQuan with OmniQuant's maps (uq_omni.cu); omni_ok: the group sizes it takes.
+bool omni_ok(const Shape& sh);
+cudaError_t launch_omni_fwd(const Shape& sh, const void* W, uq_params_omni p, uint8_t* codes, int mode, float* what,
+                            cudaStream_t st);
+cudaError_t launch_omni_bwd(const Shape& sh, const void* W, uq_params_omni p, const uint8_t* codes, const float* gup,
+                            uq_grads_omni gr, cudaStream_t st);
+cudaError_t launch_omni_scales(const Shape& sh, const void* W, const float* beta, const float* gamma, float* delta,
+                               float* zo, cudaStream_t st);
 // Launches the bounded-wait self-test (one warp, a wait that runs out).
 cudaError_t launch_wait_selftest(cudaStream_t st);
 // Streaming multiprocessors of the current device (cached per device).

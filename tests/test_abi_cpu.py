@@ -200,6 +200,29 @@ def test_bcq_gemv_workspace_size(libpath):
         assert api.uq_bcq_gemv_workspace_bytes(*bad) == -1
 
 
+@cpu_only
+def test_omni_validation(libpath):
+    from paper_2506_03781_gb300 import api
+    L = api.lib()
+    P = lambda **o: api.uq_params_omni(**{**{n: FAKE + 0x1000 * i for i, n in enumerate(api.OMNI_PARAM_NAMES)}, **o})
+    Gd = lambda **o: api.uq_grads_omni(**{**{n: FAKE + 0x10000 + 0x1000 * i for i, n in enumerate(api.OMNI_GRAD_NAMES)},
+                                         **o})
+    fwd = lambda g=128, n_in=512, p=None, **k: L.uq_quantize_fwd_omni(
+        k.get("W", FAKE), 1, 8, n_in, 3, g, p or P(), FAKE + 0x9000, k.get("map", 1), 0, 2, FAKE + 0xA000, None)
+    assert fwd(g=1024, n_in=2048) == api.UQ_ERR_UNSUPPORTED
+    assert fwd(g=384, n_in=768) == api.UQ_ERR_UNSUPPORTED
+    assert fwd(W=0) == api.UQ_ERR_ARG
+    assert fwd(p=P(beta=0)) == api.UQ_ERR_ARG
+    assert fwd(p=P(gamma=FAKE + 4)) == api.UQ_ERR_ALIGN
+    assert fwd(map=7) == api.UQ_ERR_ARG
+    assert fwd() == api.UQ_ERR_CUDA                                   # valid: only the launch fails here
+    bwd = lambda gr: L.uq_quantize_bwd_omni(FAKE, 1, 8, 512, 3, 128, P(), FAKE + 0x9000, FAKE + 0xB000, gr, None)
+    for f in api.OMNI_GRAD_NAMES:
+        assert bwd(Gd(**{f: 0})) == api.UQ_ERR_ARG and f in api.uq_last_error()
+    assert L.uq_omni_scales(FAKE, 1, 8, 512, 3, 128, FAKE, FAKE, 0, FAKE, None) == api.UQ_ERR_ARG
+    assert L.uq_omni_scales(FAKE, 1, 8, 768, 3, 96, FAKE, FAKE, FAKE, FAKE, None) == api.UQ_ERR_UNSUPPORTED
+
+
 def test_binding_rejects_host_tensors_before_calling(libpath):
     import torch
     from paper_2506_03781_gb300 import api
