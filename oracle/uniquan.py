@@ -44,6 +44,7 @@ __all__ = [
     "quantize_fwd", "quantize_bwd", "bwd_l1_mass",
     "LR_F", "LR_B", "sgd_update", "train_step",
     "omni_params", "quantize_fwd_omni", "quantize_bwd_omni", "bwd_l1_mass_omni", "export_bcq_omni",
+    "quantize_fwd_awq", "quantize_bwd_awq", "bwd_l1_mass_awq", "export_bcq_awq",
     "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
     "bcq_dequantize", "bcq_gemv",
     "clip_params", "greedy_init", "general_alternating", "unified_init",
@@ -402,6 +403,107 @@ def export_bcq_omni(W, beta, gamma, alpha, zb, codes, g):
     delta, zo = omni_params(W, beta, gamma, q, g)
     a_star, z_star = unify(delta, zo, alpha, zb)
     return pack_bitplanes(codes, q), a_star, z_star
+
+
+# ---------------------------------------------------------------------------
+# AWQ unified into BCQ (App. E, extensibility): T_A / D_A
+# ---------------------------------------------------------------------------
+
+def quantize_fwd_awq(W, sa, delta, za, alpha, zb, codes, g, mode=MAP_LOCAL_PERIODIC, step=0, p=2):
+    """UniQuan with AWQ's maps: D_A(M*_B(T_A(w))) (or M_B with MAP_FULL).
+
+    T_A(w) = (w * s_A) / Delta_A + z_A,  D_A(w~) = Delta_A (w~ - z_A) / s_A,
+    s_A [in] one scale per column (shared by every row), Delta_A, z_A per
+    group.  (The printed D_A subtracts z_O; it is read as z_A, the zero point
+    of T_A.)  fp32, in this order: x = ((w s) / Delta) + z,
+    w^ = (Delta (w~ - z)) / s.  Mapping and tie rules as quantize_fwd.
+    """
+    out, n_in = np.shape(W)
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    sg = np.broadcast_to(np.asarray(sa, F32).reshape(1, -1, g), Wg.shape)
+    delta, za = np.asarray(delta, F32), np.asarray(za, F32)
+    lv = levels(alpha, zb)
+    srt, cor, roc = sorted_levels(lv)
+    x = (((Wg * sg).astype(F32) / delta[..., None]).astype(F32) + za[..., None]).astype(F32)
+    if mode == MAP_FULL:
+        new = map_full(x, srt, cor)
+    elif step % p == 0:
+        new = map_local(x, _grouped(codes, out, g).astype(np.int64), srt, cor, roc)
+    else:
+        new = _grouped(codes, out, g).astype(np.int64)
+    wt = reconstruct(new, lv)
+    what = ((delta[..., None] * (wt - za[..., None]).astype(F32)).astype(F32) / sg).astype(F32)
+    return what.reshape(out, n_in), new.reshape(out, n_in).astype(np.uint8)
+
+
+def _bwd_terms_awq(W, sa, delta, za, alpha, zb, codes, Gup, g):
+    out, n_in = np.shape(W)
+    q = np.shape(alpha)[-1]
+    Wg = _grouped(np.asarray(W, F32), out, g)
+    s32 = np.broadcast_to(np.asarray(sa, F32).reshape(1, -1, g), Wg.shape)
+    cg = _grouped(codes, out, g).astype(np.int64)
+    x32 = (((Wg * s32).astype(F32) / np.asarray(delta, F32)[..., None]).astype(F32)
+           + np.asarray(za, F32)[..., None]).astype(F32)
+    m32 = reconstruct(cg, levels(alpha, zb))
+    tau = np.min(np.abs(np.asarray(alpha, F32)), axis=-1)
+    f = np.abs(x32 - m32) <= tau[..., None]
+    d, z = np.asarray(delta, F64)[..., None], np.asarray(za, F64)[..., None]
+    s = s32.astype(F64)
+    w = Wg.astype(F64)
+    u = w * s / d
+    C = signs(q, F64)[cg]
+    m = (C * np.asarray(alpha, F64)[..., None, :]).sum(-1) + np.asarray(zb, F64)[..., None]
+    G = _grouped(np.asarray(Gup, F64), out, g)
+    return dict(f=f, fl=f.astype(F64), u=u, m=m, C=C, G=G, d=d, z=z, s=s, w=w)
+
+
+def quantize_bwd_awq(W, sa, delta, za, alpha, zb, codes, Gup, g):
+    """Gradients of L w.r.t. (Delta_A, z_A, s_A, alpha, z_B) given G = dL/dW^.
+
+    w^ = Delta (w~ - z) / s with w~ = c . alpha + z_B (codes fixed) and the
+    straight-through path of x = w s / Delta + z filtered as in App. C.1.
+    With u = w s / Delta:
+      dDelta = sum G ((m - z) - f u) / s
+      dz_A   = -Delta sum G (1 - f) / s
+      ds_A[col] = sum over the rows of G (f w - Delta (m - z) / s) / s
+      dalpha_j = Delta sum G c_j / s,  dz_B = Delta sum G / s.
+    Decisions in fp32, values and sums in fp64.
+    """
+    t = _bwd_terms_awq(W, sa, delta, za, alpha, zb, codes, Gup, g)
+    G, s, d, z, m, fl = t["G"], t["s"], t["d"], t["z"], t["m"], t["fl"]
+    out, n_in = np.shape(W)
+    Gs = G / s
+    return dict(
+        ddelta=(Gs * ((m - z) - fl * t["u"])).sum(-1),
+        dza=-(d[..., 0] * (Gs * (1.0 - fl)).sum(-1)),
+        dsa=(Gs * (fl * t["w"] - d * (m - z) / s)).reshape(out, n_in).sum(0),
+        dalpha=(d[..., None] * Gs[..., None] * t["C"]).sum(-2), dzb=d[..., 0] * Gs.sum(-1),
+    )
+
+
+def bwd_l1_mass_awq(W, sa, delta, za, alpha, zb, codes, Gup, g):
+    """L1 mass of each reduction of quantize_bwd_awq (fp64), for tolerances."""
+    t = _bwd_terms_awq(W, sa, delta, za, alpha, zb, codes, Gup, g)
+    G, s, d, z, m, fl = t["G"], t["s"], t["d"], t["z"], t["m"], t["fl"]
+    out, n_in = np.shape(W)
+    q = np.shape(alpha)[-1]
+    Gs = np.abs(G / s)
+    mg = np.abs(d[..., 0]) * Gs.sum(-1)
+    return dict(ddelta=(Gs * np.abs((m - z) - fl * t["u"])).sum(-1), dza=np.abs(d[..., 0]) * (Gs * (1.0 - fl)).sum(-1),
+                dsa=(Gs * (np.abs(fl * t["w"]) + np.abs(d * (m - z) / s))).reshape(out, n_in).sum(0),
+                dalpha=np.repeat(mg[..., None], q, axis=-1), dzb=mg)
+
+
+def export_bcq_awq(sa, delta, za, alpha, zb, codes, g):
+    """Theorem 1 for the AWQ maps: D_A = D_R followed by the column scale
+    1 / s_A, so alpha* = Delta_A alpha, z_B* = Delta_A (z_B - z_A) and the
+    column scale stays outside the BCQ weights (AWQ folds 1/s_A into the
+    activations: W^ x = (C alpha* + z_B*) (x / s_A)).
+    Returns (planes, alpha*, z_B*, 1 / s_A)."""
+    q = np.shape(alpha)[-1]
+    a_star, z_star = unify(delta, za, alpha, zb)
+    inv = (F32(1.0) / np.asarray(sa, F32)).astype(F32)
+    return pack_bitplanes(codes, q), a_star, z_star, inv
 
 
 # ---------------------------------------------------------------------------
