@@ -120,6 +120,25 @@ typedef struct {
     float* dzb;
 } uq_grads_omni;
 
+/* UniQuan with AWQ's transformation (App. E, extensibility): sa [in] one
+ * scale per column (shared by every row), delta and za [out, in/g] per
+ * group, and the BCQ parameters alpha [out, in/g, q], zb [out, in/g]. */
+typedef struct {
+    float* sa;
+    float* delta;
+    float* za;
+    float* alpha;
+    float* zb;
+} uq_params_awq;
+
+typedef struct {
+    float* dsa;
+    float* ddelta;
+    float* dza;
+    float* dalpha;
+    float* dzb;
+} uq_grads_awq;
+
 /*
  * uq_init_params -- unified initialization (Algorithm 2 with the general
  * alternating update of Algorithm 3 and the clipping strategies of App. E.2).
@@ -262,6 +281,43 @@ uq_status uq_quantize_bwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int
  */
 uq_status uq_omni_scales(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
                          const float* beta, const float* gamma, float* delta, float* zo, void* stream);
+
+/*
+ * uq_quantize_fwd_awq -- the UniQuan quantizer with AWQ's maps (App. E,
+ * extensibility): T_A(w) = (w s_A) / Delta_A + z_A and
+ * D_A(w~) = Delta_A (w~ - z_A) / s_A (the printed D_A subtracts z_O; read
+ * as z_A).  fp32 order: x = ((w * s_A) / Delta_A) + z_A,
+ * W_hat = (Delta_A * (l(c) - z_A)) / s_A.  Mapping, level order and tie
+ * rules as uq_quantize_fwd (map, step, p_period likewise; W is not read on
+ * keep steps).  g in {32, 64, 128, 256, 512}, else UQ_ERR_UNSUPPORTED.
+ * The export is uq_export_bcq with params.delta = delta, params.zu = za
+ * (alpha* = Delta_A alpha, z_B* = Delta_A (z_B - z_A)); the column scale
+ * 1 / s_A stays outside the BCQ weights (applied to the activations).
+ */
+uq_status uq_quantize_fwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                              uq_params_awq params, uint8_t* codes, uq_map map, int64_t step, int p_period,
+                              float* W_hat, void* stream);
+
+/*
+ * uq_quantize_bwd_awq -- gradients through uq_quantize_fwd_awq with the
+ * straight-through estimator and the gradient filter of App. C.1.  With
+ * u = w s / Delta and f = |x - l(c)| <= min_j |alpha_j|:
+ *   dDelta = sum G ((l(c) - z) - f u) / s,   dz_A = -Delta sum G (1 - f) / s,
+ *   ds_A[col] = sum over the rows of G (f w - Delta (l(c) - z) / s) / s,
+ *   dalpha_j = Delta sum G c_j / s,          dz_B = Delta sum G / s.
+ * ds_A sums over every row of its column: per-row-range partials go to
+ * `workspace` (caller-owned device memory of at least
+ * uq_awq_bwd_workspace_bytes(out, in, q, g) bytes, overwritten) and are
+ * summed in range order.  fp32, deterministic.  A too small workspace is
+ * UQ_ERR_ARG.
+ */
+uq_status uq_quantize_bwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                              uq_params_awq params, const uint8_t* codes, const float* dL_dWhat,
+                              uq_grads_awq grads, float* workspace, int64_t workspace_bytes, void* stream);
+
+/* Bytes of workspace uq_quantize_bwd_awq needs (or -1 for an invalid shape).
+ * It depends on the current device's SM count; query it on that device. */
+int64_t uq_awq_bwd_workspace_bytes(int64_t out, int64_t in, int q, int g);
 
 /*
  * uq_export_bcq -- Theorem 1 and the final binary codes (the last two

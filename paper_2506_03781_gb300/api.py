@@ -30,9 +30,12 @@ EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 OMNI_PARAM_NAMES = ("beta", "gamma", "alpha", "zb")
 OMNI_GRAD_NAMES = ("dbeta", "dgamma", "dalpha", "dzb")
+AWQ_PARAM_NAMES = ("sa", "delta", "za", "alpha", "zb")
+AWQ_GRAD_NAMES = ("dsa", "ddelta", "dza", "dalpha", "dzb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
 ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
-                "uq_quantize_fwd_omni", "uq_quantize_bwd_omni", "uq_omni_scales", "uq_bcq_gemv",
+                "uq_quantize_fwd_omni", "uq_quantize_bwd_omni", "uq_omni_scales",
+                "uq_quantize_fwd_awq", "uq_quantize_bwd_awq", "uq_awq_bwd_workspace_bytes", "uq_bcq_gemv",
                 "uq_bcq_gemv_workspace_bytes", "uq_bcq_gemv_noalloc",
                 "uq_check_device", "uq_selftest_wait_timeout", "uq_last_error", "uq_abi_version")
 
@@ -61,6 +64,14 @@ class uq_grads_omni(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in OMNI_GRAD_NAMES]
 
 
+class uq_params_awq(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in AWQ_PARAM_NAMES]
+
+
+class uq_grads_awq(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in AWQ_GRAD_NAMES]
+
+
 _lib = None
 
 
@@ -80,6 +91,11 @@ def lib() -> ctypes.CDLL:
         L.uq_quantize_fwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, vp, uq_grads_omni, vp]
         L.uq_omni_scales.argtypes = [vp, i32, i64, i64, i32, i32, vp, vp, vp, vp, vp]
+        L.uq_quantize_fwd_awq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_awq, vp, i32, i64, i32, vp, vp]
+        L.uq_quantize_bwd_awq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_awq, vp, vp, uq_grads_awq, vp, i64,
+                                          vp]
+        L.uq_awq_bwd_workspace_bytes.argtypes = [i64, i64, i32, i32]
+        L.uq_awq_bwd_workspace_bytes.restype = i64
         L.uq_bcq_gemv.argtypes = [vp, vp, vp, i64, i64, i32, i32, vp, i32, i32, vp, vp, i64, vp]
         L.uq_bcq_gemv_workspace_bytes.argtypes = [i64, i64, i32]
         L.uq_bcq_gemv_workspace_bytes.restype = i64
@@ -310,6 +326,49 @@ def uq_omni_scales(W, q, g, beta, gamma, delta, zo, stream=None):
         W.data_ptr(), _wdtype(W), out, n_in, q, g, _check(beta, "beta", (out, Gr), torch.float32, dev),
         _check(gamma, "gamma", (out, Gr), torch.float32, dev), _check(delta, "delta", (out, Gr), torch.float32, dev),
         _check(zo, "zo", (out, Gr), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def _awq_params(p, out, n_in, q, g, device, need=AWQ_PARAM_NAMES):
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"sa": (n_in,), "delta": (out, Gr), "za": (out, Gr), "alpha": (out, Gr, q), "zb": (out, Gr)}
+    return uq_params_awq(**{n: _check(p[n], f"params['{n}']", shapes[n], torch.float32, device)
+                            for n in AWQ_PARAM_NAMES})
+
+
+def uq_quantize_fwd_awq(W, q, g, params, codes, W_hat, map_mode=MAP_LOCAL_PERIODIC, step=0, p_period=2,
+                        stream=None):
+    """UniQuan with AWQ's T_A / D_A (params: sa [in], delta, za, alpha, zb) into ``W_hat``."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    st = lib().uq_quantize_fwd_awq(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _awq_params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev), map_mode, step, p_period,
+        _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_awq_bwd_workspace_bytes(out, n_in, q, g) -> int:
+    """Bytes of device workspace uq_quantize_bwd_awq needs on the current device (-1: invalid shape)."""
+    return int(lib().uq_awq_bwd_workspace_bytes(out, n_in, q, g))
+
+
+def uq_quantize_bwd_awq(W, q, g, params, codes, dL_dWhat, grads, workspace=None, stream=None):
+    """Gradients w.r.t. sa, delta, za, alpha, zb of the AWQ-unified quantizer (workspace allocated if None)."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"dsa": (n_in,), "ddelta": (out, Gr), "dza": (out, Gr), "dalpha": (out, Gr, q), "dzb": (out, Gr)}
+    gp = uq_grads_awq(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev)
+                         for n in AWQ_GRAD_NAMES})
+    if workspace is None:
+        nbytes = uq_awq_bwd_workspace_bytes(out, n_in, q, g)
+        workspace = torch.empty(max(nbytes // 4, 4), dtype=torch.float32, device=dev)
+    st = lib().uq_quantize_bwd_awq(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _awq_params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), gp, workspace.data_ptr(),
+        workspace.numel() * 4, _stream(stream, dev))
     _raise(st)
 
 

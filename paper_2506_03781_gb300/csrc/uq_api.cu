@@ -214,6 +214,62 @@ uq_status uq_omni_scales(const void* W, uq_wdtype wdtype, int64_t out, int64_t i
     return cuda_status(uq::launch_omni_scales(sh, W, beta, gamma, delta, zo, (cudaStream_t)stream), "uq_omni_scales");
 }
 
+uq_status uq_quantize_fwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                              uq_params_awq p, uint8_t* codes, uq_map map, int64_t step, int p_period, float* W_hat,
+                              void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::awq_ok(sh)) return fail(UQ_ERR_UNSUPPORTED, "g=%d: the AWQ maps take g in {32, 64, 128, 256, 512}", g);
+    if (map != UQ_MAP_FULL && map != UQ_MAP_LOCAL_PERIODIC) return fail(UQ_ERR_ARG, "unknown mapping %d", (int)map);
+    if (p_period < 1) return fail(UQ_ERR_ARG, "p_period=%d must be >= 1", p_period);
+    if (step < 0) return fail(UQ_ERR_ARG, "step=%lld must be >= 0", (long long)step);
+    const int mode = map == UQ_MAP_FULL ? uq::FWD_FULL : (step % p_period == 0 ? uq::FWD_REMAP : uq::FWD_KEEP);
+    if (mode != uq::FWD_KEEP) UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.sa, "params.sa"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.za, "params.za"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(W_hat, "W_hat"));
+    return cuda_status(uq::launch_awq_fwd(sh, W, p, codes, mode, W_hat, (cudaStream_t)stream), "uq_quantize_fwd_awq");
+}
+
+int64_t uq_awq_bwd_workspace_bytes(int64_t out, int64_t in, int q, int g) {
+    if (q < 1 || q > 4 || out < 1 || in < 1 || g < 32 || in % g != 0 || in > kMaxIn || out > 0x7fffffffLL) return -1;
+    const uq::Shape sh{out, (int)in, q, g, UQ_W_BF16};
+    if (!uq::awq_ok(sh)) return -1;
+    return uq::awq_workspace_floats(sh) * (int64_t)sizeof(float);
+}
+
+uq_status uq_quantize_bwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                              uq_params_awq p, const uint8_t* codes, const float* dL_dWhat, uq_grads_awq gr,
+                              float* workspace, int64_t workspace_bytes, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::awq_ok(sh)) return fail(UQ_ERR_UNSUPPORTED, "g=%d: the AWQ maps take g in {32, 64, 128, 256, 512}", g);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.sa, "params.sa"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.za, "params.za"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(gr.dsa, "grads.dsa"));
+    UQ_TRY(check_ptr(gr.ddelta, "grads.ddelta"));
+    UQ_TRY(check_ptr(gr.dza, "grads.dza"));
+    UQ_TRY(check_ptr(gr.dalpha, "grads.dalpha"));
+    UQ_TRY(check_ptr(gr.dzb, "grads.dzb"));
+    UQ_TRY(check_ptr(workspace, "workspace"));
+    const int64_t need = uq::awq_workspace_floats(sh) * (int64_t)sizeof(float);
+    if (workspace_bytes < need)
+        return fail(UQ_ERR_ARG, "workspace of %lld bytes; the backward needs %lld (uq_awq_bwd_workspace_bytes)",
+                    (long long)workspace_bytes, (long long)need);
+    return cuda_status(uq::launch_awq_bwd(sh, W, p, codes, dL_dWhat, gr, workspace, (cudaStream_t)stream),
+                       "uq_quantize_bwd_awq");
+}
+
 uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
                         const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes, float* alpha_star,
                         float* zb_star, void* stream) {

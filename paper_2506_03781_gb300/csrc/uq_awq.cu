@@ -1,0 +1,312 @@
+// UniQuan with AWQ's transformation (App. E, extensibility): the BCQ
+// mapping, levels and gradient filter of UniQuan_F with
+//   T_A(w) = (w s_A) / Delta_A + z_A,   D_A(w~) = Delta_A (w~ - z_A) / s_A,
+// s_A one scale per column (shared by every row), Delta_A and z_A per group.
+//
+// Decomposition: column stripes x row ranges.  Thread block (cb, rb) has 8
+// warps; warp w owns work unit cb * 8 + w (NG whole groups, the lane mapping
+// of uq_common.cuh, every lane holding all of its group elements: g <= 512)
+// and walks the rows of range rb one after the other.  The unit's s_A is
+// loaded once.  The backward writes the per-row group gradients directly and
+// accumulates ds_A of its columns over its rows in registers; the range's
+// partials go to a workspace [row range][in] and a second kernel sums them in
+// range order.  Deterministic, no atomics.  HBM traffic per element (bf16 W):
+// forward remap 2 + 1 read, 4 + 1 written; backward 2 + 1 + 4 read.
+#include "uq_common.cuh"
+#include "uq_launch.h"
+
+namespace uq {
+
+#ifndef UQ_AWQ_MIN_BLOCKS
+#define UQ_AWQ_MIN_BLOCKS 3
+#endif
+#ifndef UQ_AWQ_BWD_MIN_BLOCKS
+#define UQ_AWQ_BWD_MIN_BLOCKS 2          // the backward also keeps the unit's s_A and ds_A partials in registers
+#endif
+
+constexpr int kAwqTargetBlocksPerSm = 4;
+
+template <int Q, typename WT, int LPG, int MODE>
+__global__ void __launch_bounds__(kThreads, UQ_AWQ_MIN_BLOCKS)
+awq_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const float* __restrict__ DELTA,
+               const float* __restrict__ ZA, const float* __restrict__ ALPHA, const float* __restrict__ ZB,
+               uint8_t* __restrict__ CODES, float* __restrict__ WHAT, int64_t out, int n_in, int g,
+               int64_t rows_per_range) {
+    constexpr int L = 1 << Q;
+    constexpr int NG = 32 / LPG;
+    __shared__ MapTab<Q, NG> tabs[kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    MapTab<Q, NG>& t = tabs[warp];
+    const int Gr = n_in / g;
+    const int u = blockIdx.x * kWarps + warp;
+    if (u * NG >= Gr) return;                     // no block barrier in this kernel
+    const int64_t r0 = (int64_t)blockIdx.y * rows_per_range;
+    const int64_t r1 = r0 + rows_per_range < out ? r0 + rows_per_range : out;
+    const int nv = g / (4 * LPG);
+    const int sub = lane / LPG, li = lane % LPG;
+    const int gi = u * NG + sub;
+    const bool ok = gi < Gr;
+    const int64_t cbase = (int64_t)gi * g + 4 * li;       // first column of this lane's vector 0
+    float s[4][4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v)
+        if (ok && v < nv) f4_to(ldg4(SA + cbase + 4 * LPG * v), s[v]);
+
+    for (int64_t row = r0; row < r1; ++row) {
+        const int64_t grp = row * Gr + gi;
+        const int64_t ebase = row * (int64_t)n_in + cbase;
+        float w[4][4];
+        uint32_t cv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            if (ok && v < nv) {
+                const int64_t e = ebase + 4 * LPG * v;
+                if (MODE != FWD_KEEP) WT::unpack(WT::load(W, e), w[v]);
+                if (MODE != FWD_FULL) cv[v] = *reinterpret_cast<const uint32_t*>(CODES + e);
+            }
+        }
+        const float dl = ok ? __ldg(DELTA + grp) : 1.f, za = ok ? __ldg(ZA + grp) : 0.f;
+        __syncwarp();                             // previous row is done with the tables
+        unit_levels<Q, NG>(t, (float*)nullptr, lane, ALPHA, ZB, row * Gr + u * NG, min(NG, Gr - u * NG));
+        if (MODE == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
+        else if (MODE == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+        float srt[L];
+        if (MODE == FWD_FULL) {
+#pragma unroll
+            for (int r = 0; r < L; ++r) srt[r] = t.srt[sub][r];
+        }
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            if (!(ok && v < nv)) continue;
+            const int64_t e = ebase + 4 * LPG * v;
+            float o[4];
+            uint32_t nc = 0;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                float m;
+                uint32_t code;
+                if (MODE == FWD_KEEP) {
+                    code = (cv[v] >> (8 * k)) & (L - 1);
+                    m = t.lv[sub][code];
+                } else {
+                    const float x = __fadd_rn(__fdiv_rn(__fmul_rn(w[v][k], s[v][k]), dl), za);
+                    if (MODE == FWD_REMAP) {
+                        const int c = (cv[v] >> (8 * k)) & (L - 1);
+                        const float4 nb = t.nb[sub][c];
+                        const uint32_t packed = __float_as_uint(nb.w);
+                        float best = fabsf(__fsub_rn(x, nb.y));
+                        m = nb.y;
+                        code = c;
+                        const float dlo = fabsf(__fsub_rn(x, nb.x));
+                        if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
+                        const float dhi = fabsf(__fsub_rn(x, nb.z));
+                        if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                    } else {
+                        const int r = nearest_rank<L>(x, srt, m);
+                        code = t.cor[sub][r];
+                    }
+                }
+                o[k] = __fdiv_rn(__fmul_rn(dl, __fsub_rn(m, za)), s[v][k]);
+                nc |= code << (8 * k);
+            }
+            if (MODE != FWD_KEEP) *reinterpret_cast<uint32_t*>(CODES + e) = nc;
+            *reinterpret_cast<float4*>(WHAT + e) = make_float4(o[0], o[1], o[2], o[3]);
+        }
+    }
+}
+
+template <int Q, typename WT, int LPG>
+__global__ void __launch_bounds__(kThreads, UQ_AWQ_BWD_MIN_BLOCKS)
+awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const float* __restrict__ DELTA,
+               const float* __restrict__ ZA, const float* __restrict__ ALPHA, const float* __restrict__ ZB,
+               const uint8_t* __restrict__ CODES, const float* __restrict__ GUP, float* __restrict__ DDELTA,
+               float* __restrict__ DZA, float* __restrict__ DALPHA, float* __restrict__ DZB,
+               float* __restrict__ PART, int64_t out, int n_in, int g, int64_t rows_per_range) {
+    constexpr int L = 1 << Q;
+    constexpr int NG = 32 / LPG;
+    using SR8 = SegReduce<LPG>;
+    __shared__ LvTab<Q, NG> tabs[kWarps];
+    __shared__ float tau_s[kWarps][NG];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    LvTab<Q, NG>& t = tabs[warp];
+    const int Gr = n_in / g;
+    const int u = blockIdx.x * kWarps + warp;
+    if (u * NG >= Gr) return;                     // no block barrier in this kernel
+    const int64_t r0 = (int64_t)blockIdx.y * rows_per_range;
+    const int64_t r1 = r0 + rows_per_range < out ? r0 + rows_per_range : out;
+    const int nv = g / (4 * LPG);
+    const int sub = lane / LPG, li = lane % LPG;
+    const int gi = u * NG + sub;
+    const bool ok = gi < Gr;
+    const int64_t cbase = (int64_t)gi * g + 4 * li;
+    float s[4][4], dsa[4][4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) dsa[v][k] = 0.f;
+        if (ok && v < nv) f4_to(ldg4(SA + cbase + 4 * LPG * v), s[v]);
+    }
+
+    for (int64_t row = r0; row < r1; ++row) {
+        const int64_t grp = row * Gr + gi;
+        const int64_t ebase = row * (int64_t)n_in + cbase;
+        float w[4][4], G[4][4];
+        uint32_t cv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            if (ok && v < nv) {
+                const int64_t e = ebase + 4 * LPG * v;
+                WT::unpack(WT::load(W, e), w[v]);
+                f4_to(ldg4(GUP + e), G[v]);
+                cv[v] = __ldg(reinterpret_cast<const unsigned int*>(CODES + e));
+            }
+        }
+        const float dl = ok ? __ldg(DELTA + grp) : 1.f, za = ok ? __ldg(ZA + grp) : 0.f;
+        __syncwarp();                             // previous row is done with the tables
+        unit_levels<Q, NG>(t, tau_s[warp], lane, ALPHA, ZB, row * Gr + u * NG, min(NG, Gr - u * NG));
+        const float tau = tau_s[warp][sub];
+        float acc[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            if (!(ok && v < nv)) continue;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int c = (cv[v] >> (8 * k)) & (L - 1);
+                const float m = t.lv[sub][c];
+                const float ws = __fmul_rn(w[v][k], s[v][k]);
+                const float uu = __fdiv_rn(ws, dl);
+                const float x = __fadd_rn(uu, za);
+                const bool f = fabsf(__fsub_rn(x, m)) <= tau;
+                const float gs = G[v][k] / s[v][k];
+                const float mz = m - za;
+                acc[0] += gs * (mz - (f ? uu : 0.f));
+                acc[1] += f ? 0.f : gs;
+                acc[2] += gs;
+#pragma unroll
+                for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? gs : -gs;
+                dsa[v][k] += gs * ((f ? w[v][k] : 0.f) - dl * mz / s[v][k]);
+            }
+        }
+        const int slot0 = SR8::run(acc, lane);
+        if (ok && SR8::writer(lane)) {
+#pragma unroll
+            for (int i = 0; i < SR8::NOUT; ++i) {
+                const int slot = slot0 + i;
+                const float tot = acc[i];
+                if (slot == 0) DDELTA[grp] = tot;
+                else if (slot == 1) DZA[grp] = -(dl * tot);
+                else if (slot == 2) DZB[grp] = dl * tot;
+                else if (slot >= 4 && slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * tot;
+            }
+        }
+    }
+    // this row range's ds_A partials of the unit's columns
+    float* prow = PART + (int64_t)blockIdx.y * n_in + cbase;
+#pragma unroll
+    for (int v = 0; v < 4; ++v)
+        if (ok && v < nv)
+            *reinterpret_cast<float4*>(prow + 4 * LPG * v) = make_float4(dsa[v][0], dsa[v][1], dsa[v][2], dsa[v][3]);
+}
+
+// ds_A[col] = sum over the row ranges of PART[range, col], in range order.
+__global__ void __launch_bounds__(256)
+awq_colsum_kernel(const float* __restrict__ PART, float* __restrict__ DSA, int n_in, int ranges) {
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < n_in; c += gridDim.x * blockDim.x) {
+        float acc = 0.f;
+        for (int r = 0; r < ranges; ++r) acc += __ldg(PART + (int64_t)r * n_in + c);
+        DSA[c] = acc;
+    }
+}
+
+bool awq_ok(const Shape& sh) { return sh.g == 32 || sh.g == 64 || sh.g == 128 || sh.g == 256 || sh.g == 512; }
+
+// Row ranges: enough blocks (column stripes x ranges) for about
+// kAwqTargetBlocksPerSm blocks per SM, at least one row per range.
+static void awq_grid(const Shape& sh, int lpg, unsigned& col_blocks, int64_t& ranges, int64_t& rows_per_range) {
+    const int NG = 32 / lpg;
+    const int units = (sh.n_in / sh.g + NG - 1) / NG;
+    col_blocks = (unsigned)((units + kWarps - 1) / kWarps);
+    int64_t want = ((int64_t)sm_count() * kAwqTargetBlocksPerSm + col_blocks - 1) / col_blocks;
+    if (want > sh.out) want = sh.out;
+    if (want < 1) want = 1;
+    rows_per_range = (sh.out + want - 1) / want;
+    ranges = (sh.out + rows_per_range - 1) / rows_per_range;
+}
+
+int64_t awq_workspace_floats(const Shape& sh) {
+    unsigned cb;
+    int64_t ranges, rpr;
+    awq_grid(sh, lanes_per_group(sh.g), cb, ranges, rpr);
+    return ranges * (int64_t)sh.n_in;
+}
+
+template <int Q, typename WT, int LPG>
+static cudaError_t awq_lpg(bool bwd, int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                           float* what, const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    unsigned cb;
+    int64_t ranges, rpr;
+    awq_grid(sh, LPG, cb, ranges, rpr);
+    const dim3 grid(cb, (unsigned)ranges);
+    if (bwd) {
+        awq_bwd_kernel<Q, WT, LPG><<<grid, kThreads, 0, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes, gup,
+                                                             gr.ddelta, gr.dza, gr.dalpha, gr.dzb, work, sh.out,
+                                                             sh.n_in, sh.g, rpr);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        int blocks = (sh.n_in + 255) / 256;
+        awq_colsum_kernel<<<blocks, 256, 0, st>>>(work, gr.dsa, sh.n_in, (int)ranges);
+        return cudaGetLastError();
+    }
+    if (mode == FWD_KEEP)
+        awq_fwd_kernel<Q, WT, LPG, FWD_KEEP><<<grid, kThreads, 0, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes,
+                                                                        what, sh.out, sh.n_in, sh.g, rpr);
+    else if (mode == FWD_REMAP)
+        awq_fwd_kernel<Q, WT, LPG, FWD_REMAP><<<grid, kThreads, 0, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes,
+                                                                         what, sh.out, sh.n_in, sh.g, rpr);
+    else
+        awq_fwd_kernel<Q, WT, LPG, FWD_FULL><<<grid, kThreads, 0, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes,
+                                                                        what, sh.out, sh.n_in, sh.g, rpr);
+    return cudaGetLastError();
+}
+
+template <int Q, typename WT>
+static cudaError_t awq_g(bool bwd, int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                         float* what, const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    switch (lanes_per_group(sh.g)) {
+        case 4: return awq_lpg<Q, WT, 4>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        case 8: return awq_lpg<Q, WT, 8>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        case 16: return awq_lpg<Q, WT, 16>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        default: return awq_lpg<Q, WT, 32>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+    }
+}
+
+template <int Q>
+static cudaError_t awq_w(bool bwd, int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                         float* what, const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    if (sh.wdtype == UQ_W_BF16) return awq_g<Q, WBF16>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+    return awq_g<Q, WF32>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+}
+
+static cudaError_t awq_dispatch(bool bwd, int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                                float* what, const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    switch (sh.q) {
+        case 1: return awq_w<1>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        case 2: return awq_w<2>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        case 3: return awq_w<3>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+        default: return awq_w<4>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
+    }
+}
+
+cudaError_t launch_awq_fwd(const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes, int mode, float* what,
+                           cudaStream_t st) {
+    return awq_dispatch(false, mode, sh, W, p, codes, what, nullptr, uq_grads_awq{}, nullptr, st);
+}
+
+cudaError_t launch_awq_bwd(const Shape& sh, const void* W, uq_params_awq p, const uint8_t* codes, const float* gup,
+                           uq_grads_awq gr, float* work, cudaStream_t st) {
+    return awq_dispatch(true, 0, sh, W, p, const_cast<uint8_t*>(codes), nullptr, gup, gr, work, st);
+}
+
+}  // namespace uq

@@ -59,6 +59,14 @@ cudaError_t launch_omni_bwd(const Shape& sh, const void* W, uq_params_omni p, co
                             uq_grads_omni gr, cudaStream_t st);
 cudaError_t launch_omni_scales(const Shape& sh, const void* W, const float* beta, const float* gamma, float* delta,
                                float* zo, cudaStream_t st);
+// UniQuan with AWQ's maps (uq_awq.cu); awq_ok: the group sizes it takes;
+// awq_workspace_floats: floats of per-row-range ds_A partials the backward needs.
+bool awq_ok(const Shape& sh);
+int64_t awq_workspace_floats(const Shape& sh);
+cudaError_t launch_awq_fwd(const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes, int mode, float* what,
+                           cudaStream_t st);
+cudaError_t launch_awq_bwd(const Shape& sh, const void* W, uq_params_awq p, const uint8_t* codes, const float* gup,
+                           uq_grads_awq gr, float* work, cudaStream_t st);
 // Launches the bounded-wait self-test (one warp, a wait that runs out).
 cudaError_t launch_wait_selftest(cudaStream_t st);
 // Streaming multiprocessors of the current device (cached per device).

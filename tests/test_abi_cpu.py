@@ -223,6 +223,30 @@ def test_omni_validation(libpath):
     assert L.uq_omni_scales(FAKE, 1, 8, 768, 3, 96, FAKE, FAKE, FAKE, FAKE, None) == api.UQ_ERR_UNSUPPORTED
 
 
+@cpu_only
+def test_awq_validation(libpath):
+    from paper_2506_03781_gb300 import api
+    L = api.lib()
+    P = lambda **o: api.uq_params_awq(**{**{n: FAKE + 0x1000 * i for i, n in enumerate(api.AWQ_PARAM_NAMES)}, **o})
+    Gd = lambda **o: api.uq_grads_awq(**{**{n: FAKE + 0x10000 + 0x1000 * i for i, n in enumerate(api.AWQ_GRAD_NAMES)},
+                                        **o})
+    fwd = lambda g=128, n_in=512, p=None, W=FAKE, step=0: L.uq_quantize_fwd_awq(
+        W, 1, 8, n_in, 3, g, p or P(), FAKE + 0x9000, 1, step, 2, FAKE + 0xA000, None)
+    assert fwd(g=1024, n_in=2048) == api.UQ_ERR_UNSUPPORTED
+    assert fwd(W=0) == api.UQ_ERR_ARG
+    assert fwd(W=0, step=1) == api.UQ_ERR_CUDA                        # keep step: W is not read
+    assert fwd(p=P(sa=0)) == api.UQ_ERR_ARG
+    assert fwd(p=P(za=FAKE + 4)) == api.UQ_ERR_ALIGN
+    bwd = lambda gr=None, ws=FAKE + 0x20000, nb=1 << 30: L.uq_quantize_bwd_awq(
+        FAKE, 1, 8, 512, 3, 128, P(), FAKE + 0x9000, FAKE + 0xB000, gr or Gd(), ws, nb, None)
+    for f in api.AWQ_GRAD_NAMES:
+        assert bwd(Gd(**{f: 0})) == api.UQ_ERR_ARG and f in api.uq_last_error()
+    assert bwd(ws=0) == api.UQ_ERR_ARG
+    assert bwd(nb=0) == api.UQ_ERR_ARG and "workspace" in api.uq_last_error()
+    assert api.uq_awq_bwd_workspace_bytes(8, 512, 3, 96) == -1
+    assert api.uq_awq_bwd_workspace_bytes(8, 512, 3, 128) >= 8 * 4
+
+
 def test_binding_rejects_host_tensors_before_calling(libpath):
     import torch
     from paper_2506_03781_gb300 import api
