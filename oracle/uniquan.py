@@ -36,7 +36,7 @@ import itertools
 import numpy as np
 
 __all__ = [
-    "MAP_FULL", "MAP_LOCAL_PERIODIC",
+    "MAP_FULL", "MAP_LOCAL_PERIODIC", "FILTER_STE", "FILTER_ELEMENT",
     "EXPORT_REUSE_CODES", "EXPORT_REMAP_EQ4",
     "CLIP_FIXED_MIN", "CLIP_FIXED_MAX", "CLIP_BALANCED",
     "signs", "levels", "sorted_levels",
@@ -45,7 +45,7 @@ __all__ = [
     "LR_F", "LR_B", "sgd_update", "train_step",
     "omni_params", "quantize_fwd_omni", "quantize_bwd_omni", "bwd_l1_mass_omni", "export_bcq_omni",
     "quantize_fwd_awq", "quantize_bwd_awq", "bwd_l1_mass_awq", "export_bcq_awq",
-    "unify", "codes_eq4", "pack_bitplanes", "export_bcq",
+    "unify", "codes_eq4", "pack_bitplanes", "export_bcq", "export_bcq_half",
     "bcq_dequantize", "bcq_gemv",
     "clip_params", "greedy_init", "general_alternating", "unified_init",
     "rtn",
@@ -56,6 +56,8 @@ F64 = np.float64
 
 MAP_FULL = 0
 MAP_LOCAL_PERIODIC = 1
+FILTER_STE = 0
+FILTER_ELEMENT = 1
 EXPORT_REUSE_CODES = 0
 EXPORT_REMAP_EQ4 = 1
 CLIP_FIXED_MIN = 0
@@ -206,7 +208,7 @@ def quantize_fwd(W, s, sr, delta, zu, alpha, zb, codes, g, mode=MAP_LOCAL_PERIOD
 # Backward: straight-through estimator with gradient filtering (App. C.1)
 # ---------------------------------------------------------------------------
 
-def _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+def _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, filter_mode=FILTER_STE):
     out, n_in = np.shape(W)
     q = np.shape(alpha)[-1]
     Wg = _grouped(np.asarray(W, F32), out, g)
@@ -227,12 +229,14 @@ def _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
     C = signs(q, F64)[cg]                                   # [out, Gr, g, q]
     m64 = (C * np.asarray(alpha, F64)[..., None, :]).sum(-1) + np.asarray(zb, F64)[..., None]
     G64 = _grouped(np.asarray(Gup, F64), out, g)
+    if filter_mode == FILTER_ELEMENT:
+        G64 = np.where(f, G64, 0.0)                         # a filtered element drops out entirely
     gbar = G64 * d64                                        # dL/dw~ = G * Delta
     fu = np.where(f, u64, 0.0)
     return dict(f=f, u=u64, m=m64, zu=zu64, s=s64, sr=sr64, G=G64, gbar=gbar, fu=fu, C=C)
 
 
-def quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+def quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, filter_mode=FILTER_STE):
     """Gradients of L w.r.t. Theta_IF given G = dL/dW^ (App. C.1, Eq. 3).
 
     Differentiates w^ = Delta * (w~ - z_U) with
@@ -249,9 +253,14 @@ def quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
       ds_r    = -sum_{i in row} G_i Delta f_i u_i / s_r
     Filter decisions in fp32, values and sums in fp64.  Returns a dict of
     fp64 arrays shaped like the parameters.
+
+    filter_mode FILTER_STE is the reading above (the filter cuts only the
+    straight-through path); FILTER_ELEMENT is the alternative reading in
+    which a filtered element drops out of every gradient: G_i is replaced by
+    f_i G_i in all the sums (so dz_U is identically zero).
     """
     out, n_in = np.shape(W)
-    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g)
+    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, filter_mode)
     gbar, fu = t["gbar"], t["fu"]
     return dict(
         ds=(-gbar * fu / t["s"]).reshape(out, n_in),
@@ -263,14 +272,14 @@ def quantize_bwd(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
     )
 
 
-def bwd_l1_mass(W, s, sr, delta, zu, alpha, zb, codes, Gup, g):
+def bwd_l1_mass(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, filter_mode=FILTER_STE):
     """L1 mass sum_i |term_i| of every reduction in quantize_bwd (fp64).
 
     A summation of n terms in any order cannot be trusted beyond a multiple
     of (unit roundoff) x (sum of |terms|); the parity tests scale their
     tolerance by this mass.  ds gets its own per-element values back.
     """
-    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g)
+    t = _bwd_terms(W, s, sr, delta, zu, alpha, zb, codes, Gup, g, filter_mode)
     gbar, fu = t["gbar"], t["fu"]
     q = np.shape(alpha)[-1]
     mass_gbar = np.abs(gbar).sum(-1)
@@ -590,6 +599,15 @@ def pack_bitplanes(codes, q):
     bits = bits.reshape(q, out, n_in // 32, 32)
     weights = (np.uint64(1) << np.arange(32, dtype=np.uint64))
     return (bits.astype(np.uint64) * weights).sum(-1).astype(np.uint32)
+
+
+def export_bcq_half(W, delta, zu, alpha, zb, codes, g, mode=EXPORT_REUSE_CODES):
+    """export_bcq with alpha* and z_B* stored as 16-bit reals (App. F.1 counts
+    16 bits per real of Theta_B*): the fp32 values of export_bcq rounded to
+    IEEE half precision, nearest even.  Returns (planes, alpha* bits uint16,
+    z_B* bits uint16, codes used)."""
+    planes, a_s, z_s, c = export_bcq(W, delta, zu, alpha, zb, codes, g, mode)
+    return planes, a_s.astype(np.float16).view(np.uint16), z_s.astype(np.float16).view(np.uint16), c
 
 
 def export_bcq(W, delta, zu, alpha, zb, codes, g, mode=EXPORT_REUSE_CODES):

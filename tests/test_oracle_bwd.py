@@ -147,3 +147,46 @@ def test_l1_mass_bounds_sums():
                        pb["codes"], pb["Gup"], pb["g"])
     for k in ("ddelta", "dzu", "dzb", "dalpha", "dsr"):
         assert np.all(np.abs(gr[k]) <= ms[k] * (1 + 1e-12) + 1e-300), k
+
+
+@pytest.mark.parametrize("q", [1, 2, 3])
+def test_element_filter_matches_finite_differences_of_the_masked_surrogate(q):
+    """The whole-element filter: a filtered element contributes nothing, i.e.
+    the gradient of sum over the UNfiltered elements of G w^ (filtered ones
+    frozen)."""
+    pb = make_problem(100 + q, q)
+    P, x0, f, margin = frozen_state(pb, q)
+    assert margin.min() > 1e-4 and 0 < f.mean() < 1
+    grads = O.quantize_bwd(pb["W"], pb["s"], pb["sr"], pb["delta"], pb["zu"], pb["alpha"], pb["zb"],
+                           pb["codes"], pb["Gup"], pb["g"], filter_mode=O.FILTER_ELEMENT)
+    masked = dict(pb)
+    masked["Gup"] = np.where(f.reshape(pb["Gup"].shape) > 0, pb["Gup"], 0).astype(F32)
+    name_of = {"delta": "ddelta", "zu": "dzu", "zb": "dzb", "alpha": "dalpha", "s": "ds", "sr": "dsr"}
+    rng = np.random.default_rng(17)
+    for k in ("delta", "zu", "zb", "alpha", "s", "sr"):
+        for _ in range(3):
+            idx = tuple(rng.integers(n) for n in P[k].shape)
+            h = 1e-6 * max(1.0, abs(P[k][idx]))
+            Pp = {kk: vv.copy() for kk, vv in P.items()}
+            Pm = {kk: vv.copy() for kk, vv in P.items()}
+            Pp[k][idx] += h
+            Pm[k][idx] -= h
+            args = (x0, pb["codes"], pb["W"], masked["Gup"], pb["g"], q)
+            fd = (surrogate(Pp, f, *args) - surrogate(Pm, f, *args)) / (2 * h)
+            got = grads[name_of[k]][idx]
+            assert abs(got - fd) <= 1e-5 * max(abs(fd), 1e-7), (k, idx, got, fd)
+    assert np.all(grads["dzu"] == 0.0)
+
+
+def test_half_export_rounds_to_nearest_even():
+    """The 16-bit export equals IEEE half rounding of the fp32 export, checked
+    with Python's own half-precision packing ('e', round half to even)."""
+    import struct
+    pb = make_problem(600, 3, out=4, n_in=256, g=64)
+    planes, a32, z32, _ = O.export_bcq(pb["W"], pb["delta"], pb["zu"], pb["alpha"], pb["zb"], pb["codes"], pb["g"])
+    planes_h, a16, z16, _ = O.export_bcq_half(pb["W"], pb["delta"], pb["zu"], pb["alpha"], pb["zb"], pb["codes"],
+                                              pb["g"])
+    assert np.array_equal(planes, planes_h)
+    for v32, v16 in ((a32, a16), (z32, z16)):
+        for a, b in zip(v32.ravel(), v16.ravel()):
+            assert struct.unpack("<H", struct.pack("<e", float(a)))[0] == int(b)
