@@ -407,6 +407,64 @@ def time_block_step(dev, steps=20, warmup=3, samples=4):
     return res
 
 
+def time_variants(dev, stream, peak, q=3, g=128, out=14336, n_in=4096, reps=20):
+    """CUDA-event times of the OmniQuant- and AWQ-unified quantizer kernels
+    (forward remap and keep steps, backward) on a matrix of the headline
+    shape with random parameters and inputs (every call moves far more than
+    the L2 holds)."""
+    import torch
+    from paper_2506_03781_gb300 import api, roofline
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(99)
+    Wd = (torch.randn(out, n_in, generator=gen, device=dev) * 0.02).to(torch.bfloat16)
+    Gr = n_in // g
+    codes = torch.randint(0, 1 << q, (out, n_in), generator=gen, device=dev, dtype=torch.uint8)
+    what = torch.empty(out, n_in, device=dev)
+    Gup = torch.randn(out, n_in, generator=gen, device=dev) * 0.01
+    lv = torch.tensor([2.0 ** (q - 2 - j) for j in range(q)], device=dev)
+    alpha = (lv * (1 + 0.05 * torch.randn(out, Gr, q, generator=gen, device=dev))).contiguous()
+    zb = ((1 << q) - 1) / 2 + 0.1 * torch.randn(out, Gr, generator=gen, device=dev)
+    omni = {"beta": 0.9 + 0.1 * torch.rand(out, Gr, generator=gen, device=dev),
+            "gamma": 0.9 + 0.1 * torch.rand(out, Gr, generator=gen, device=dev), "alpha": alpha, "zb": zb}
+    og = {"dbeta": torch.empty(out, Gr, device=dev), "dgamma": torch.empty(out, Gr, device=dev),
+          "dalpha": torch.empty(out, Gr, q, device=dev), "dzb": torch.empty(out, Gr, device=dev)}
+    awq = {"sa": 0.5 + torch.rand(n_in, generator=gen, device=dev), "delta": torch.full((out, Gr), 0.01, device=dev),
+           "za": torch.full((out, Gr), 3.5, device=dev), "alpha": alpha, "zb": zb}
+    ag = {"dsa": torch.empty(n_in, device=dev), "ddelta": torch.empty(out, Gr, device=dev),
+          "dza": torch.empty(out, Gr, device=dev), "dalpha": torch.empty(out, Gr, q, device=dev),
+          "dzb": torch.empty(out, Gr, device=dev)}
+    ws = torch.empty(max(api.uq_awq_bwd_workspace_bytes(out, n_in, q, g) // 4, 4), device=dev)
+    calls = {
+        "omni_fwd_remap": lambda: api.uq_quantize_fwd_omni(Wd, q, g, omni, codes, what, api.MAP_LOCAL_PERIODIC, 0, 2,
+                                                            stream=stream),
+        "omni_fwd_keep": lambda: api.uq_quantize_fwd_omni(Wd, q, g, omni, codes, what, api.MAP_LOCAL_PERIODIC, 1, 2,
+                                                           stream=stream),
+        "omni_bwd": lambda: api.uq_quantize_bwd_omni(Wd, q, g, omni, codes, Gup, og, stream=stream),
+        "awq_fwd_remap": lambda: api.uq_quantize_fwd_awq(Wd, q, g, awq, codes, what, api.MAP_LOCAL_PERIODIC, 0, 2,
+                                                          stream=stream),
+        "awq_fwd_keep": lambda: api.uq_quantize_fwd_awq(Wd, q, g, awq, codes, what, api.MAP_LOCAL_PERIODIC, 1, 2,
+                                                         stream=stream),
+        "awq_bwd": lambda: api.uq_quantize_bwd_awq(Wd, q, g, awq, codes, Gup, ag, workspace=ws, stream=stream),
+    }
+    res = {}
+    for name, fn in calls.items():
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        nbytes = roofline.bytes_per_launch(name, out, n_in, q, g, 2)
+        res[name] = {"avg_ms": ms, "gbs": nbytes / ms / 1e6, "frac": nbytes / ms / 1e6 / peak}
+    del Wd, codes, what, Gup, ws
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_gpu(args):
     import torch
     from paper_2506_03781_gb300 import api, roofline, synth
@@ -532,6 +590,9 @@ def run_gpu(args):
     # deployment: the BCQ product from the exported format (one bf16 token)
     gemv = time_gemv(q, g, dev, stream, peak)
 
+    # UniQuan with OmniQuant's and AWQ's maps (App. E) on the same shape
+    variants = time_variants(dev, stream, peak, q, g, out, n_in)
+
     # Algorithm 1 on a Llama-3-8B-shaped block (the quantizer inside the loop)
     block = None if args.no_block else time_block_step(dev)
 
@@ -621,6 +682,7 @@ def run_gpu(args):
             "train_step": train,
             "bcq_gemv": gemv,
             "block_step": block,
+            "unified_variants": variants,
             "q_sweep": sweep,
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,

@@ -83,6 +83,11 @@ typedef enum { UQ_MAP_FULL = 0, UQ_MAP_LOCAL_PERIODIC = 1 } uq_map;
  * from the original weights by Eq. 4. */
 typedef enum { UQ_EXPORT_REUSE_CODES = 0, UQ_EXPORT_REMAP_EQ4 = 1 } uq_export_mode;
 
+/* Gradient filter (App. C.1): cut only the straight-through path of a
+ * filtered element (the library's reading, used by uq_quantize_bwd), or drop
+ * the filtered element from every gradient (the alternative reading). */
+typedef enum { UQ_FILTER_STE = 0, UQ_FILTER_ELEMENT = 1 } uq_filter;
+
 /* The learnable parameters Theta_IF = Theta_F u Theta_B (Eq. 1, Sec. 2.3). */
 typedef struct {
     float* delta;   /* [out, in/g]    Delta                                */
@@ -206,6 +211,17 @@ uq_status uq_quantize_fwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
 uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
                           uq_params params, const uint8_t* codes, const float* dL_dWhat,
                           uq_grads grads, void* stream);
+
+/*
+ * uq_quantize_bwd_ex -- uq_quantize_bwd with a choice of gradient filter:
+ * UQ_FILTER_STE is exactly uq_quantize_bwd; with UQ_FILTER_ELEMENT every
+ * term of an element with |x - l(c)| > tau is dropped (G_i replaced by
+ * f_i G_i in every sum, so dz_U is zero).  Same arguments, layouts and
+ * numerics otherwise; an unknown filter is UQ_ERR_ARG.
+ */
+uq_status uq_quantize_bwd_ex(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                             uq_params params, const uint8_t* codes, const float* dL_dWhat, uq_grads grads,
+                             uq_filter filter, void* stream);
 
 /*
  * uq_train_step -- one optimisation step of Algorithm 1's inner loop, fused
@@ -334,6 +350,18 @@ int64_t uq_awq_bwd_workspace_bytes(int64_t out, int64_t in, int q, int g);
 uq_status uq_export_bcq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
                         uq_params params, const uint8_t* codes, uq_export_mode mode,
                         uint32_t* bitplanes, float* alpha_star, float* zb_star, void* stream);
+
+/*
+ * uq_export_bcq_half -- uq_export_bcq with alpha* and z_B* stored as 16-bit
+ * reals (the storage App. F.1 counts: g k + 16 (k + 1) bits per group): the
+ * fp32 values uq_export_bcq computes, rounded to IEEE half precision (nearest
+ * even; overflow to infinity), written as raw half bits to alpha_star
+ * [out, in/g, q] and zb_star [out, in/g] (uint16).  Bit-planes as
+ * uq_export_bcq.
+ */
+uq_status uq_export_bcq_half(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                             uq_params params, const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes,
+                             uint16_t* alpha_star, uint16_t* zb_star, void* stream);
 
 /*
  * uq_bcq_gemv -- the BCQ matrix-vector product of deployment, computed from

@@ -26,6 +26,7 @@ CLIP_FIXED_MIN, CLIP_FIXED_MAX, CLIP_BALANCED = 0, 1, 2
 MAP_FULL, MAP_LOCAL_PERIODIC = 0, 1
 LR_THETA_F, LR_THETA_B = 0.005, 0.0005     # learning rates of the hyperparameter table (App. C.1)
 EXPORT_REUSE_CODES, EXPORT_REMAP_EQ4 = 0, 1
+FILTER_STE, FILTER_ELEMENT = 0, 1
 
 PARAM_NAMES = ("delta", "zu", "s", "sr", "alpha", "zb")
 OMNI_PARAM_NAMES = ("beta", "gamma", "alpha", "zb")
@@ -34,6 +35,7 @@ AWQ_PARAM_NAMES = ("sa", "delta", "za", "alpha", "zb")
 AWQ_GRAD_NAMES = ("dsa", "ddelta", "dza", "dalpha", "dzb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
 ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
+                "uq_quantize_bwd_ex", "uq_export_bcq_half",
                 "uq_quantize_fwd_omni", "uq_quantize_bwd_omni", "uq_omni_scales",
                 "uq_quantize_fwd_awq", "uq_quantize_bwd_awq", "uq_awq_bwd_workspace_bytes", "uq_bcq_gemv",
                 "uq_bcq_gemv_workspace_bytes", "uq_bcq_gemv_noalloc",
@@ -88,6 +90,8 @@ def lib() -> ctypes.CDLL:
         L.uq_quantize_fwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, vp]
         L.uq_export_bcq.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
+        L.uq_quantize_bwd_ex.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, uq_grads, i32, vp]
+        L.uq_export_bcq_half.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, i32, vp, vp, vp, vp]
         L.uq_quantize_fwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, i32, i64, i32, vp, vp]
         L.uq_quantize_bwd_omni.argtypes = [vp, i32, i64, i64, i32, i32, uq_params_omni, vp, vp, uq_grads_omni, vp]
         L.uq_omni_scales.argtypes = [vp, i32, i64, i64, i32, i32, vp, vp, vp, vp, vp]
@@ -261,6 +265,40 @@ def uq_train_step(W, q, g, params, codes, dL_dWhat, W_hat, step, lr_F=LR_THETA_F
         _check(codes, "codes", (out, n_in), torch.uint8, dev),
         _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), float(lr_F), float(lr_B), map_mode, step,
         p_period, _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_quantize_bwd_ex(W, q, g, params, codes, dL_dWhat, grads, filter=FILTER_STE, stream=None):
+    """uq_quantize_bwd with a choice of gradient filter (FILTER_STE or FILTER_ELEMENT)."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    shapes = {"ddelta": (out, Gr), "dzu": (out, Gr), "ds": (out, n_in), "dsr": (out,),
+              "dalpha": (out, Gr, q), "dzb": (out, Gr)}
+    gp = uq_grads(**{n: _check(grads[n], f"grads['{n}']", shapes[n], torch.float32, dev) for n in GRAD_NAMES})
+    st = lib().uq_quantize_bwd_ex(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), gp, filter, _stream(stream, dev))
+    _raise(st)
+
+
+def uq_export_bcq_half(W, q, g, params, codes, bitplanes, alpha_star, zb_star, mode=EXPORT_REUSE_CODES,
+                       stream=None, shape=None, wdtype=None):
+    """uq_export_bcq with alpha*, z_B* as IEEE half: ``alpha_star``, ``zb_star`` are torch.float16 tensors."""
+    if W is not None:
+        out, n_in = _dims(W, g)
+        wd, dev, wptr = _wdtype(W), W.device, W.data_ptr()
+    else:
+        out, n_in = shape if shape is not None else codes.shape
+        wd, dev, wptr = (W_BF16 if wdtype is None else wdtype), codes.device, None
+    Gr = n_in // g if g > 0 and n_in % g == 0 else 0
+    cptr = _check(codes, "codes", (out, n_in), torch.uint8, dev) if codes is not None else None
+    st = lib().uq_export_bcq_half(
+        wptr, wd, out, n_in, q, g, _params(params, out, n_in, q, g, dev, ("delta", "zu", "alpha", "zb")),
+        cptr, mode, _check(bitplanes, "bitplanes", (q, out, n_in // 32), torch.int32, dev),
+        _check(alpha_star, "alpha_star", (out, Gr, q), torch.float16, dev),
+        _check(zb_star, "zb_star", (out, Gr), torch.float16, dev), _stream(stream, dev))
     _raise(st)
 
 

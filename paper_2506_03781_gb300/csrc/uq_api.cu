@@ -132,6 +132,53 @@ uq_status uq_quantize_bwd(const void* W, uq_wdtype wdtype, int64_t out, int64_t 
     return cuda_status(uq::launch_bwd(sh, W, p, codes, dL_dWhat, gr, (cudaStream_t)stream), "uq_quantize_bwd");
 }
 
+uq_status uq_quantize_bwd_ex(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                             const uint8_t* codes, const float* dL_dWhat, uq_grads gr, uq_filter filter,
+                             void* stream) {
+    if (filter != UQ_FILTER_STE && filter != UQ_FILTER_ELEMENT)
+        return fail(UQ_ERR_ARG, "unknown gradient filter %d", (int)filter);
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.s, "params.s"));
+    UQ_TRY(check_ptr(p.sr, "params.sr"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(gr.ddelta, "grads.ddelta"));
+    UQ_TRY(check_ptr(gr.dzu, "grads.dzu"));
+    UQ_TRY(check_ptr(gr.ds, "grads.ds"));
+    UQ_TRY(check_ptr(gr.dsr, "grads.dsr"));
+    UQ_TRY(check_ptr(gr.dalpha, "grads.dalpha"));
+    UQ_TRY(check_ptr(gr.dzb, "grads.dzb"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_bwd(sh, W, p, codes, dL_dWhat, gr, (cudaStream_t)stream, (int)filter),
+                       "uq_quantize_bwd_ex");
+}
+
+uq_status uq_export_bcq_half(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                             const uint8_t* codes, uq_export_mode mode, uint32_t* bitplanes, uint16_t* alpha_star,
+                             uint16_t* zb_star, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (mode != UQ_EXPORT_REUSE_CODES && mode != UQ_EXPORT_REMAP_EQ4)
+        return fail(UQ_ERR_ARG, "unknown export mode %d", (int)mode);
+    if (mode == UQ_EXPORT_REMAP_EQ4) UQ_TRY(check_ptr(W, "W"));
+    else UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(bitplanes, "bitplanes"));
+    UQ_TRY(check_ptr(alpha_star, "alpha_star"));
+    UQ_TRY(check_ptr(zb_star, "zb_star"));
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    return cuda_status(uq::launch_export_half(sh, W, p, codes, (int)mode, bitplanes, alpha_star, zb_star,
+                                              (cudaStream_t)stream),
+                       "uq_export_bcq_half");
+}
+
 uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
                         uint8_t* codes, const float* dL_dWhat, float lr_F, float lr_B, uq_map map, int64_t step,
                         int p_period, float* W_hat, void* stream) {

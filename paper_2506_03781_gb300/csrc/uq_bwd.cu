@@ -24,7 +24,9 @@ namespace uq {
 #define UQ_BWD_MIN_BLOCKS 3
 #endif
 
-template <int Q, typename WT, int LPG>
+// ELEM: the whole-element filter (a filtered element drops out of every
+// gradient); otherwise the filter cuts the straight-through path only.
+template <int Q, typename WT, int LPG, bool ELEM>
 __global__ void __launch_bounds__(kThreads, UQ_BWD_MIN_BLOCKS)
 bwd_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
            const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
@@ -100,14 +102,15 @@ bwd_kernel(const void* __restrict__ W, const float* __restrict__ S, const float*
                         const float x = transform_x(w[k], s[k], dl, sr, zu, uu);
                         const bool f = fabsf(__fsub_rn(x, m)) <= tau;
                         const float fu = f ? uu : 0.f;
-                        const float gfu = G[k] * fu;
+                        const float gk = (ELEM && !f) ? 0.f : G[k];
+                        const float gfu = gk * fu;
                         ds[k] = -__fdividef(dl * gfu, s[k]);
-                        acc[0] += G[k] * ((m - zu) - fu);
-                        acc[1] += f ? 0.f : G[k];
-                        acc[2] += G[k];
+                        acc[0] += gk * ((m - zu) - fu);
+                        acc[1] += f ? 0.f : gk;
+                        acc[2] += gk;
                         acc[3] += gfu;
 #pragma unroll
-                        for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? G[k] : -G[k];
+                        for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? gk : -gk;
                     }
                     *reinterpret_cast<float4*>(DS + ebase + 4 * LPG * (c0 + v)) = make_float4(ds[0], ds[1], ds[2], ds[3]);
                 }
@@ -142,45 +145,49 @@ bwd_kernel(const void* __restrict__ W, const float* __restrict__ S, const float*
     }
 }
 
-template <int Q, typename WT, int LPG>
+template <int Q, typename WT, int LPG, bool ELEM>
 static cudaError_t run_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
                            uq_grads gr, cudaStream_t st) {
     constexpr int NG = 32 / LPG;
     const int Gr = sh.n_in / sh.g;
     const int R = rows_per_block((Gr + NG - 1) / NG);
     const int64_t blocks = (sh.out + R - 1) / R;
-    bwd_kernel<Q, WT, LPG><<<dim3((unsigned)blocks), kThreads, 0, st>>>(
+    bwd_kernel<Q, WT, LPG, ELEM><<<dim3((unsigned)blocks), kThreads, 0, st>>>(
         W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr, gr.ddelta, gr.dzu, gr.dzb, gr.dalpha,
         sh.out, sh.n_in, sh.g, R);
     return cudaGetLastError();
 }
 
-template <int Q, typename WT>
-static cudaError_t bwd_g(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
-                         uq_grads gr, cudaStream_t st) {
+template <int Q, typename WT, bool ELEM>
+static cudaError_t bwd_gf(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
+                          uq_grads gr, cudaStream_t st) {
     switch (lanes_per_group(sh.g)) {
-        case 4: return run_bwd<Q, WT, 4>(sh, W, p, codes, gup, gr, st);
-        case 8: return run_bwd<Q, WT, 8>(sh, W, p, codes, gup, gr, st);
-        case 16: return run_bwd<Q, WT, 16>(sh, W, p, codes, gup, gr, st);
-        default: return run_bwd<Q, WT, 32>(sh, W, p, codes, gup, gr, st);
+        case 4: return run_bwd<Q, WT, 4, ELEM>(sh, W, p, codes, gup, gr, st);
+        case 8: return run_bwd<Q, WT, 8, ELEM>(sh, W, p, codes, gup, gr, st);
+        case 16: return run_bwd<Q, WT, 16, ELEM>(sh, W, p, codes, gup, gr, st);
+        default: return run_bwd<Q, WT, 32, ELEM>(sh, W, p, codes, gup, gr, st);
     }
 }
 
 template <int Q>
 static cudaError_t bwd_w(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
-                         uq_grads gr, cudaStream_t st) {
-    if (sh.wdtype == UQ_W_BF16) return bwd_g<Q, WBF16>(sh, W, p, codes, gup, gr, st);
-    return bwd_g<Q, WF32>(sh, W, p, codes, gup, gr, st);
+                         uq_grads gr, int filter, cudaStream_t st) {
+    const bool elem = filter == UQ_FILTER_ELEMENT;
+    if (sh.wdtype == UQ_W_BF16)
+        return elem ? bwd_gf<Q, WBF16, true>(sh, W, p, codes, gup, gr, st)
+                    : bwd_gf<Q, WBF16, false>(sh, W, p, codes, gup, gr, st);
+    return elem ? bwd_gf<Q, WF32, true>(sh, W, p, codes, gup, gr, st)
+                : bwd_gf<Q, WF32, false>(sh, W, p, codes, gup, gr, st);
 }
 
 cudaError_t launch_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
-                       uq_grads gr, cudaStream_t st) {
-    if (stream_path_ok(sh)) return launch_bwd_stream(sh, W, p, codes, gup, gr, st);
+                       uq_grads gr, cudaStream_t st, int filter) {
+    if (stream_path_ok(sh)) return launch_bwd_stream(sh, W, p, codes, gup, gr, st, filter);
     switch (sh.q) {
-        case 1: return bwd_w<1>(sh, W, p, codes, gup, gr, st);
-        case 2: return bwd_w<2>(sh, W, p, codes, gup, gr, st);
-        case 3: return bwd_w<3>(sh, W, p, codes, gup, gr, st);
-        default: return bwd_w<4>(sh, W, p, codes, gup, gr, st);
+        case 1: return bwd_w<1>(sh, W, p, codes, gup, gr, filter, st);
+        case 2: return bwd_w<2>(sh, W, p, codes, gup, gr, filter, st);
+        case 3: return bwd_w<3>(sh, W, p, codes, gup, gr, filter, st);
+        default: return bwd_w<4>(sh, W, p, codes, gup, gr, filter, st);
     }
 }
 

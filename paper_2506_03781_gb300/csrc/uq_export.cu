@@ -10,21 +10,34 @@
 // holds the four bits in order.  Consecutive threads write consecutive
 // words.  HBM traffic per element: 1 (codes) or 2-4 (weights) read, q/8
 // written, plus the group parameters.
+#include <cuda_fp16.h>
+
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
 namespace uq {
 
+// alpha*, z_B* as fp32, or as IEEE half bits rounded to nearest even (the
+// 16-bit reals of the storage count of App. F.1).
+struct OutF32 {
+    using T = float;
+    static __device__ __forceinline__ T cvt(float v) { return v; }
+};
+struct OutF16 {
+    using T = uint16_t;
+    static __device__ __forceinline__ T cvt(float v) { return __half_as_ushort(__float2half_rn(v)); }
+};
+
 __device__ __forceinline__ uint32_t gather_bit(uint32_t four_codes, int j) {
     return (((four_codes >> j) & 0x01010101u) * 0x01020408u) >> 24;
 }
 
-template <int Q, typename WT, bool EQ4>
+template <int Q, typename WT, bool EQ4, typename OT>
 __global__ void __launch_bounds__(kThreads)
 export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const float* __restrict__ ZU,
               const float* __restrict__ ALPHA, const float* __restrict__ ZB, const uint8_t* __restrict__ CODES,
-              uint32_t* __restrict__ PLANES, float* __restrict__ ASTAR, float* __restrict__ ZSTAR, int64_t out,
-              int n_in, int g) {
+              uint32_t* __restrict__ PLANES, typename OT::T* __restrict__ ASTAR, typename OT::T* __restrict__ ZSTAR,
+              int64_t out, int n_in, int g) {
     constexpr int L = 1 << Q;
     constexpr uint32_t kMask = uint32_t(L - 1) * 0x01010101u;
     const int words = n_in / 32;
@@ -36,8 +49,8 @@ export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const
     for (int64_t grp = tid; grp < out * Gr; grp += nthr) {
         const float d = __ldg(DELTA + grp);
 #pragma unroll
-        for (int j = 0; j < Q; ++j) ASTAR[grp * Q + j] = __fmul_rn(d, __ldg(ALPHA + grp * Q + j));
-        ZSTAR[grp] = __fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp)));
+        for (int j = 0; j < Q; ++j) ASTAR[grp * Q + j] = OT::cvt(__fmul_rn(d, __ldg(ALPHA + grp * Q + j)));
+        ZSTAR[grp] = OT::cvt(__fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp))));
     }
 
     // (row, wcol) of chunk ch = row * words + wcol, advanced by nthr chunks
@@ -113,31 +126,43 @@ static int export_grid(int64_t work) {
     return (int)(want < cap ? (want < 1 ? 1 : want) : cap);
 }
 
-template <int Q, typename WT, bool EQ4>
+template <int Q, typename WT, bool EQ4, typename OT>
 static cudaError_t run_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, uint32_t* planes,
-                              float* astar, float* zstar, cudaStream_t st) {
+                              typename OT::T* astar, typename OT::T* zstar, cudaStream_t st) {
     const int grid = export_grid(sh.out * (int64_t)(sh.n_in / 32));
-    export_kernel<Q, WT, EQ4><<<grid, kThreads, 0, st>>>(W, p.delta, p.zu, p.alpha, p.zb, codes, planes, astar,
-                                                         zstar, sh.out, sh.n_in, sh.g);
+    export_kernel<Q, WT, EQ4, OT><<<grid, kThreads, 0, st>>>(W, p.delta, p.zu, p.alpha, p.zb, codes, planes, astar,
+                                                             zstar, sh.out, sh.n_in, sh.g);
     return cudaGetLastError();
 }
 
-template <int Q>
+template <int Q, typename OT>
 static cudaError_t export_q(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
-                            uint32_t* planes, float* astar, float* zstar, cudaStream_t st) {
-    if (mode == UQ_EXPORT_REUSE_CODES) return run_export<Q, WF32, false>(sh, W, p, codes, planes, astar, zstar, st);
-    if (sh.wdtype == UQ_W_BF16) return run_export<Q, WBF16, true>(sh, W, p, codes, planes, astar, zstar, st);
-    return run_export<Q, WF32, true>(sh, W, p, codes, planes, astar, zstar, st);
+                            uint32_t* planes, typename OT::T* astar, typename OT::T* zstar, cudaStream_t st) {
+    if (mode == UQ_EXPORT_REUSE_CODES)
+        return run_export<Q, WF32, false, OT>(sh, W, p, codes, planes, astar, zstar, st);
+    if (sh.wdtype == UQ_W_BF16) return run_export<Q, WBF16, true, OT>(sh, W, p, codes, planes, astar, zstar, st);
+    return run_export<Q, WF32, true, OT>(sh, W, p, codes, planes, astar, zstar, st);
+}
+
+template <typename OT>
+static cudaError_t export_any(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
+                              uint32_t* planes, typename OT::T* astar, typename OT::T* zstar, cudaStream_t st) {
+    switch (sh.q) {
+        case 1: return export_q<1, OT>(sh, W, p, codes, mode, planes, astar, zstar, st);
+        case 2: return export_q<2, OT>(sh, W, p, codes, mode, planes, astar, zstar, st);
+        case 3: return export_q<3, OT>(sh, W, p, codes, mode, planes, astar, zstar, st);
+        default: return export_q<4, OT>(sh, W, p, codes, mode, planes, astar, zstar, st);
+    }
 }
 
 cudaError_t launch_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
                           uint32_t* planes, float* astar, float* zstar, cudaStream_t st) {
-    switch (sh.q) {
-        case 1: return export_q<1>(sh, W, p, codes, mode, planes, astar, zstar, st);
-        case 2: return export_q<2>(sh, W, p, codes, mode, planes, astar, zstar, st);
-        case 3: return export_q<3>(sh, W, p, codes, mode, planes, astar, zstar, st);
-        default: return export_q<4>(sh, W, p, codes, mode, planes, astar, zstar, st);
-    }
+    return export_any<OutF32>(sh, W, p, codes, mode, planes, astar, zstar, st);
+}
+
+cudaError_t launch_export_half(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
+                               uint32_t* planes, uint16_t* astar, uint16_t* zstar, cudaStream_t st) {
+    return export_any<OutF16>(sh, W, p, codes, mode, planes, astar, zstar, st);
 }
 
 }  // namespace uq

@@ -22,9 +22,12 @@ struct Shape {
 cudaError_t launch_fwd(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
                        float* what, cudaStream_t st);
 cudaError_t launch_bwd(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
-                       uq_grads gr, cudaStream_t st);
+                       uq_grads gr, cudaStream_t st, int filter = UQ_FILTER_STE);
 cudaError_t launch_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
                           uint32_t* planes, float* astar, float* zstar, cudaStream_t st);
+// The same export with alpha*, z_B* written as IEEE half (bits), rounded to nearest even.
+cudaError_t launch_export_half(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, int mode,
+                               uint32_t* planes, uint16_t* astar, uint16_t* zstar, cudaStream_t st);
 cudaError_t launch_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
                         cudaStream_t st);
 
@@ -33,7 +36,7 @@ bool stream_path_ok(const Shape& sh);
 cudaError_t launch_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
                               float* what, cudaStream_t st);
 cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
-                              const float* gup, uq_grads gr, cudaStream_t st);
+                              const float* gup, uq_grads gr, cudaStream_t st, int filter = UQ_FILTER_STE);
 // Fused optimisation step (uq_step.cu): backward of step t, SGD update,
 // forward of step t + 1 in `mode` (a FWD_* value).  step_path_ok tells
 // whether the shape is one the fused kernel handles.

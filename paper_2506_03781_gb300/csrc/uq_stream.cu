@@ -79,7 +79,9 @@ __device__ void drain(unsigned long long (&bars)[NST], long long waited, long lo
 // Backward
 // ---------------------------------------------------------------------------
 
-template <int Q, typename WT, int G_>
+// ELEM: the whole-element filter (a filtered element drops out of every
+// gradient); otherwise the filter cuts the straight-through path only.
+template <int Q, typename WT, int G_, bool ELEM>
 __global__ void __launch_bounds__(kThreads, UQ_STREAM_BWD_MIN_BLOCKS)
 bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
                   const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
@@ -203,14 +205,15 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                         const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
                         const bool f = fabsf(__fsub_rn(x, m)) <= tau;
                         const float fu = f ? uu : 0.f;
-                        const float gfu = G[kq] * fu;
+                        const float gk = (ELEM && !f) ? 0.f : G[kq];
+                        const float gfu = gk * fu;
                         ds[kq] = -__fdividef(dl * gfu, s4[kq]);
-                        acc[0] += G[kq] * (mm.y - fu);
-                        acc[1] += f ? 0.f : G[kq];
-                        acc[2] += G[kq];
+                        acc[0] += gk * (mm.y - fu);
+                        acc[1] += f ? 0.f : gk;
+                        acc[2] += gk;
                         acc[3] += gfu;
 #pragma unroll
-                        for (int jj = 0; jj < Q; ++jj) acc[4 + jj] += ((c >> jj) & 1) ? G[kq] : -G[kq];
+                        for (int jj = 0; jj < Q; ++jj) acc[4 + jj] += ((c >> jj) & 1) ? gk : -gk;
                     }
                     *reinterpret_cast<float4*>(DS + ebase + el) = make_float4(ds[0], ds[1], ds[2], ds[3]);
                 }
@@ -462,7 +465,10 @@ static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
     return cudaSuccess;
 }
 
-template <int Q, typename WT, int G_>
+template <typename St, bool ELEM>
+struct BwdTag {};
+
+template <int Q, typename WT, int G_, bool ELEM>
 static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
                                   const float* gup, uq_grads gr, cudaStream_t st) {
     using St = Stage<Q, WT, G_, true, true, true, UQ_BWD_STAGE_BYTES>;
@@ -470,9 +476,10 @@ static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, c
     const int R = rows_per_block(U);
     const int n_rb = (int)((sh.out + R - 1) / R);
     const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
-    auto kern = bwd_stream_kernel<Q, WT, G_>;
+    auto kern = bwd_stream_kernel<Q, WT, G_, ELEM>;
     int grid = 0;
-    cudaError_t e = grid_for<St>(kern, dyn, n_rb, grid);
+    // one occupancy cache (and shared-memory opt-in) per kernel variant
+    cudaError_t e = grid_for<BwdTag<St, ELEM>>(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr,
                                       gr.ddelta, gr.dzu, gr.dzb, gr.dalpha, sh.out, sh.n_in, R, n_rb);
@@ -505,12 +512,19 @@ static cudaError_t run_fwd_stream(const Shape& sh, const void* W, uq_params p, u
     return run_fwd_stream_mode<Q, WT, G_, FWD_FULL>(sh, W, p, codes, what, st);
 }
 
+template <int Q, typename WT, bool ELEM>
+static cudaError_t bwd_stream_gf(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
+                                 const float* gup, uq_grads gr, cudaStream_t st) {
+    if (sh.g == 32) return run_bwd_stream<Q, WT, 32, ELEM>(sh, W, p, codes, gup, gr, st);
+    if (sh.g == 64) return run_bwd_stream<Q, WT, 64, ELEM>(sh, W, p, codes, gup, gr, st);
+    return run_bwd_stream<Q, WT, 128, ELEM>(sh, W, p, codes, gup, gr, st);
+}
+
 template <int Q, typename WT>
 static cudaError_t bwd_stream_g(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
-                                const float* gup, uq_grads gr, cudaStream_t st) {
-    if (sh.g == 32) return run_bwd_stream<Q, WT, 32>(sh, W, p, codes, gup, gr, st);
-    if (sh.g == 64) return run_bwd_stream<Q, WT, 64>(sh, W, p, codes, gup, gr, st);
-    return run_bwd_stream<Q, WT, 128>(sh, W, p, codes, gup, gr, st);
+                                const float* gup, uq_grads gr, int filter, cudaStream_t st) {
+    if (filter == UQ_FILTER_ELEMENT) return bwd_stream_gf<Q, WT, true>(sh, W, p, codes, gup, gr, st);
+    return bwd_stream_gf<Q, WT, false>(sh, W, p, codes, gup, gr, st);
 }
 
 template <int Q, typename WT>
@@ -523,9 +537,9 @@ static cudaError_t fwd_stream_g(const Shape& sh, const void* W, uq_params p, uin
 
 template <int Q>
 static cudaError_t bwd_stream_w(const Shape& sh, const void* W, uq_params p, const uint8_t* codes,
-                                const float* gup, uq_grads gr, cudaStream_t st) {
-    if (sh.wdtype == UQ_W_BF16) return bwd_stream_g<Q, WBF16>(sh, W, p, codes, gup, gr, st);
-    return bwd_stream_g<Q, WF32>(sh, W, p, codes, gup, gr, st);
+                                const float* gup, uq_grads gr, int filter, cudaStream_t st) {
+    if (sh.wdtype == UQ_W_BF16) return bwd_stream_g<Q, WBF16>(sh, W, p, codes, gup, gr, filter, st);
+    return bwd_stream_g<Q, WF32>(sh, W, p, codes, gup, gr, filter, st);
 }
 
 template <int Q>
@@ -536,12 +550,12 @@ static cudaError_t fwd_stream_w(const Shape& sh, const void* W, uq_params p, uin
 }
 
 cudaError_t launch_bwd_stream(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, const float* gup,
-                              uq_grads gr, cudaStream_t st) {
+                              uq_grads gr, cudaStream_t st, int filter) {
     switch (sh.q) {
-        case 1: return bwd_stream_w<1>(sh, W, p, codes, gup, gr, st);
-        case 2: return bwd_stream_w<2>(sh, W, p, codes, gup, gr, st);
-        case 3: return bwd_stream_w<3>(sh, W, p, codes, gup, gr, st);
-        default: return bwd_stream_w<4>(sh, W, p, codes, gup, gr, st);
+        case 1: return bwd_stream_w<1>(sh, W, p, codes, gup, gr, filter, st);
+        case 2: return bwd_stream_w<2>(sh, W, p, codes, gup, gr, filter, st);
+        case 3: return bwd_stream_w<3>(sh, W, p, codes, gup, gr, filter, st);
+        default: return bwd_stream_w<4>(sh, W, p, codes, gup, gr, filter, st);
     }
 }
 

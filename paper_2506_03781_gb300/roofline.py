@@ -28,6 +28,21 @@ def bytes_per_launch(kind: str, out: int, n_in: int, q: int, g: int, wbytes: int
         return n * (wbytes + 4 + 1 + 4 + 4 + 4 + 1) + 2 * gp + 2 * out * 4
     if kind == "step_keep":        # as step_remap, codes not rewritten
         return n * (wbytes + 4 + 1 + 4 + 4 + 4) + 2 * gp + 2 * out * 4
+    # OmniQuant maps: per group beta, gamma, alpha, z_B; no element-wise scale; W read on every step
+    ogp = groups * (3 + q) * 4
+    if kind == "omni_fwd_remap" or kind == "omni_fwd_full":   # read W, codes; write w^, codes
+        return n * (wbytes + 1 + 4 + 1) + ogp
+    if kind == "omni_fwd_keep":    # read W (for the group scales), codes; write w^
+        return n * (wbytes + 1 + 4) + ogp
+    if kind == "omni_bwd":         # read W, codes, dL/dw^; write the group gradients
+        return n * (wbytes + 1 + 4) + 2 * ogp
+    # AWQ maps: s_A per column, Delta_A, z_A, alpha, z_B per group
+    if kind == "awq_fwd_remap" or kind == "awq_fwd_full":
+        return n * (wbytes + 1 + 4 + 1) + gp + n_in * 4
+    if kind == "awq_fwd_keep":     # read codes; write w^ (W not read)
+        return n * (1 + 4) + gp + n_in * 4
+    if kind == "awq_bwd":          # read W, codes, dL/dw^; write group gradients and ds_A
+        return n * (wbytes + 1 + 4) + 2 * gp + 2 * n_in * 4
     if kind == "gemv":             # read planes, alpha*, z*, one token x (wbytes per value); write y
         return q * n // 8 + groups * (q + 1) * 4 + n_in * wbytes + out * 4
     if kind == "export_reuse":     # read codes; write planes, alpha*, z*

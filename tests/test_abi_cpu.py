@@ -247,6 +247,24 @@ def test_awq_validation(libpath):
     assert api.uq_awq_bwd_workspace_bytes(8, 512, 3, 128) >= 8 * 4
 
 
+@cpu_only
+def test_bwd_ex_and_half_export_validation(libpath):
+    from paper_2506_03781_gb300 import api
+    L = api.lib()
+    bwd = lambda flt, gr=None: L.uq_quantize_bwd_ex(FAKE, api.W_BF16, 8, 256, 3, 128, _params(api), FAKE + 0x9000,
+                                                    FAKE + 0xB000, gr or _grads(api), flt, None)
+    assert bwd(2) == api.UQ_ERR_ARG and "filter" in api.uq_last_error()
+    assert bwd(api.FILTER_ELEMENT, _grads(api, ds=0)) == api.UQ_ERR_ARG
+    assert bwd(api.FILTER_ELEMENT) == api.UQ_ERR_CUDA                 # valid: only the launch fails here
+    ex = lambda mode=0, a=FAKE, W=FAKE, codes=FAKE: L.uq_export_bcq_half(W, 1, 8, 256, 3, 128, _params(api), codes,
+                                                                         mode, FAKE, a, FAKE, None)
+    assert ex(mode=5) == api.UQ_ERR_ARG
+    assert ex(a=FAKE + 2) == api.UQ_ERR_ALIGN
+    assert ex(mode=1, W=0) == api.UQ_ERR_ARG
+    assert ex(codes=0) == api.UQ_ERR_ARG
+    assert ex() == api.UQ_ERR_CUDA
+
+
 def test_binding_rejects_host_tensors_before_calling(libpath):
     import torch
     from paper_2506_03781_gb300 import api
