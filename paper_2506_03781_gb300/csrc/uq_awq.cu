@@ -139,12 +139,18 @@ awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const f
     const int gi = u * NG + sub;
     const bool ok = gi < Gr;
     const int64_t cbase = (int64_t)gi * g + 4 * li;
-    float s[4][4], dsa[4][4];
+    // s_A of the unit's columns and its reciprocal, once: only x (the filter
+    // decision) needs the exact division; the gradient values take 1/s_A.
+    float s[4][4], rs[4][4], dsa[4][4];
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
 #pragma unroll
         for (int k = 0; k < 4; ++k) dsa[v][k] = 0.f;
-        if (ok && v < nv) f4_to(ldg4(SA + cbase + 4 * LPG * v), s[v]);
+        if (ok && v < nv) {
+            f4_to(ldg4(SA + cbase + 4 * LPG * v), s[v]);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) rs[v][k] = 1.f / s[v][k];
+        }
     }
 
     for (int64_t row = r0; row < r1; ++row) {
@@ -179,14 +185,14 @@ awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const f
                 const float uu = __fdiv_rn(ws, dl);
                 const float x = __fadd_rn(uu, za);
                 const bool f = fabsf(__fsub_rn(x, m)) <= tau;
-                const float gs = G[v][k] / s[v][k];
+                const float gs = G[v][k] * rs[v][k];
                 const float mz = m - za;
                 acc[0] += gs * (mz - (f ? uu : 0.f));
                 acc[1] += f ? 0.f : gs;
                 acc[2] += gs;
 #pragma unroll
                 for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? gs : -gs;
-                dsa[v][k] += gs * ((f ? w[v][k] : 0.f) - dl * mz / s[v][k]);
+                dsa[v][k] += gs * ((f ? w[v][k] : 0.f) - dl * mz * rs[v][k]);
             }
         }
         const int slot0 = SR8::run(acc, lane);

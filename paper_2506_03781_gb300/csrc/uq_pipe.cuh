@@ -9,6 +9,7 @@
 #pragma once
 
 #include "uq_common.cuh"
+#include "uq_launch.h"
 
 namespace uq {
 
@@ -87,7 +88,8 @@ constexpr int kMaxStages = 16;
 // Shared-memory stage layout of one work unit.  HAS_X: weights and s are
 // staged; HAS_G: dL/dW^ is staged; HAS_C: code words are staged.  The group
 // parameters (Delta, z_U, z_B, alpha of the unit's NG groups) always are.
-template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET>
+// HAS_S: s is staged with the weights (by default exactly when they are).
+template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET, bool HAS_S = HAS_X>
 struct Stage {
     static constexpr int LPG = G_ <= 64 ? 4 : 8;
     static constexpr int NG = 32 / LPG;                  // groups per unit
@@ -95,7 +97,7 @@ struct Stage {
     static constexpr int UE = NG * G_;                   // elements per unit
     static constexpr int WBYTES = sizeof(typename WT::raw) / 4;
     static constexpr int SZ_W = HAS_X ? UE * WBYTES : 0;
-    static constexpr int SZ_S = HAS_X ? UE * 4 : 0;
+    static constexpr int SZ_S = HAS_S ? UE * 4 : 0;
     static constexpr int SZ_G = HAS_G ? UE * 4 : 0;
     static constexpr int SZ_C = HAS_C ? UE : 0;
     static constexpr int SZ_P = NG * 4, SZ_A = NG * Q * 4;
@@ -125,5 +127,67 @@ struct Ring {
         if (++s == NST) { s = 0; parity ^= 1u; }
     }
 };
+
+// Work items of one warp: for its row blocks k = 0, 1, ... (block rows
+// (blockIdx.x + k * gridDim.x) * R + row_sub) the units wr, wr + WPR, ...
+// (n_w per row block).  Positions advance with Cursor::next, without
+// integer division.
+struct Items {
+    int R, WPR, row_sub, wr, n_w, n_blocks;
+    long long total;
+    __device__ Items(int U, int Rr, int n_rb, int warp) {
+        R = Rr;
+        WPR = kWarps / R;
+        row_sub = warp / WPR;
+        wr = warp % WPR;
+        n_w = wr < U ? (U - wr + WPR - 1) / WPR : 0;
+        n_blocks = (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+        total = (long long)n_blocks * n_w;
+    }
+    __device__ int64_t row(int k) const { return ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * R + row_sub; }
+    __device__ int unit(int j) const { return wr + WPR * j; }
+};
+
+struct Cursor {
+    int k = 0, j = 0;                        // row block, unit slot
+    __device__ void next(int n_w) {
+        if (++j == n_w) { j = 0; ++k; }
+    }
+};
+
+
+// After a wait ran out: waits (bounded again) for the copies of items
+// [waited, issued) of a warp's stage ring, so that none lands in shared
+// memory after the block has exited.  Lane 0 only.
+template <int NST>
+__device__ void drain(unsigned long long (&bars)[NST], long long waited, long long issued) {
+    for (long long i = waited; i < issued; ++i)
+        tma::bar_wait(tma::smem_addr(&bars[i % NST]), (uint32_t)((i / NST) & 1));
+}
+
+constexpr int kMaxDevices = 64;
+
+// Persistent grid: min(row blocks, SMs x resident blocks per SM).  The
+// shared-memory attribute and the occupancy of a kernel instantiation are
+// set and queried once per device (KERN is a distinct type per call site).
+template <typename Tag, typename KERN>
+static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
+    static int per_sm_cache[kMaxDevices] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    int per_sm = (dev >= 0 && dev < kMaxDevices) ? per_sm_cache[dev] : 0;
+    if (per_sm == 0) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) per_sm = 1;
+        if (dev >= 0 && dev < kMaxDevices) per_sm_cache[dev] = per_sm;
+    }
+    const long long cap = (long long)sm_count() * per_sm;
+    grid = (int)(n_rb < cap ? n_rb : cap);
+    return cudaSuccess;
+}
 
 }  // namespace uq

@@ -38,43 +38,6 @@ __device__ unsigned int g_stream_err = 0;
 #endif
 constexpr int kRowRing = 32;             // row blocks whose ds_r partials wait in shared memory
 
-// Work items of one warp: for its row blocks k = 0, 1, ... (block rows
-// (blockIdx.x + k * gridDim.x) * R + row_sub) the units wr, wr + WPR, ...
-// (n_w per row block).  Positions advance with Cursor::next, without
-// integer division.
-struct Items {
-    int R, WPR, row_sub, wr, n_w, n_blocks;
-    long long total;
-    __device__ Items(int U, int Rr, int n_rb, int warp) {
-        R = Rr;
-        WPR = kWarps / R;
-        row_sub = warp / WPR;
-        wr = warp % WPR;
-        n_w = wr < U ? (U - wr + WPR - 1) / WPR : 0;
-        n_blocks = (n_rb - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
-        total = (long long)n_blocks * n_w;
-    }
-    __device__ int64_t row(int k) const { return ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * R + row_sub; }
-    __device__ int unit(int j) const { return wr + WPR * j; }
-};
-
-struct Cursor {
-    int k = 0, j = 0;                        // row block, unit slot
-    __device__ void next(int n_w) {
-        if (++j == n_w) { j = 0; ++k; }
-    }
-};
-
-
-// After a wait ran out: waits (bounded again) for the copies of items
-// [waited, issued) of a warp's stage ring, so that none lands in shared
-// memory after the block has exited.  Lane 0 only.
-template <int NST>
-__device__ void drain(unsigned long long (&bars)[NST], long long waited, long long issued) {
-    for (long long i = waited; i < issued; ++i)
-        tma::bar_wait(tma::smem_addr(&bars[i % NST]), (uint32_t)((i / NST) & 1));
-}
-
 // ---------------------------------------------------------------------------
 // Backward
 // ---------------------------------------------------------------------------
@@ -424,8 +387,6 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // Launchers
 // ---------------------------------------------------------------------------
 
-constexpr int kMaxDevices = 64;
-
 int sm_count() {
     static int cached[kMaxDevices] = {0};
     int dev = 0, n = 0;
@@ -440,29 +401,6 @@ bool stream_path_ok(const Shape& sh) {
     if (!(sh.g == 32 || sh.g == 64 || sh.g == 128)) return false;
     const int ue = sh.g == 32 ? 256 : 512;
     return sh.n_in % ue == 0;
-}
-
-// Persistent grid: min(row blocks, SMs x resident blocks per SM).  The
-// shared-memory attribute and the occupancy of a kernel instantiation are
-// set and queried once per device (KERN is a distinct type per call site).
-template <typename Tag, typename KERN>
-static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
-    static int per_sm_cache[kMaxDevices] = {0};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    int per_sm = (dev >= 0 && dev < kMaxDevices) ? per_sm_cache[dev] : 0;
-    if (per_sm == 0) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-        if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
-        if (e != cudaSuccess) return e;
-        if (per_sm < 1) per_sm = 1;
-        if (dev >= 0 && dev < kMaxDevices) per_sm_cache[dev] = per_sm;
-    }
-    const long long cap = (long long)sm_count() * per_sm;
-    grid = (int)(n_rb < cap ? n_rb : cap);
-    return cudaSuccess;
 }
 
 template <typename St, bool ELEM>
