@@ -217,6 +217,114 @@ struct SegReduce {
     }
 };
 
+// ---------------------------------------------------------------------------
+// Backward terms of the pipelined kernels (App. C.1 filter, Eq. 1, Eq. 3)
+// ---------------------------------------------------------------------------
+//
+// The filter f = (|x - w~| <= tau) decides an integer-like outcome, so it is
+// always taken on the IEEE value x = fl(fl(w / den) + z_U).  The gradient
+// values only need u = w / den to a few ulps.  The pipelined backward
+// therefore forms u from the hardware reciprocal estimate of den (PTX
+// rcp.approx.ftz.f32, relative error at most 2^-23 for normal results) and
+// takes the filter from it only where that is provably the IEEE decision:
+//
+//   with u' = fl(w r), x' = fl(u' + z_U), d' = fl(x' - w~): |u' - u| <=
+//   2^-22 |u'| (the reciprocal's 2^-23 plus one rounding on each side), and
+//   one rounding of each sum on each side adds 2^-23 of its magnitude, so
+//   |d' - d| <= 2^-21 |x'| + 2^-22 |z_U| + 2^-23 |w~| to first order
+//   (subnormal results add at most 2^-148).
+//
+// With E = 2^-18 |x'| + 2^-19 (|z_U| + sum_j |alpha_j| + |z_B|) + 2^-126 (at
+// least eight times that bound, since |w~| <= sum_j |alpha_j| + |z_B|), a
+// vector of 4 elements whose every ||d'| - tau| exceeds E, with every |den|
+// below 2^125 (so that r is a normal number), gets the same filter as the
+// IEEE path.  Any other vector -- one element near the filter boundary, a
+// den outside that range, an infinity or a NaN anywhere (every comparison
+// with them is false) -- is recomputed with the IEEE division.  Either way
+// every decision equals that of x computed by transform_x.
+//
+// The same reciprocal gives 1/s = r (Delta s_r), so ds = -G Delta f u / s =
+// -(G f u) (r k) with k = (Delta Delta) s_r per group and row; a group whose
+// k is not a normal number below 2^125 takes the IEEE path for every vector
+// (eg = infinity below).
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
+// Per group: the part of E that does not depend on the element, or infinity
+// when the reciprocal path may not be used for the group (k out of range).
+__device__ __forceinline__ float bwd_margin(float zu, float zb, const float* alpha, int q, float k) {
+    float m = __fadd_rn(fabsf(zu), fabsf(zb));
+    for (int j = 0; j < q; ++j) m = __fadd_rn(m, fabsf(alpha[j]));
+    const bool k_ok = fabsf(k) < 0x1p125f && fabsf(k) >= 0x1p-125f;
+    return k_ok ? __fmaf_rn(m, 0x1p-19f, 0x1p-126f) : __int_as_float(0x7f800000);
+}
+
+// Backward of 4 consecutive elements of one group.  tab[c] = (l(c), l(c) -
+// z_U) for code word c.  Writes ds (dL/ds), and accumulates
+//   acc[0] += G (w~ - z_U - f u)      (dDelta)
+//   acc[1] += G (1 - f)               (dz_U / -Delta)
+//   acc[2] += G                       (dz_B / Delta; S)
+//   acc[3] += G f u                   (Delta-free part of ds_r)
+//   acc[4 + j] += G where bit j of c is set (P_j; dalpha_j = Delta (2 P_j - S))
+// ELEM: the whole-element filter (G -> f G in every term).
+template <int Q, bool ELEM>
+__device__ __forceinline__ void bwd_vec4(const float w[4], const float s4[4], const float G[4], uint32_t cv,
+                                         const float2* __restrict__ tab, float dl, float sr, float zu, float tau,
+                                         float eg, float k, float ds[4], float acc[8]) {
+    constexpr int L = 1 << Q;
+    float2 mm[4];
+    float u[4], d[4], rk[4];
+    bool sure = true;
+#pragma unroll
+    for (int kq = 0; kq < 4; ++kq) {
+        mm[kq] = tab[(cv >> (8 * kq)) & (L - 1)];
+        const float den = __fmul_rn(__fmul_rn(dl, s4[kq]), sr);
+        const float r = rcp_approx(den);
+        u[kq] = __fmul_rn(w[kq], r);
+        const float x = __fadd_rn(u[kq], zu);
+        d[kq] = __fsub_rn(x, mm[kq].x);
+        rk[kq] = __fmul_rn(r, k);
+        const float E = __fmaf_rn(fabsf(x), 0x1p-18f, eg);
+        sure = sure & (fabsf(__fsub_rn(fabsf(d[kq]), tau)) > E) & (fabsf(den) < 0x1p125f);
+    }
+    if (!sure) {
+#pragma unroll
+        for (int kq = 0; kq < 4; ++kq) {
+            const float x = transform_x(w[kq], s4[kq], dl, sr, zu, u[kq]);
+            d[kq] = __fsub_rn(x, mm[kq].x);
+            rk[kq] = __fdividef(dl, s4[kq]);
+        }
+    }
+#pragma unroll
+    for (int kq = 0; kq < 4; ++kq) {
+        const int c = (cv >> (8 * kq)) & (L - 1);
+        const bool f = fabsf(d[kq]) <= tau;
+        const float fu = f ? u[kq] : 0.f;
+        const float gk = (ELEM && !f) ? 0.f : G[kq];
+        const float gfu = __fmul_rn(gk, fu);
+        ds[kq] = -__fmul_rn(gfu, rk[kq]);
+        acc[0] = __fmaf_rn(gk, __fsub_rn(mm[kq].y, fu), acc[0]);
+        acc[1] = f ? acc[1] : __fadd_rn(acc[1], gk);
+        acc[2] = __fadd_rn(acc[2], gk);
+        acc[3] = __fadd_rn(acc[3], gfu);
+#pragma unroll
+        for (int j = 0; j < Q; ++j)
+            if ((c >> j) & 1) acc[4 + j] = __fadd_rn(acc[4 + j], gk);
+    }
+}
+
+// After SegReduce<LPG>::run over the bwd_vec4 accumulators (LPG 4 or 8):
+// S = slot 2's total, fetched from the lane that holds it.
+template <int LPG>
+__device__ __forceinline__ float seg_slot2(const float v[8], int lane) {
+    static_assert(LPG == 4 || LPG == 8, "slot 2 sits in v[0] of lane 2 / NOUT");
+    return __shfl_sync(kFull, v[0], (lane & ~(LPG - 1)) | (2 / SegReduce<LPG>::NOUT));
+}
+
 // Rows per block for the unit mapping: the largest power of two R <= 8 with
 // R * units_per_row <= 8 (at least 1).
 __host__ __device__ inline int rows_per_block(int units_per_row) {

@@ -75,6 +75,7 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
     __shared__ __align__(8) unsigned long long bars[kWarps][2];
     __shared__ StepTab<Q, NG> tabs[kWarps];
     __shared__ float tau_s[kWarps][NG];
+    __shared__ float eg_s[kWarps][NG];            // element-independent part of the filter margin
     __shared__ float red[2][kWarps];              // ds_r partials (Delta S3 sums) of row blocks k, k + 1
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -160,10 +161,13 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
 #pragma unroll
                     for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
                     tau_s[warp][kk] = m;
+                    const float kg = __fmul_rn(__fmul_rn(pd[kk], pd[kk]), sr);
+                    eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, kg);
                 }
             }
             __syncwarp();
-            const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub];
+            const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+            const float kds = __fmul_rn(__fmul_rn(dl, dl), sr);         // Delta / s = r kds, r = 1 / den
             const int64_t ebase = row * n_in + (int64_t)unit * UE;
             float acc[8];
 #pragma unroll
@@ -177,30 +181,17 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                 f4_to(*sp, s4);
                 f4_to(*reinterpret_cast<const float4*>(st + St::OFF_G + el * 4), G);
                 const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+                float ds[4];
+                bwd_vec4<Q, false>(w, s4, G, cv, t.a[sub], dl, sr, zu, tau, eg, kds, ds, acc);
 #pragma unroll
-                for (int kq = 0; kq < 4; ++kq) {
-                    const int c = (cv >> (8 * kq)) & (L - 1);
-                    const float2 mm = t.a[sub][c];
-                    float uu;
-                    const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
-                    const bool f = fabsf(__fsub_rn(x, mm.x)) <= tau;
-                    const float fu = f ? uu : 0.f;
-                    const float gfu = G[kq] * fu;
-                    const float ds = -__fdividef(dl * gfu, s4[kq]);
-                    sn[kq] = __fsub_rn(s4[kq], __fmul_rn(lr_f, ds));
-                    acc[0] += G[kq] * (mm.y - fu);
-                    acc[1] += f ? 0.f : G[kq];
-                    acc[2] += G[kq];
-                    acc[3] += gfu;
-#pragma unroll
-                    for (int jj = 0; jj < Q; ++jj) acc[4 + jj] += ((c >> jj) & 1) ? G[kq] : -G[kq];
-                }
+                for (int kq = 0; kq < 4; ++kq) sn[kq] = __fsub_rn(s4[kq], __fmul_rn(lr_f, ds[kq]));
                 const float4 s_new = make_float4(sn[0], sn[1], sn[2], sn[3]);
                 *reinterpret_cast<float4*>(S + ebase + el) = s_new;
                 *sp = s_new;                       // the forward of step t + 1 reads s' from the stage
             }
             __syncwarp();                          // every lane has read the old staged parameters
             const int slot0 = SR8::run(acc, lane);
+            const float S = seg_slot2<LPG>(acc, lane);
             if (SR8::writer(lane)) {
                 const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
 #pragma unroll
@@ -221,9 +212,9 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                         ZB[grp] = v;
                     } else if (slot == 3) {
                         prow += dl * tot;                          // Delta S3 of the group
-                    } else if (slot - 4 < Q) {                     // dalpha_j = Delta tot
+                    } else if (slot - 4 < Q) {                     // dalpha_j = Delta (2 P_j - S)
                         const int j = slot - 4;
-                        const float v = __fsub_rn(pa[sub * Q + j], __fmul_rn(lr_b, dl * tot));
+                        const float v = __fsub_rn(pa[sub * Q + j], __fmul_rn(lr_b, dl * __fmaf_rn(2.f, tot, -S)));
                         pa[sub * Q + j] = v;
                         ALPHA[grp * Q + j] = v;
                     }

@@ -60,6 +60,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ float2 tabs[kWarps][NG][L];          // (l(c), l(c) - z_U) per group slot and code word
     __shared__ float tau_s[kWarps][NG];
+    __shared__ float eg_s[kWarps][NG];              // element-independent part of the filter margin
     __shared__ float red[kRowRing][kWarps];       // per row block and warp: sum of Delta S3
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
@@ -142,10 +143,13 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 #pragma unroll
                         for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
                         tau_s[warp][kk] = m;
+                        const float kg = __fmul_rn(__fmul_rn(pd[kk], pd[kk]), sr);
+                        eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, kg);
                     }
                 }
                 __syncwarp();
-                const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub];
+                const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+                const float kds = __fmul_rn(__fmul_rn(dl, dl), sr);     // Delta / s = r kds, r = 1 / den
                 const int unit = it.unit(j);
                 const int64_t ebase = row * n_in + (int64_t)unit * UE;
                 float acc[8];
@@ -159,28 +163,11 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_G + el * 4), G);
                     const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
-#pragma unroll
-                    for (int kq = 0; kq < 4; ++kq) {
-                        const int c = (cv >> (8 * kq)) & (L - 1);
-                        const float2 mm = t[sub][c];
-                        const float m = mm.x;
-                        float uu;
-                        const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
-                        const bool f = fabsf(__fsub_rn(x, m)) <= tau;
-                        const float fu = f ? uu : 0.f;
-                        const float gk = (ELEM && !f) ? 0.f : G[kq];
-                        const float gfu = gk * fu;
-                        ds[kq] = -__fdividef(dl * gfu, s4[kq]);
-                        acc[0] += gk * (mm.y - fu);
-                        acc[1] += f ? 0.f : gk;
-                        acc[2] += gk;
-                        acc[3] += gfu;
-#pragma unroll
-                        for (int jj = 0; jj < Q; ++jj) acc[4 + jj] += ((c >> jj) & 1) ? gk : -gk;
-                    }
+                    bwd_vec4<Q, ELEM>(w, s4, G, cv, t[sub], dl, sr, zu, tau, eg, kds, ds, acc);
                     *reinterpret_cast<float4*>(DS + ebase + el) = make_float4(ds[0], ds[1], ds[2], ds[3]);
                 }
                 const int slot0 = SR8::run(acc, lane);
+                const float S = seg_slot2<LPG>(acc, lane);
                 if (SR8::writer(lane)) {
                     const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
 #pragma unroll
@@ -191,7 +178,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                         else if (slot == 1) DZU[grp] = -(dl * tot);
                         else if (slot == 2) DZB[grp] = dl * tot;
                         else if (slot == 3) prow += dl * tot;
-                        else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * tot;
+                        else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * __fmaf_rn(2.f, tot, -S);
                     }
                 }
             }

@@ -109,5 +109,26 @@ def oracle_bwd(W, P, codes, Gup, g):
     return O.quantize_bwd(*args), O.bwd_l1_mass(*args)
 
 
+def boundary_weights(P, codes, g, seed, ulps=4):
+    """fp32 weights that put every element within `ulps` ulps of the filter
+    boundary |x - w~| = tau (App. C.1): x is aimed at w~ +- tau (1 + k 2^-23),
+    k uniform in [-ulps, ulps], and w = (x - z_U) Delta s s_r in fp64, so
+    roughly half the elements are filtered and some sit exactly on the
+    boundary.  Built from the oracle's levels; the codes are the given ones."""
+    out, n_in = P["s"].shape
+    Gr = n_in // g
+    lv = O.levels(P["alpha"], P["zb"])
+    m = O.reconstruct(np.asarray(codes).reshape(out, Gr, g).astype(np.int64), lv).astype(np.float64)
+    tau = np.abs(np.asarray(P["alpha"], np.float64)).min(-1)[..., None]
+    rng = np.random.default_rng(seed)
+    x = m + rng.choice([-1.0, 1.0], m.shape) * tau * (1.0 + rng.integers(-ulps, ulps + 1, m.shape) * 2.0 ** -23)
+    den = (np.asarray(P["delta"], np.float64)[..., None] * np.asarray(P["s"], np.float64).reshape(out, Gr, g)
+           * np.asarray(P["sr"], np.float64)[:, None, None])
+    W = ((x - np.asarray(P["zu"], np.float64)[..., None]) * den).astype(F32).reshape(out, n_in)
+    x32, _ = O.transform_F(W.reshape(out, Gr, g), P["s"].reshape(out, Gr, g), P["delta"], P["zu"], P["sr"][:, None])
+    gap = np.abs(x32 - O.reconstruct(np.asarray(codes).reshape(out, Gr, g).astype(np.int64), lv)) - tau
+    return W, gap.reshape(out, n_in)
+
+
 def slice_rows(P, rows):
     return {k: np.ascontiguousarray(np.asarray(v)[rows]) for k, v in P.items()}

@@ -142,6 +142,24 @@ def test_edge_level_ties_negative_alpha_and_high_code_bits():
     C.assert_grads_close(gr, ref, mass, "ties-bwd")
 
 
+@pytest.mark.parametrize("q,g", [(1, 32), (2, 64), (3, 128), (4, 128), (3, 256)])
+def test_bwd_filter_boundary_within_ulps(q, g):
+    """Every element within 4 ulps of the filter boundary |x - w~| = tau, some
+    exactly on it: the filter decisions must be those of the IEEE quotient
+    (a flipped decision moves ds of that element from 0 to -G Delta u / s or
+    back, far outside the tolerance), whichever way the kernel forms x."""
+    out, n_in = 24, 1024
+    _, W0, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=700 + 10 * q + g, wdtype="f32")
+    _, codes = O.quantize_fwd(W0, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                              O.MAP_LOCAL_PERIODIC, 0, 2)
+    W, gap = C.boundary_weights(P, codes, g, seed=q + g)
+    assert 0.3 < (gap > 0).mean() < 0.7 and (gap == 0).mean() > 0.02
+    gr = C.gpu_bwd(W, P, codes, Gup, q, g)
+    ref, mass = C.oracle_bwd(W, P, codes, Gup, g)
+    C.assert_grads_close(gr, ref, mass, f"boundary q={q} g={g}")
+    assert np.array_equal(gr["ds"] == 0, ref["ds"] == 0)          # the same elements filtered
+
+
 def test_exact_decision_ties_are_bit_exact():
     """Dyadic weights and parameters put many elements exactly half-way
     between two levels; both sides must take the same (documented) choice."""

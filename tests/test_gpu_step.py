@@ -192,6 +192,26 @@ def test_step_equals_separate_entry_points(out, n_in, g):
         assert np.array_equal(a[1], b[1]) and np.array_equal(a[2], b[2]), (t, mode)
 
 
+@pytest.mark.parametrize("q,g", [(2, 64), (3, 128)])
+def test_step_filter_boundary_within_ulps(q, g):
+    """Weights within 4 ulps of the filter boundary (every vector of the
+    backward phase takes the IEEE fallback): the fused step still equals the
+    separate entry points bit for bit, and the oracle (the forward of t + 1 is
+    a keep step, so no mapping near-ties enter)."""
+    out, n_in = 16, 1024
+    _, W0, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=40 + q, wdtype="f32")
+    _, codes = O.quantize_fwd(W0, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                              O.MAP_LOCAL_PERIODIC, 0, 2)
+    W, gap = C.boundary_weights(P, codes, g, seed=q)
+    assert 0.3 < (gap > 0).mean() < 0.7
+    a = gpu_step(W, P, codes, Gup, q, g, 0, O.MAP_LOCAL_PERIODIC, 2)
+    b = separate_path(W, P, codes, Gup, q, g, 0, O.MAP_LOCAL_PERIODIC, 2)
+    for k in PK:
+        assert np.array_equal(a[0][k], b[0][k]), k
+    assert np.array_equal(a[1], b[1]) and np.array_equal(a[2], b[2])
+    check_against_oracle(W, W, P, codes, Gup, q, g, 0, O.MAP_LOCAL_PERIODIC, 2, label=f"boundary q{q} g{g}")
+
+
 def test_multistep_chain_equals_separate_entry_points():
     """Eight consecutive steps (remap and keep alternating) on each path,
     each from its own state: still bit-identical."""
