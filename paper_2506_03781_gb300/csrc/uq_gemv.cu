@@ -43,6 +43,13 @@ constexpr size_t kGemvSmemLimit = 227 * 1024;   // dynamic shared memory a block
 __host__ __device__ constexpr int gemv_tile_groups(int g) { return g < kTileCols ? kTileCols / g : 1; }
 // 32-bit words of one stage: 8 rows x (q planes x 16 words + the tile's alpha* and z*).
 __host__ __device__ constexpr int gemv_stage_words(int q, int ng) { return kBatchRows * (q * kTileWords + ng * (q + 1)); }
+// Stages per warp: as many (up to kMaxStagesGemv) as fit next to the tables.
+__host__ __device__ constexpr int gemv_stages(int q, int ng) {
+    return (int)((kGemvSmemLimit - kGemvFixedSmem) / (kGemvWarps * (size_t)gemv_stage_words(q, ng) * 4)) >
+                   kMaxStagesGemv
+               ? kMaxStagesGemv
+               : (int)((kGemvSmemLimit - kGemvFixedSmem) / (kGemvWarps * (size_t)gemv_stage_words(q, ng) * 4));
+}
 
 struct XF32 {
     static __device__ __forceinline__ float get(const void* x, int64_t i) { return static_cast<const float*>(x)[i]; }
@@ -75,10 +82,14 @@ template <int Q, typename XT, int NGT>
 __global__ void __launch_bounds__(kGemvThreads, 1)
 bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __restrict__ ASTAR,
                         const float* __restrict__ ZSTAR, const void* __restrict__ X, float* __restrict__ PART,
-                        int64_t out, int n_in, int g, int batch, int n_tiles, int64_t rows_per_block, int NS) {
+                        int64_t out, int n_in, int g, int batch, int n_tiles, int64_t rows_per_block, bool pwide) {
     constexpr int PR = NGT * (Q + 1);                 // parameter words per row and tile
     constexpr int PW = kBatchRows * Q * kTileWords;   // plane words per stage (the parameters follow)
     constexpr int SW = gemv_stage_words(Q, NGT);
+    constexpr int NS = gemv_stages(Q, NGT);
+    static_assert(NS >= 2, "two stages must fit");
+    // 16-byte pieces of one row's alpha* and z* in a tile (pwide layout)
+    constexpr int PA = NGT * Q / 4, PP = NGT * (Q + 1) / 4;
     constexpr int LPG = 32 / NGT;                     // lanes per group within a tile (NGT >= 2)
     extern __shared__ __align__(16) float gsm[];
     float* lut = gsm;                                 // [2][256][32]
@@ -107,7 +118,7 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
     const bool valid = c0 + 16 * lane < n_in;
     using SR = SegReduce<32>;
 
-    // copies of this warp's k-th row batch into stage k % NS
+    // copies of this warp's k-th row batch into stage k % NS (NS a compile-time constant)
     auto issue = [&](int k) {
         uint32_t* st = wst + (size_t)(k % NS) * SW;
         const int rb = kBatchRows * (warp + kGemvWarps * k);
@@ -129,6 +140,21 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
         }
         const float* ab = atile + (int64_t)rb * Gr * Q;
         const float* zb = ztile + (int64_t)rb * Gr;
+        if constexpr (NGT % 4 == 0) {
+            if (pwide) {                                            // whole tile, 16-byte aligned rows
+#pragma unroll
+                for (int i = 0; i < (kBatchRows * PP + 31) / 32; ++i) {
+                    const int e = lane + 32 * i;
+                    const int rr = e / PP, f = e - rr * PP;
+                    if (e < kBatchRows * PP && rr < rows) {
+                        const bool isa = f < PA;
+                        const float* src = isa ? ab + (int64_t)rr * Gr * Q + 4 * f : zb + (int64_t)rr * Gr + 4 * (f - PA);
+                        cp16(st + PW + rr * PR + 4 * f, src);        // z* follows alpha* in the stage row
+                    }
+                }
+                return;
+            }
+        }
 #pragma unroll
         for (int i = 0; i < (kBatchRows * PR + 31) / 32; ++i) {
             const int e = lane + 32 * i;
@@ -266,12 +292,14 @@ template <int Q, typename XT, int NGT>
 static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in,
                             int g, const void* x, int batch, float* y, float* work, cudaStream_t st) {
     auto kern = bcq_gemv_partial_kernel<Q, XT, NGT>;
-    // stages per warp: as many (up to 4) as fit next to the tables
     constexpr size_t stage_bytes = (size_t)gemv_stage_words(Q, NGT) * 4;
-    size_t ns = (kGemvSmemLimit - kGemvFixedSmem) / (kGemvWarps * stage_bytes);
-    if (ns > (size_t)kMaxStagesGemv) ns = kMaxStagesGemv;
-    static_assert((kGemvSmemLimit - kGemvFixedSmem) / (kGemvWarps * stage_bytes) >= 2, "two stages must fit");
-    const size_t smem = kGemvFixedSmem + kGemvWarps * ns * stage_bytes;
+    constexpr size_t smem = kGemvFixedSmem + kGemvWarps * (size_t)gemv_stages(Q, NGT) * stage_bytes;
+    static_assert(gemv_stages(Q, NGT) >= 2 && smem <= kGemvSmemLimit, "two stages must fit");
+    // alpha* and z* rows of a tile move in 16-byte pieces when every tile is
+    // whole (in a multiple of 512) and holds a multiple of 4 groups (both
+    // arrays start on 16-byte boundaries: the entry point checks that);
+    // otherwise in 4-byte pieces
+    const bool pwide = NGT % 4 == 0 && n_in % kTileCols == 0;
     static int per_sm_cache[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -303,7 +331,7 @@ static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const fl
         if (best < 0.0 || cost < best) { best = cost; n_rb = nb; rpb = r; }
     }
     kern<<<(unsigned)(n_rb * n_tiles), kGemvThreads, smem, st>>>(planes, astar, zstar, x, work, out, n_in, g, batch,
-                                                                 n_tiles, rpb, (int)ns);
+                                                                 n_tiles, rpb, pwide);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int64_t n = (int64_t)batch * out;
