@@ -127,6 +127,7 @@ awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const f
     using SR8 = SegReduce<LPG>;
     __shared__ LvTab<Q, NG> tabs[kWarps];
     __shared__ float tau_s[kWarps][NG];
+    __shared__ float amag_s[kWarps][NG];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     LvTab<Q, NG>& t = tabs[warp];
     const int Gr = n_in / g;
@@ -169,22 +170,32 @@ awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const f
         }
         const float dl = ok ? __ldg(DELTA + grp) : 1.f, za = ok ? __ldg(ZA + grp) : 0.f;
         __syncwarp();                             // previous row is done with the tables
-        unit_levels<Q, NG>(t, tau_s[warp], lane, ALPHA, ZB, row * Gr + u * NG, min(NG, Gr - u * NG));
+        unit_levels<Q, NG>(t, tau_s[warp], lane, ALPHA, ZB, row * Gr + u * NG, min(NG, Gr - u * NG), amag_s[warp]);
         const float tau = tau_s[warp][sub];
+        // x = (w s_A) / Delta_A + z_A: one reciprocal of Delta_A per group, the
+        // filter proven equal to the IEEE one (shared_div_filter4)
+        const float rdl = rcp_approx(dl);
+        const float eg = ok ? bwd_margin_of(__fadd_rn(fabsf(za), amag_s[warp][sub]), dl) : 0.f;
         float acc[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i] = 0.f;
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
             if (!(ok && v < nv)) continue;
+            float ws[4], m4[4], uv[4];
+            bool fv[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                ws[k] = __fmul_rn(w[v][k], s[v][k]);
+                m4[k] = t.lv[sub][(cv[v] >> (8 * k)) & (L - 1)];
+            }
+            shared_div_filter4(ws, dl, rdl, za, m4, tau, eg, uv, fv);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int c = (cv[v] >> (8 * k)) & (L - 1);
-                const float m = t.lv[sub][c];
-                const float ws = __fmul_rn(w[v][k], s[v][k]);
-                const float uu = __fdiv_rn(ws, dl);
-                const float x = __fadd_rn(uu, za);
-                const bool f = fabsf(__fsub_rn(x, m)) <= tau;
+                const float m = m4[k];
+                const float uu = uv[k];
+                const bool f = fv[k];
                 const float gs = G[v][k] * rs[v][k];
                 const float mz = m - za;
                 acc[0] += gs * (mz - (f ? uu : 0.f));

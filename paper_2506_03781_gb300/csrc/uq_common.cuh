@@ -119,11 +119,13 @@ struct MapTab {                      // + sorted order and local-mapping neighbo
     uint8_t rk[NS][L];
 };
 
-// Levels l(c) of the NS groups grp0 + k (k < n_ok) and tau = min_j |alpha_j|.
+// Levels l(c) of the NS groups grp0 + k (k < n_ok), tau = min_j |alpha_j| and,
+// if amag is given, sum_j |alpha_j| + |z_B| (a bound on every |l(c)|).
 // Whole warp; ends with __syncwarp().
 template <int Q, int NS, typename TAB>
 __device__ __forceinline__ void unit_levels(TAB& t, float* tau, int lane, const float* __restrict__ alpha,
-                                            const float* __restrict__ zb, int64_t grp0, int n_ok) {
+                                            const float* __restrict__ zb, int64_t grp0, int n_ok,
+                                            float* amag = nullptr) {
     constexpr int L = 1 << Q;
     constexpr int E = NS * L;
 #pragma unroll
@@ -135,12 +137,19 @@ __device__ __forceinline__ void unit_levels(TAB& t, float* tau, int lane, const 
             float a[Q];
 #pragma unroll
             for (int j = 0; j < Q; ++j) a[j] = __ldg(alpha + grp * Q + j);
-            lvv = level_of<Q>(c, a, __ldg(zb + grp));
+            const float zbv = __ldg(zb + grp);
+            lvv = level_of<Q>(c, a, zbv);
             if (tau != nullptr && c == 0) {
                 float m = fabsf(a[0]);
 #pragma unroll
                 for (int j = 1; j < Q; ++j) m = fminf(m, fabsf(a[j]));
                 tau[k] = m;
+                if (amag != nullptr) {
+                    float s = fabsf(zbv);
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) s = __fadd_rn(s, fabsf(a[j]));
+                    amag[k] = s;
+                }
             }
         }
         t.lv[k][c] = lvv;
@@ -256,11 +265,15 @@ __device__ __forceinline__ float rcp_approx(float x) {
 
 // Per group: the part of E that does not depend on the element, or infinity
 // when the reciprocal path may not be used for the group (k out of range).
+// mag = |z_U| + sum_j |alpha_j| + |z_B|.
+__device__ __forceinline__ float bwd_margin_of(float mag, float k) {
+    const bool k_ok = fabsf(k) < 0x1p125f && fabsf(k) >= 0x1p-125f;
+    return k_ok ? __fmaf_rn(mag, 0x1p-19f, 0x1p-126f) : __int_as_float(0x7f800000);
+}
 __device__ __forceinline__ float bwd_margin(float zu, float zb, const float* alpha, int q, float k) {
     float m = __fadd_rn(fabsf(zu), fabsf(zb));
     for (int j = 0; j < q; ++j) m = __fadd_rn(m, fabsf(alpha[j]));
-    const bool k_ok = fabsf(k) < 0x1p125f && fabsf(k) >= 0x1p-125f;
-    return k_ok ? __fmaf_rn(m, 0x1p-19f, 0x1p-126f) : __int_as_float(0x7f800000);
+    return bwd_margin_of(m, k);
 }
 
 // Backward of 4 consecutive elements of one group.  tab[c] = (l(c), l(c) -
@@ -315,6 +328,36 @@ __device__ __forceinline__ void bwd_vec4(const float w[4], const float s4[4], co
         for (int j = 0; j < Q; ++j)
             if ((c >> j) & 1) acc[4 + j] = __fadd_rn(acc[4 + j], gk);
     }
+}
+
+// Filter decisions of 4 elements whose x = nu / dv + z share the divisor dv
+// (OmniQuant's Delta_O, AWQ's Delta_A; App. E): u = nu / dv from r =
+// rcp_approx(dv) where the margin test above proves the decision equal to
+// that of the IEEE quotient, else (the whole vector) from __fdiv_rn.  m[k] =
+// w~ of element k; eg = bwd_margin(z, z_B, alpha, q, dv), which is infinity
+// unless dv is a normal number below 2^125.  Returns u (for the gradient
+// values) and f.
+__device__ __forceinline__ void shared_div_filter4(const float nu[4], float dv, float r, float z, const float m[4],
+                                                   float tau, float eg, float u[4], bool f[4]) {
+    float d[4];
+    bool sure = true;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        u[k] = __fmul_rn(nu[k], r);
+        const float x = __fadd_rn(u[k], z);
+        d[k] = __fsub_rn(x, m[k]);
+        const float E = __fmaf_rn(fabsf(x), 0x1p-18f, eg);
+        sure = sure & (fabsf(__fsub_rn(fabsf(d[k]), tau)) > E);
+    }
+    if (!sure) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            u[k] = __fdiv_rn(nu[k], dv);
+            d[k] = __fsub_rn(__fadd_rn(u[k], z), m[k]);
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) f[k] = fabsf(d[k]) <= tau;
 }
 
 // After SegReduce<LPG>::run over the bwd_vec4 accumulators (LPG 4 or 8):

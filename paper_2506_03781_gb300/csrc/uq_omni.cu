@@ -504,6 +504,10 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
             }
             __syncwarp();
             const float tau = tau_s[warp][sub];
+            // x = w / Delta_O + z_O: one reciprocal of Delta_O per group, the
+            // filter proven equal to the IEEE one (shared_div_filter4)
+            const float rdl = rcp_approx(dl);
+            const float eg = bwd_margin(zo, pb[sub], pa + sub * Q, Q, dl);
             float acc[8];
 #pragma unroll
             for (int q8 = 0; q8 < 8; ++q8) acc[q8] = 0.f;
@@ -513,19 +517,24 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 float G[4];
                 f4_to(*reinterpret_cast<const float4*>(st + St::OFF_G + el * 4), G);
                 const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+                float m4[4], uv[4];
+                bool fv[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) m4[k] = lvs[warp][sub][(cv >> (8 * k)) & (L - 1)];
+                shared_div_filter4(w[v], dl, rdl, zo, m4, tau, eg, uv, fv);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int c = (cv >> (8 * k)) & (L - 1);
-                    const float m = lvs[warp][sub][c];
-                    const float uu = __fdiv_rn(w[v][k], dl);
-                    const float x = __fadd_rn(uu, zo);
-                    const bool f = fabsf(__fsub_rn(x, m)) <= tau;
+                    const float m = m4[k];
+                    const float uu = uv[k];
+                    const bool f = fv[k];
                     const float gk = G[k];
                     acc[0] += gk * ((m - zo) - (f ? uu : 0.f));
                     acc[1] += f ? 0.f : gk;
                     acc[2] += gk;
 #pragma unroll
-                    for (int j = 0; j < Q; ++j) acc[4 + j] += ((c >> j) & 1) ? gk : -gk;
+                    for (int j = 0; j < Q; ++j)                  // P_j: dalpha_j = Delta (2 P_j - S)
+                        if ((c >> j) & 1) acc[4 + j] += gk;
                 }
             }
             const int slot0 = SR8::run(acc, lane);
@@ -548,7 +557,7 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 DGAMMA[grp] = A * dDg + B * dzg;
                 DZB[grp] = dl * sg[2];
 #pragma unroll
-                for (int j = 0; j < Q; ++j) DALPHA[grp * Q + j] = dl * sg[4 + j];
+                for (int j = 0; j < Q; ++j) DALPHA[grp * Q + j] = dl * __fmaf_rn(2.f, sg[4 + j], -sg[2]);
             }
         }
         __syncwarp();                                    // stage, tables and sums are free again

@@ -83,6 +83,34 @@ def test_awq_backward_within_l1_mass_tolerance(out, n_in, g, q):
         assert not bad.any(), f"{k}: {int(bad.sum())} outside; worst {(err / (mass[k] + 1e-30)).max():.3g}"
 
 
+@pytest.mark.parametrize("q,g", [(1, 32), (2, 64), (3, 128), (4, 128), (3, 512)])
+def test_awq_backward_filter_boundary_within_ulps(q, g):
+    """Weights placed within 4 ulps of the filter boundary |x - w~| = tau
+    (x = (w s_A) / Delta_A + z_A): the decisions must be those of the IEEE
+    quotient however the kernel forms x."""
+    out, n_in = 24, 1024
+    raw, W, P, codes, Gup = inputs(out, n_in, q, g, seed=650 + q + g, wdtype="f32")
+    Gr = n_in // g
+    m = O.reconstruct(codes.reshape(out, Gr, g).astype(np.int64), O.levels(P["alpha"], P["zb"])).astype(np.float64)
+    tau = np.abs(P["alpha"].astype(np.float64)).min(-1)[..., None]
+    rng = np.random.default_rng(q + g)
+    xt = m + rng.choice([-1.0, 1.0], m.shape) * tau * (1.0 + rng.integers(-4, 5, m.shape) * 2.0 ** -23)
+    wn = ((xt - P["za"].astype(np.float64)[..., None]) * P["delta"].astype(np.float64)[..., None]
+          / P["sa"].astype(np.float64).reshape(1, Gr, g))
+    W2 = wn.astype(F32).reshape(out, n_in)
+    Wd = api.weights_tensor(W2, C.dev())
+    nan = lambda *s: torch.full(s, float("nan"), device=C.dev())
+    gr = {"dsa": nan(n_in), "ddelta": nan(out, Gr), "dza": nan(out, Gr), "dalpha": nan(out, Gr, q),
+          "dzb": nan(out, Gr)}
+    api.uq_quantize_bwd_awq(Wd, q, g, dev_params(P), torch.from_numpy(codes).cuda(), torch.from_numpy(Gup).cuda(), gr)
+    args = (W2, P["sa"], P["delta"], P["za"], P["alpha"], P["zb"], codes, Gup, g)
+    ref, mass = O.quantize_bwd_awq(*args), O.bwd_l1_mass_awq(*args)
+    for k in ("dsa", "ddelta", "dza", "dalpha", "dzb"):
+        err = np.abs(C.host(gr[k]).astype(np.float64) - ref[k])
+        bad = err > 1e-4 * mass[k] + 1e-30
+        assert not bad.any(), f"{k}: {int(bad.sum())} outside; worst {(err / (mass[k] + 1e-30)).max():.3g}"
+
+
 @pytest.mark.parametrize("g", [32, 128, 512])
 def test_awq_export_through_uq_export_bcq_bit_exact(g):
     q = 3

@@ -101,6 +101,41 @@ def test_omni_backward_within_l1_mass_tolerance(out, n_in, g, q):
         assert not bad.any(), f"{k}: {int(bad.sum())} outside; worst {(err / (mass[k] + 1e-30)).max():.3g}"
 
 
+@pytest.mark.parametrize("q,g", [(1, 32), (2, 64), (3, 128), (4, 128), (3, 256)])
+def test_omni_backward_filter_boundary_within_ulps(q, g):
+    """Weights placed within 4 ulps of the filter boundary |x - w~| = tau
+    (x = w / Delta_O + z_O), the group's smallest and largest weight kept so
+    that Delta_O and z_O do not move: the decisions must be those of the IEEE
+    quotient however the kernel forms x (a flipped decision moves dz-terms by
+    a whole G, far outside the tolerance)."""
+    out, n_in = 24, 1024
+    raw, W, P, codes, Gup = inputs(out, n_in, q, g, seed=600 + q + g, wdtype="f32")
+    Gr = n_in // g
+    delta, zo = O.omni_params(W, P["beta"], P["gamma"], q, g)
+    m = O.reconstruct(codes.reshape(out, Gr, g).astype(np.int64), O.levels(P["alpha"], P["zb"])).astype(np.float64)
+    tau = np.abs(P["alpha"].astype(np.float64)).min(-1)[..., None]
+    rng = np.random.default_rng(q + g)
+    xt = m + rng.choice([-1.0, 1.0], m.shape) * tau * (1.0 + rng.integers(-4, 5, m.shape) * 2.0 ** -23)
+    Wg = W.reshape(out, Gr, g).astype(np.float64)
+    wn = (xt - zo.astype(np.float64)[..., None]) * delta.astype(np.float64)[..., None]
+    lo, hi = Wg.min(-1, keepdims=True), Wg.max(-1, keepdims=True)
+    inside = (wn > lo) & (wn < hi) & (Wg > lo) & (Wg < hi)        # the extremes themselves stay
+    W2 = np.where(inside, wn, Wg).astype(F32).reshape(out, n_in)
+    assert np.array_equal(O.omni_params(W2, P["beta"], P["gamma"], q, g)[0], delta) and inside.mean() > 0.5
+    Wd = api.weights_tensor(W2, C.dev())
+    gr = {"dbeta": torch.full((out, Gr), float("nan"), device=C.dev()),
+          "dgamma": torch.full((out, Gr), float("nan"), device=C.dev()),
+          "dalpha": torch.full((out, Gr, q), float("nan"), device=C.dev()),
+          "dzb": torch.full((out, Gr), float("nan"), device=C.dev())}
+    api.uq_quantize_bwd_omni(Wd, q, g, dev_params(P), torch.from_numpy(codes).cuda(), torch.from_numpy(Gup).cuda(), gr)
+    args = (W2, P["beta"], P["gamma"], P["alpha"], P["zb"], codes, Gup, g)
+    ref, mass = O.quantize_bwd_omni(*args), O.bwd_l1_mass_omni(*args)
+    for k in ("dbeta", "dgamma", "dalpha", "dzb"):
+        err = np.abs(C.host(gr[k]).astype(np.float64) - ref[k])
+        bad = err > 1e-4 * mass[k] + 1e-30
+        assert not bad.any(), f"{k}: {int(bad.sum())} outside; worst {(err / (mass[k] + 1e-30)).max():.3g}"
+
+
 def test_omni_unsupported_group_size_raises():
     raw, W, P, codes, _ = inputs(4, 2048, 2, 1024, seed=1)
     Wd = api.weights_tensor(raw, C.dev())
