@@ -1,7 +1,10 @@
 // Unified initialization (Algorithm 2) with the clipping strategies of
-// App. E.2 and the general alternating update of Algorithm 3: one warp per
-// group, the group's transformed weights x and code words kept in shared
-// memory.  Runs once before training; not on the per-step path.
+// App. E.2 and the general alternating update of Algorithm 3: one lane per
+// group for g <= 128 (init_lane_kernel), one warp per group for larger
+// groups (init_kernel); the group's transformed weights x and code words
+// kept in shared memory.  Runs once before training; not on the per-step
+// path.  A round of the alternating update that moves no code (and not z_B)
+// is a fixed point: the remaining rounds are skipped, which changes nothing.
 //
 // Sums that feed alpha and z_B are taken in fp64 (the group's fp32 values
 // are summed exactly in practice); the normal equations C^T C alpha =
@@ -94,9 +97,10 @@ __device__ __forceinline__ void solve_fp64(const long long Ain[Q][Q], const doub
 #pragma unroll
     for (int k = 0; k < Q; ++k) {
         int p = k;
+        double piv = fabs(A[k][k]);
 #pragma unroll
         for (int i = k + 1; i < Q; ++i)
-            if (fabs(A[i][k]) > fabs(A[p][k])) p = i;
+            if (fabs(A[i][k]) > piv) { piv = fabs(A[i][k]); p = i; }
 #pragma unroll
         for (int i = k + 1; i < Q; ++i) {
             if (i == p) {
@@ -242,12 +246,16 @@ __global__ void init_kernel(const void* __restrict__ W, int64_t n_groups, int n_
             }
             float srt[L];
             sorted_levels<Q>(tb, lane, a, zb, srt);
+            bool moved = false;
             for (int i = lane; i < g; i += 32) {
                 float m;
                 const int r = nearest_rank<L>(xs[i], srt, m);
+                moved |= cs[i] != tb.cor[r];
                 cs[i] = tb.cor[r];
             }
+            moved = __any_sync(kFull, moved);
             __syncwarp();
+            const float zb_prev = zb;
             if (G == 1) {
                 double sres = 0.0;
                 for (int i = lane; i < g; i += 32) {
@@ -260,6 +268,9 @@ __global__ void init_kernel(const void* __restrict__ W, int64_t n_groups, int n_
                 sres = warp_sum_d(sres);
                 zb = (float)(sres / (double)g);
             }
+            // a fixed point (no code and not z_B moved): the remaining rounds
+            // would repeat it bit for bit (warp-uniform: zb and moved are)
+            if (!moved && __float_as_uint(zb) == __float_as_uint(zb_prev)) break;
         }
 
         // --- candidate error with the full mapping (Eq. 2), s = s_r = 1 ---
@@ -303,9 +314,265 @@ __global__ void init_kernel(const void* __restrict__ W, int64_t n_groups, int n_
     }
 }
 
+// ---------------------------------------------------------------------------
+// One lane per group (g <= 128)
+// ---------------------------------------------------------------------------
+//
+// The same computation as init_kernel, laid out for a GPU whose fp64 rate is
+// a small fraction of its fp32 rate: lane l of a warp owns group 32 w + l
+// whole, so every fp64 sum is lane-local (no fp64 shuffles) and each lane
+// solves the normal equations of its own group once (init_kernel solves
+// them on all 32 lanes of the group's warp).  y = x - z_B is kept in fp64
+// across the T rounds (z_B only moves when G == 1).  Shared memory per warp,
+// element-major so that the 32 lanes touch consecutive words: y [g][32]
+// fp64, x [g][32] fp32, code words [g][32], and the sorted levels and their
+// code words [L][32].  Every fp32 operation and every decision is the one
+// init_kernel takes; the fp64 sums run in another order (lane-sequential),
+// which gives the same values whenever they are exact.
+constexpr int kLaneInitMaxG = 128;
+
+template <int Q>
+__device__ __forceinline__ void lane_sorted_levels(const float a[Q], float zb, float* srt_s, uint8_t* cor_s,
+                                                   int lane, float srt[1 << Q], uint64_t& cor) {
+    constexpr int L = 1 << Q;
+    float lv[L];
+#pragma unroll
+    for (int c = 0; c < L; ++c) lv[c] = level_of<Q>(c, a, zb);
+#pragma unroll
+    for (int c = 0; c < L; ++c) {
+        int r = 0;
+#pragma unroll
+        for (int c2 = 0; c2 < L; ++c2) r += (lv[c2] < lv[c]) || (lv[c2] == lv[c] && c2 < c);
+        srt_s[r * 32 + lane] = lv[c];
+        cor_s[r * 32 + lane] = static_cast<uint8_t>(c);
+    }
+    cor = 0;
+#pragma unroll
+    for (int r = 0; r < L; ++r) {
+        srt[r] = srt_s[r * 32 + lane];
+        cor |= uint64_t(cor_s[r * 32 + lane]) << (4 * r);
+    }
+}
+
+template <int Q, typename WT, int G_>
+__global__ void init_lane_kernel(const void* __restrict__ W, int64_t n_groups, int n_in, int G, int T, int clip,
+                                 float* __restrict__ DELTA, float* __restrict__ ZU, float* __restrict__ S,
+                                 float* __restrict__ SR, float* __restrict__ ALPHA, float* __restrict__ ZB,
+                                 uint8_t* __restrict__ CODES) {
+    constexpr int L = 1 << Q;
+    constexpr size_t WARP_BYTES = (size_t)G_ * 32 * (8 + 4 + 1) + (size_t)L * 32 * (4 + 1);
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char* base = smem + (size_t)warp * ((WARP_BYTES + 15) & ~size_t(15));
+    double* yd = reinterpret_cast<double*>(base);                       // [G_][32]
+    float* xs = reinterpret_cast<float*>(yd + G_ * 32);                 // [G_][32]
+    float* srt_s = xs + G_ * 32;                                        // [L][32]
+    uint8_t* cs = reinterpret_cast<uint8_t*>(srt_s + L * 32);           // [G_][32]
+    uint8_t* cor_s = cs + G_ * 32;                                      // [L][32]
+
+    const int64_t grp0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + warp) * 32;
+    if (grp0 >= n_groups) return;                      // whole warp; no block barrier in this kernel
+    const int64_t grp_raw = grp0 + lane;
+    const bool live = grp_raw < n_groups;
+    const int64_t grp = live ? grp_raw : n_groups - 1; // absent lanes repeat the last group, store nothing
+    const int Gr = n_in / G_;
+    const int64_t row = grp / Gr;
+    const int64_t eoff = row * (int64_t)n_in + (grp % Gr) * (int64_t)G_;
+    auto wval = [&](int i) -> float {
+        if constexpr (sizeof(typename WT::raw) == sizeof(float4))
+            return __ldg(static_cast<const float*>(W) + eoff + i);
+        else
+            return __uint_as_float(uint32_t(__ldg(static_cast<const unsigned short*>(W) + eoff + i)) << 16);
+    };
+    auto X = [&](int i) -> float& { return xs[i * 32 + lane]; };
+    auto C = [&](int i) -> uint8_t& { return cs[i * 32 + lane]; };
+    auto Y = [&](int i) -> double& { return yd[i * 32 + lane]; };
+
+    float wmin = INFINITY, wmax = -INFINITY;
+#pragma unroll 2
+    for (int i = 0; i < G_; ++i) {
+        const float w = wval(i);
+        wmin = fminf(wmin, w);
+        wmax = fmaxf(wmax, w);
+    }
+    const float top = (float)(L - 1);
+    const float rng = fmaxf(__fsub_rn(wmax, wmin), 1e-12f);
+
+    double e_best = INFINITY;
+    float bd = 0.f, bz = 0.f, bzb = top * 0.5f, ba[Q];
+#pragma unroll
+    for (int j = 0; j < Q; ++j) ba[j] = 0.f;
+    float srt[L];
+    uint64_t cor;
+
+    for (int gi = 1; gi <= G; ++gi) {
+        const float gamma = __fdiv_rn((float)gi, (float)G);
+        const float dc = __fdiv_rn(__fmul_rn(gamma, rng), top);
+        float zc;
+        if (clip == UQ_CLIP_FIXED_MIN) zc = __fdiv_rn(-wmin, dc);
+        else if (clip == UQ_CLIP_FIXED_MAX) zc = __fsub_rn(top, __fdiv_rn(wmax, dc));
+        else zc = __fdiv_rn(-__fmul_rn(gamma, wmin), dc);
+#pragma unroll 2
+        for (int i = 0; i < G_; ++i) {
+            float u;
+            X(i) = transform_x(wval(i), 1.f, dc, 1.f, zc, u);
+            C(i) = 0;
+        }
+
+        // --- Algorithm 3: greedy start (one bit at a time) ---
+        float a[Q], zb = bzb;
+#pragma unroll
+        for (int j = 0; j < Q; ++j) {
+            double sabs = 0.0;
+#pragma unroll 2
+            for (int i = 0; i < G_; ++i) {
+                float r = __fsub_rn(X(i), zb);
+                const int c = C(i);
+#pragma unroll
+                for (int jj = 0; jj < j; ++jj) r = __fsub_rn(r, ((c >> jj) & 1) ? a[jj] : -a[jj]);
+                sabs += (double)fabsf(r);
+                if (r >= 0.f) C(i) = (uint8_t)(c | (1 << j));
+            }
+            a[j] = (float)(sabs / (double)G_);
+        }
+#pragma unroll 2
+        for (int i = 0; i < G_; ++i) Y(i) = (double)X(i) - (double)zb;
+
+        // --- T rounds of alpha, C (and z_B when G == 1) ---
+        for (int it = 0; it < T; ++it) {
+            long long ctc[Q][Q];
+            double cty[Q];
+            // off-diagonal entries of C^T C from counts of differing bits:
+            // sum_i c_ij c_ik = g - 2 #{i: bit j != bit k}; the diagonal is g
+            uint32_t diff[Q][Q];
+#pragma unroll
+            for (int j = 0; j < Q; ++j) {
+                cty[j] = 0.0;
+#pragma unroll
+                for (int k = 0; k < Q; ++k) diff[j][k] = 0u;
+            }
+#pragma unroll 2
+            for (int i = 0; i < G_; ++i) {
+                const uint32_t c = C(i);
+                const double y = Y(i);
+#pragma unroll
+                for (int j = 0; j < Q; ++j) {
+                    cty[j] += ((c >> j) & 1) ? y : -y;
+#pragma unroll
+                    for (int k = j + 1; k < Q; ++k) diff[j][k] += ((c >> j) ^ (c >> k)) & 1u;
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < Q; ++j) {
+                ctc[j][j] = G_;
+#pragma unroll
+                for (int k = j + 1; k < Q; ++k) {
+                    ctc[j][k] = (long long)G_ - 2 * (long long)diff[j][k];
+                    ctc[k][j] = ctc[j][k];
+                }
+            }
+            if (!int_singular<Q>(ctc)) {
+                double sol[Q];
+                solve_fp64<Q>(ctc, cty, sol);
+#pragma unroll
+                for (int j = 0; j < Q; ++j) a[j] = (float)sol[j];
+            }
+            lane_sorted_levels<Q>(a, zb, srt_s, cor_s, lane, srt, cor);
+            bool moved = false;
+#pragma unroll 2
+            for (int i = 0; i < G_; ++i) {
+                float m;
+                const int r = nearest_rank<L>(X(i), srt, m);
+                const uint8_t c = (uint8_t)((cor >> (4 * r)) & 15u);
+                moved |= c != C(i);
+                C(i) = c;
+            }
+            const float zb_prev = zb;
+            if (G == 1) {
+                double sres = 0.0;
+#pragma unroll 2
+                for (int i = 0; i < G_; ++i) {
+                    const int c = C(i);
+                    double ca = 0.0;
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) ca += ((c >> j) & 1) ? (double)a[j] : -(double)a[j];
+                    sres += (double)X(i) - ca;
+                }
+                zb = (float)(sres / (double)G_);
+#pragma unroll 2
+                for (int i = 0; i < G_; ++i) Y(i) = (double)X(i) - (double)zb;
+            }
+            // No code moved (and z_B did not either): the next round would
+            // solve the same system, get the same alpha and the same codes, so
+            // every remaining round repeats this state bit for bit.
+            if (!moved && __float_as_uint(zb) == __float_as_uint(zb_prev)) break;
+        }
+
+        // --- candidate error with the full mapping (Eq. 2), s = s_r = 1 ---
+        lane_sorted_levels<Q>(a, zb, srt_s, cor_s, lane, srt, cor);
+        double e = 0.0;
+#pragma unroll 2
+        for (int i = 0; i < G_; ++i) {
+            float m;
+            nearest_rank<L>(X(i), srt, m);
+            const float what = __fmul_rn(dc, __fsub_rn(m, zc));
+            const double df = (double)wval(i) - (double)what;
+            e += df * df;
+        }
+        if (e < e_best) {
+            e_best = e;
+            bd = dc;
+            bz = zc;
+            bzb = zb;
+#pragma unroll
+            for (int j = 0; j < Q; ++j) ba[j] = a[j];
+        }
+    }
+
+    lane_sorted_levels<Q>(ba, bzb, srt_s, cor_s, lane, srt, cor);
+    if (!live) return;                                 // no warp-wide operation follows
+    DELTA[grp] = bd;
+    ZU[grp] = bz;
+    ZB[grp] = bzb;
+#pragma unroll
+    for (int j = 0; j < Q; ++j) ALPHA[grp * Q + j] = ba[j];
+    if (grp % Gr == 0) SR[row] = 1.f;
+#pragma unroll 2
+    for (int i = 0; i < G_; ++i) {
+        float u, m;
+        const float x = transform_x(wval(i), 1.f, bd, 1.f, bz, u);
+        const int r = nearest_rank<L>(x, srt, m);
+        CODES[eoff + i] = (uint8_t)((cor >> (4 * r)) & 15u);
+        S[eoff + i] = 1.f;
+    }
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t run_init_lane(const Shape& sh, const void* W, int G, int T, int clip, uq_params p,
+                                 uint8_t* codes, cudaStream_t st) {
+    constexpr int L = 1 << Q;
+    constexpr size_t warp_bytes = (((size_t)G_ * 32 * 13 + (size_t)L * 32 * 5) + 15) & ~size_t(15);
+    // as many warps as fit in the 227 KB a block may opt in to, at most 16
+    constexpr int wpb = (int)((227 * 1024) / warp_bytes) > 16 ? 16 : (int)((227 * 1024) / warp_bytes);
+    static_assert(wpb >= 1, "one warp's tables must fit");
+    const int64_t n_groups = sh.out * (int64_t)(sh.n_in / G_);
+    const size_t dyn = warp_bytes * wpb;
+    auto kern = init_lane_kernel<Q, WT, G_>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    if (e != cudaSuccess) return e;
+    const int64_t per_block = (int64_t)wpb * 32;
+    const int64_t blocks = (n_groups + per_block - 1) / per_block;
+    kern<<<dim3((unsigned)blocks), wpb * 32, dyn, st>>>(W, n_groups, sh.n_in, G, T, clip, p.delta, p.zu, p.s, p.sr,
+                                                       p.alpha, p.zb, codes);
+    return cudaGetLastError();
+}
+
 template <int Q, typename WT>
 static cudaError_t run_init(const Shape& sh, const void* W, int G, int T, int clip, uq_params p, uint8_t* codes,
                             cudaStream_t st) {
+    if (sh.g == 32) return run_init_lane<Q, WT, 32>(sh, W, G, T, clip, p, codes, st);
+    if (sh.g == 64) return run_init_lane<Q, WT, 64>(sh, W, G, T, clip, p, codes, st);
+    if (sh.g == kLaneInitMaxG) return run_init_lane<Q, WT, 128>(sh, W, G, T, clip, p, codes, st);
     const int64_t n_groups = sh.out * (int64_t)(sh.n_in / sh.g);
     const size_t per_warp = (size_t)sh.g * (sizeof(float) + 1);
     int wpc = (int)((96 * 1024) / per_warp);
