@@ -322,14 +322,38 @@ __global__ void init_kernel(const void* __restrict__ W, int64_t n_groups, int n_
 // a small fraction of its fp32 rate: lane l of a warp owns group 32 w + l
 // whole, so every fp64 sum is lane-local (no fp64 shuffles) and each lane
 // solves the normal equations of its own group once (init_kernel solves
-// them on all 32 lanes of the group's warp).  y = x - z_B is kept in fp64
-// across the T rounds (z_B only moves when G == 1).  Shared memory per warp,
-// element-major so that the 32 lanes touch consecutive words: y [g][32]
-// fp64, x [g][32] fp32, code words [g][32], and the sorted levels and their
-// code words [L][32].  Every fp32 operation and every decision is the one
-// init_kernel takes; the fp64 sums run in another order (lane-sequential),
-// which gives the same values whenever they are exact.
+// them on all 32 lanes of the group's warp).  During the T rounds x is
+// fixed and only the code words move, so C^T (x - z_B) and C^T C are formed
+// from per-code-word sums of x and counts (a round touches only the elements
+// whose code moved).  Shared memory per warp, element-major so that the 32
+// lanes touch consecutive words (init_lane_warp_bytes).  Every fp32
+// operation and every decision is the one init_kernel takes; the fp64 sums
+// run in another order (lane-sequential, grouped by code word), which gives
+// the same values whenever they are exact.
 constexpr int kLaneInitMaxG = 128;
+
+// Shared memory of one warp: the per-code sums of x [L][32] fp64, x
+// [g][32], the sorted levels [L][32], the code words [g][32] and the codes
+// of the sorted levels [L][32]; rounded up to 16 bytes.
+__host__ __device__ constexpr size_t init_lane_warp_bytes(int q, int g) {
+    return (((size_t)(1 << q) * 32 * (8 + 4 + 1) + (size_t)g * 32 * (4 + 1)) + 15) & ~size_t(15);
+}
+
+// Counts of the L code words of one group (at most 255 each), 8 bits per
+// code word packed in 64-bit registers; c is a compile-time index wherever
+// get() is used, add() takes any c.
+template <int L>
+struct CodeHist {
+    uint64_t lo = 0, hi = 0;                           // code words 0..7, 8..15
+    __device__ __forceinline__ void add(int c, int d) {
+        const uint64_t v = (uint64_t)(int64_t)d << (8 * (c & 7));
+        if (L <= 8 || c < 8) lo += v;
+        else hi += v;
+    }
+    __device__ __forceinline__ int get(int c) const {
+        return (int)(((c < 8 ? lo : hi) >> (8 * (c & 7))) & 0xffu);
+    }
+};
 
 template <int Q>
 __device__ __forceinline__ void lane_sorted_levels(const float a[Q], float zb, float* srt_s, uint8_t* cor_s,
@@ -360,12 +384,12 @@ __global__ void init_lane_kernel(const void* __restrict__ W, int64_t n_groups, i
                                  float* __restrict__ SR, float* __restrict__ ALPHA, float* __restrict__ ZB,
                                  uint8_t* __restrict__ CODES) {
     constexpr int L = 1 << Q;
-    constexpr size_t WARP_BYTES = (size_t)G_ * 32 * (8 + 4 + 1) + (size_t)L * 32 * (4 + 1);
+    constexpr size_t WARP_BYTES = init_lane_warp_bytes(Q, G_);
     extern __shared__ __align__(16) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    unsigned char* base = smem + (size_t)warp * ((WARP_BYTES + 15) & ~size_t(15));
-    double* yd = reinterpret_cast<double*>(base);                       // [G_][32]
-    float* xs = reinterpret_cast<float*>(yd + G_ * 32);                 // [G_][32]
+    unsigned char* base = smem + (size_t)warp * WARP_BYTES;
+    double* bx = reinterpret_cast<double*>(base);                       // [L][32]
+    float* xs = reinterpret_cast<float*>(bx + L * 32);                  // [G_][32]
     float* srt_s = xs + G_ * 32;                                        // [L][32]
     uint8_t* cs = reinterpret_cast<uint8_t*>(srt_s + L * 32);           // [G_][32]
     uint8_t* cor_s = cs + G_ * 32;                                      // [L][32]
@@ -386,7 +410,7 @@ __global__ void init_lane_kernel(const void* __restrict__ W, int64_t n_groups, i
     };
     auto X = [&](int i) -> float& { return xs[i * 32 + lane]; };
     auto C = [&](int i) -> uint8_t& { return cs[i * 32 + lane]; };
-    auto Y = [&](int i) -> double& { return yd[i * 32 + lane]; };
+    auto BX = [&](int c) -> double& { return bx[c * 32 + lane]; };
 
     float wmin = INFINITY, wmax = -INFINITY;
 #pragma unroll 2
@@ -435,42 +459,48 @@ __global__ void init_lane_kernel(const void* __restrict__ W, int64_t n_groups, i
             }
             a[j] = (float)(sabs / (double)G_);
         }
+        // Per code word c: the fp64 sum of x over the group's elements with
+        // code c (bx) and their count (hist).  Then C^T (x - z_B) =
+        // sum_c s(c) (bx_c - n_c z_B) and C^T C = sum_c n_c s(c) s(c)^T, where
+        // s(c) is the sign vector of c; a round only moves the elements whose
+        // code changed from one sum to the other.
+        CodeHist<L> hist;
+#pragma unroll
+        for (int c = 0; c < L; ++c) BX(c) = 0.0;
 #pragma unroll 2
-        for (int i = 0; i < G_; ++i) Y(i) = (double)X(i) - (double)zb;
+        for (int i = 0; i < G_; ++i) {
+            const int c = C(i);
+            BX(c) += (double)X(i);
+            hist.add(c, 1);
+        }
 
         // --- T rounds of alpha, C (and z_B when G == 1) ---
         for (int it = 0; it < T; ++it) {
             long long ctc[Q][Q];
             double cty[Q];
-            // off-diagonal entries of C^T C from counts of differing bits:
-            // sum_i c_ij c_ik = g - 2 #{i: bit j != bit k}; the diagonal is g
-            uint32_t diff[Q][Q];
 #pragma unroll
             for (int j = 0; j < Q; ++j) {
                 cty[j] = 0.0;
 #pragma unroll
-                for (int k = 0; k < Q; ++k) diff[j][k] = 0u;
+                for (int k = 0; k < Q; ++k) ctc[j][k] = 0;
             }
-#pragma unroll 2
-            for (int i = 0; i < G_; ++i) {
-                const uint32_t c = C(i);
-                const double y = Y(i);
+            const double zbd = (double)zb;
+#pragma unroll
+            for (int c = 0; c < L; ++c) {
+                const int n = hist.get(c);
+                const double yc = BX(c) - (double)n * zbd;
 #pragma unroll
                 for (int j = 0; j < Q; ++j) {
-                    cty[j] += ((c >> j) & 1) ? y : -y;
+                    const bool sj = (c >> j) & 1;
+                    cty[j] += sj ? yc : -yc;
 #pragma unroll
-                    for (int k = j + 1; k < Q; ++k) diff[j][k] += ((c >> j) ^ (c >> k)) & 1u;
+                    for (int k = j; k < Q; ++k) ctc[j][k] += (sj == (bool)((c >> k) & 1)) ? n : -n;
                 }
             }
 #pragma unroll
-            for (int j = 0; j < Q; ++j) {
-                ctc[j][j] = G_;
+            for (int j = 0; j < Q; ++j)
 #pragma unroll
-                for (int k = j + 1; k < Q; ++k) {
-                    ctc[j][k] = (long long)G_ - 2 * (long long)diff[j][k];
-                    ctc[k][j] = ctc[j][k];
-                }
-            }
+                for (int k = 0; k < j; ++k) ctc[j][k] = ctc[k][j];
             if (!int_singular<Q>(ctc)) {
                 double sol[Q];
                 solve_fp64<Q>(ctc, cty, sol);
@@ -482,25 +512,32 @@ __global__ void init_lane_kernel(const void* __restrict__ W, int64_t n_groups, i
 #pragma unroll 2
             for (int i = 0; i < G_; ++i) {
                 float m;
-                const int r = nearest_rank<L>(X(i), srt, m);
-                const uint8_t c = (uint8_t)((cor >> (4 * r)) & 15u);
-                moved |= c != C(i);
-                C(i) = c;
+                const float x = X(i);
+                const int r = nearest_rank<L>(x, srt, m);
+                const int c = (int)((cor >> (4 * r)) & 15u);
+                const int old = C(i);
+                if (c != old) {
+                    moved = true;
+                    const double xd = (double)x;
+                    BX(old) -= xd;
+                    BX(c) += xd;
+                    hist.add(old, -1);
+                    hist.add(c, 1);
+                    C(i) = (uint8_t)c;
+                }
             }
             const float zb_prev = zb;
             if (G == 1) {
+                // z_B = mean of x - C alpha = sum_c (bx_c - n_c (s(c) . alpha)) / g
                 double sres = 0.0;
-#pragma unroll 2
-                for (int i = 0; i < G_; ++i) {
-                    const int c = C(i);
+#pragma unroll
+                for (int c = 0; c < L; ++c) {
                     double ca = 0.0;
 #pragma unroll
                     for (int j = 0; j < Q; ++j) ca += ((c >> j) & 1) ? (double)a[j] : -(double)a[j];
-                    sres += (double)X(i) - ca;
+                    sres += BX(c) - (double)hist.get(c) * ca;
                 }
                 zb = (float)(sres / (double)G_);
-#pragma unroll 2
-                for (int i = 0; i < G_; ++i) Y(i) = (double)X(i) - (double)zb;
             }
             // No code moved (and z_B did not either): the next round would
             // solve the same system, get the same alpha and the same codes, so
@@ -551,7 +588,7 @@ template <int Q, typename WT, int G_>
 static cudaError_t run_init_lane(const Shape& sh, const void* W, int G, int T, int clip, uq_params p,
                                  uint8_t* codes, cudaStream_t st) {
     constexpr int L = 1 << Q;
-    constexpr size_t warp_bytes = (((size_t)G_ * 32 * 13 + (size_t)L * 32 * 5) + 15) & ~size_t(15);
+    constexpr size_t warp_bytes = init_lane_warp_bytes(Q, G_);
     // as many warps as fit in the 227 KB a block may opt in to, at most 16
     constexpr int wpb = (int)((227 * 1024) / warp_bytes) > 16 ? 16 : (int)((227 * 1024) / warp_bytes);
     static_assert(wpb >= 1, "one warp's tables must fit");
