@@ -343,6 +343,51 @@ def time_gemv(q, g, dev, stream, peak, shapes=((14336, 4096), (8192, 28672)), re
     return res
 
 
+def time_link(hp, hin, hout, reps=3):
+    """The copy ceiling of the end-to-end number, measured in this process:
+    the same pinned host buffers copied to the device alone, back alone, and
+    both directions at once (CUDA events on the copy streams), in GB/s, and
+    the weights/s those copies alone would allow."""
+    import torch
+    from paper_2506_03781_gb300 import api
+    hs = hp.steps[0]
+    dev = {**hs.dev, **hs.params}
+    up_b, down_b = hp.bytes_in(hin), hp.bytes_out(hout)
+
+    def h2d():
+        with torch.cuda.stream(hp.up):
+            for name in api.HostStep.IN_KEYS:
+                dev[name].copy_(hin[name], non_blocking=True)
+
+    def d2h():
+        with torch.cuda.stream(hp.down):
+            hout["W_hat"].copy_(hs.dev["W_hat"], non_blocking=True)
+            hout["codes"].copy_(hs.dev["codes"], non_blocking=True)
+            for name in api.GRAD_NAMES:
+                hout[name].copy_(hs.grads[name], non_blocking=True)
+
+    def timed(fns):
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(torch.cuda.current_stream())
+        for st in (hp.up, hp.down):
+            st.wait_event(e0)
+        for _ in range(reps):
+            for f in fns:
+                f()
+        for st in (hp.up, hp.down):
+            torch.cuda.current_stream().wait_stream(st)
+        e1.record(torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / 1e3 / reps
+
+    t_up, t_down, t_both = timed([h2d]), timed([d2h]), timed([h2d, d2h])
+    return {"h2d_gbs": up_b / t_up / 1e9, "d2h_gbs": down_b / t_down / 1e9,
+            "duplex_ms_per_step": t_both * 1e3,
+            "copy_ceiling_weights_per_s": hs.out * hs.n_in / t_both}
+
+
 def time_block_step(dev, steps=20, warmup=3, samples=4):
     """Algorithm 1 on a Llama-3-8B-shaped block (seq 2048, bf16 block
     compute, the block workload's q and g): ms per optimisation step (block
@@ -621,6 +666,7 @@ def run_gpu(args):
     e2e_ms = e0.elapsed_time(e1)
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
     e2e_value = weak_scaling_value(N, e2e_steps, world, e2e_ms / 1e3)
+    link = time_link(hp, hin, hout)
 
     # bit-width sweep of the same matrix (the workload is specified for q in {2, 3, 4})
     sweep = {}
@@ -676,7 +722,7 @@ def run_gpu(args):
             },
             "e2e": {"value": e2e_value, "unit": "weights/s",
                     "h2d_bytes_per_step": hp.bytes_in(hin), "d2h_bytes_per_step": hp.bytes_out(hout),
-                    "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps,
+                    "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps, "link": link,
                     "api": "paper_2506_03781_gb300.api.HostPipeline (pinned host buffers, uploads/compute/"
                            "downloads of consecutive steps overlapped)"},
             "train_step": train,
