@@ -388,7 +388,7 @@ def time_link(hp, hin, hout, reps=3):
             "copy_ceiling_weights_per_s": hs.out * hs.n_in / t_both}
 
 
-def time_block_step(dev, steps=20, warmup=3, samples=4):
+def time_block_step(dev, steps=20, warmup=4, samples=4):
     """Algorithm 1 on a Llama-3-8B-shaped block (seq 2048, bf16 block
     compute, the block workload's q and g): ms per optimisation step (block
     forward + backward in torch, then uq_train_step for the seven weights),
@@ -445,7 +445,10 @@ def time_block_step(dev, steps=20, warmup=3, samples=4):
     res = {"block": shape.name, "seq": shape.seq, "q": wl.q, "g": wl.g, "weights": n_w, "steps": steps,
            "ms_per_step": ms, "quantizer_ms_per_step": qms, "quantizer_share": qms / ms,
            "codes_moved_per_remap_step": statistics.mean(moved) if moved else None,
-           "loss_first": float(losses[0]), "loss_last": float(losses[-1]), "init_s": init_s,
+           # mean loss of each epoch (one pass over the samples, from the first step on)
+           "loss_per_epoch": [float(torch.stack(losses[k:k + samples]).mean())
+                              for k in range(0, len(losses) - samples + 1, samples)],
+           "init_s": init_s,
            "paper_step_s_a100_derived": 0.25}
     del rec, Y, Xd, Xhd
     torch.cuda.empty_cache()
