@@ -159,11 +159,11 @@ def cpu_cores():
 # CPU oracle timing (the cpu_baseline / --impl reference legs)
 # ---------------------------------------------------------------------------
 
-def oracle_sample_inputs(wl, q, rows):
-    """Oracle-initialised inputs of the first ``rows`` rows of the workload."""
+def oracle_sample_inputs(wl, q, rows, row0=0):
+    """Oracle-initialised inputs of rows row0 .. row0 + rows of the workload."""
     import oracle as O
     from paper_2506_03781_gb300 import synth
-    _, W = synth.workload_weights(wl, 0, slice(0, rows))
+    _, W = synth.workload_weights(wl, 0, slice(row0, row0 + rows))
     g = wl.g
     init = O.unified_init(W, q, g, G=2, T=2)
     P = {k: init[k] for k in ("delta", "zu", "s", "sr", "alpha", "zb")}
@@ -172,12 +172,15 @@ def oracle_sample_inputs(wl, q, rows):
     return W, P, init["codes"], Gup
 
 
-def time_oracle_step(wl, q, rows, budget_s):
+def time_oracle_step(wl, q, rows, budget_s, row0=0, barrier=None):
     """Runs oracle steps (fwd at step t + bwd) until budget_s elapses; returns
-    (weights per second, steps run, seconds)."""
+    (weights per second, steps run, seconds).  With a barrier, the timed loop
+    starts once every party has prepared its inputs."""
     import oracle as O
-    W, P, codes, Gup = oracle_sample_inputs(wl, q, rows)
+    W, P, codes, Gup = oracle_sample_inputs(wl, q, rows, row0)
     g = wl.g
+    if barrier is not None:
+        barrier.wait()
     t0 = time.perf_counter()
     n = 0
     while True:
@@ -189,6 +192,56 @@ def time_oracle_step(wl, q, rows, budget_s):
         if el >= budget_s and n >= 2:
             break
     return W.size * n / el, n, el
+
+
+def _oracle_shard(wl_name, q, row0, rows, budget_s, barrier, results):
+    """One process of the row-parallel oracle timing (spawned; no CUDA)."""
+    from paper_2506_03781_gb300 import synth
+    wl = synth.WORKLOADS[wl_name]
+    _, n, el = time_oracle_step(wl, q, rows, budget_s, row0, barrier)
+    results.put((rows * wl.matrices[0].n_in * n, el))
+
+
+def time_oracle_parallel(wl, q, rows, budget_s, workers):
+    """The same oracle steps on `workers` row shards at once, one process
+    each (rows are independent): every process prepares its shard, waits at
+    a barrier, then runs budget_s seconds.  Returns (aggregate weights per
+    second, the longest process's seconds).  Spawned processes, one numpy
+    thread each."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    barrier, results = ctx.Barrier(workers), ctx.Queue()
+    saved = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+    os.environ.update({k: "1" for k in saved})
+    import queue
+    procs, out = [], []
+    try:
+        procs = [ctx.Process(target=_oracle_shard, args=(wl.name, q, k * rows, rows, budget_s, barrier, results))
+                 for k in range(workers)]
+        for pr in procs:
+            pr.start()
+        deadline = time.perf_counter() + 10 * budget_s + 300
+        while len(out) < workers and time.perf_counter() < deadline:
+            try:
+                out.append(results.get(timeout=5))
+            except queue.Empty:
+                if any(pr.exitcode not in (None, 0) for pr in procs):
+                    break                               # a worker failed: no all-core figure
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+        for pr in procs:
+            pr.join(timeout=5)
+            if pr.is_alive():
+                pr.kill()                               # this call's own child process
+                pr.join()
+    if len(out) < workers:
+        return None, None
+    el = max(o[1] for o in out)
+    return sum(o[0] for o in out) / el, el
 
 
 # ---------------------------------------------------------------------------
@@ -683,13 +736,19 @@ def run_gpu(args):
 
     result = None
     if rank == 0:
-        cpu = None
+        cpu = cpu_all = None
         if world == 1 and not args.no_cpu_baseline:
             rows = 96
             v, n, el = time_oracle_step(wl, q, rows, args.cpu_budget)
             cpu = {"value": v, "unit": "weights/s", "cores": 1, "kind": "oracle",
                    "sample": f"first {rows} rows of {out}x{n_in} ({rows * n_in} weights), {n} oracle steps "
                              f"(local remap/keep alternating + backward) in {el:.1f} s, numpy single thread"}
+            workers = max(1, min(cpu_cores(), out // rows))
+            vp, elp = time_oracle_parallel(wl, q, rows, args.cpu_budget, workers)
+            if vp is not None:
+                cpu_all = {"value": vp, "unit": "weights/s", "cores": workers, "kind": "oracle",
+                           "sample": f"{workers} processes, each on its own {rows}-row shard of {out}x{n_in}, the "
+                                     f"same oracle steps for {elp:.1f} s (row-parallel, one numpy thread each)"}
         result = {
             "metric": METRIC,
             "value": value,
@@ -736,6 +795,7 @@ def run_gpu(args):
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,
             "cpu_baseline": cpu,
+            "cpu_baseline_all_cores": cpu_all,
         }
         print(json.dumps(result))
     if world > 1:
