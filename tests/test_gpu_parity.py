@@ -77,7 +77,7 @@ def test_export(q, g, mode):
 
 @pytest.mark.parametrize("clip", [api.CLIP_FIXED_MIN, api.CLIP_FIXED_MAX, api.CLIP_BALANCED])
 @pytest.mark.parametrize("G,T", [(1, 15), (7, 5)])
-@pytest.mark.parametrize("g", [32, 128, 256])
+@pytest.mark.parametrize("g", [32, 64, 128, 256])
 @pytest.mark.parametrize("q", QS)
 def test_init(q, g, G, T, clip):
     out, n_in = 9, g * 6
