@@ -11,9 +11,12 @@
 // accumulates ds_A of its columns over its rows in registers; the range's
 // partials go to a workspace [row range][in] and a second kernel sums them in
 // range order.  Deterministic, no atomics.  HBM traffic per element (bf16 W):
-// forward remap 2 + 1 read, 4 + 1 written; backward 2 + 1 + 4 read.
+// forward remap 2 + 1 read, 4 + 1 written; backward 2 + 1 + 4 read.  The
+// forward steps that map run on the pipelined skeleton instead (below) for
+// g in {32, 64, 128} and rows of whole work units.
 #include "uq_common.cuh"
 #include "uq_launch.h"
+#include "uq_pipe.cuh"
 
 namespace uq {
 
@@ -227,6 +230,219 @@ awq_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const f
             *reinterpret_cast<float4*>(prow + 4 * LPG * v) = make_float4(dsa[v][0], dsa[v][1], dsa[v][2], dsa[v][3]);
 }
 
+// ---------------------------------------------------------------------------
+// Pipelined forward (g in {32, 64, 128}, rows of whole work units)
+// ---------------------------------------------------------------------------
+//
+// The persistent TMA-pipelined skeleton of uq_pipe.cuh: every warp streams
+// its (row block, unit) items through a ring of shared-memory stages, with
+// bounded mbarrier waits (a wait that runs out sets g_awq_err, reported by
+// uq_check_device).  A stage holds the weights (not on keep steps), s_A of
+// the unit's columns in the s slot (the same for every row, so it comes from
+// L2 after the first rows), the code words (not for the full mapping) and
+// Delta_A, z_A, z_B, alpha in the Delta, z_U, z_B, alpha slots.  Only the
+// steps that map (remap, full) use it.
+
+__device__ unsigned int g_awq_err = 0;
+
+#ifndef UQ_AWQ_FWD_STAGE_BYTES
+#define UQ_AWQ_FWD_STAGE_BYTES 5632
+#endif
+
+template <int Q, typename WT, int G_, int MODE>
+using AwqFwdStage = Stage<Q, WT, G_, MODE != FWD_KEEP, false, MODE != FWD_FULL, UQ_AWQ_FWD_STAGE_BYTES, true>;
+
+template <typename St, int KIND>
+struct AwqTag {};
+
+template <int Q, typename St>
+__device__ __forceinline__ void awq_issue(const Items& it, const Cursor& c, int s, uint32_t bar, unsigned char* wsm,
+                                          const void* W, const float* SA, const uint8_t* CODES, const float* DELTA,
+                                          const float* ZA, const float* ZB, const float* ALPHA, int64_t out, int n_in,
+                                          int Gr) {
+    const int64_t row = it.row(c.k);
+    if (row >= out) { tma::bar_arrive(bar); return; }
+    const int64_t col0 = (int64_t)it.unit(c.j) * St::UE;
+    const int64_t e0 = row * n_in + col0;
+    const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * St::NG;
+    const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+    tma::fence_async_smem();
+    tma::bar_arrive_tx(bar, St::TX);
+    if constexpr (St::SZ_W > 0)
+        tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
+    tma::copy_g2s(d + St::OFF_S, SA + col0, St::SZ_S, bar);
+    if constexpr (St::SZ_C > 0) tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+    tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_Z, ZA + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+}
+
+template <int Q, typename WT, int G_, int MODE>
+__global__ void __launch_bounds__(kThreads, 3)
+awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const float* __restrict__ DELTA,
+                      const float* __restrict__ ZA, const float* __restrict__ ALPHA, const float* __restrict__ ZB,
+                      uint8_t* __restrict__ CODES, float* __restrict__ WHAT, int64_t out, int n_in, int R, int n_rb) {
+    using St = AwqFwdStage<Q, WT, G_, MODE>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) unsigned long long bars[kWarps][NST];
+    __shared__ MapTab<Q, NG> tabs[kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sub = lane / LPG, li = lane % LPG;
+    const int U = n_in / UE, Gr = n_in / G_;
+    const Items it(U, R, n_rb, warp);
+    unsigned char* wsm = smem + (size_t)warp * St::WARP_BYTES;
+    MapTab<Q, NG>& t = tabs[warp];
+
+    if (lane == 0) {
+        for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+    Cursor ic;
+    long long issued = 0;
+    if (lane == 0) {
+        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+            awq_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, CODES, DELTA, ZA, ZB, ALPHA, out,
+                             n_in, Gr);
+            ic.next(it.n_w);
+        }
+    }
+    Ring<NST> ring;
+    Cursor cc;
+    for (long long i = 0; i < it.total; ++i) {
+        const int s = ring.s;
+        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
+            if (lane == 0) {
+                atomicOr(&g_awq_err, 1u);
+                drain(bars[warp], i, issued);
+            }
+            return;                                      // no block barrier in this kernel
+        }
+        const int64_t row = it.row(cc.k);
+        if (row < out) {
+            const unsigned char* st = wsm + (size_t)s * St::BYTES;
+            const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
+            const float* pz = reinterpret_cast<const float*>(st + St::OFF_Z);
+            const float* pb = reinterpret_cast<const float*>(st + St::OFF_B);
+            const float* pa = reinterpret_cast<const float*>(st + St::OFF_A);
+#pragma unroll
+            for (int e = lane; e < NG * L; e += 32) {
+                const int kk = e / L, c = e % L;
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
+                t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+            }
+            __syncwarp();
+            if constexpr (MODE == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
+            else if constexpr (MODE == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            const float dl = pd[sub], za = pz[sub];
+            const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
+            float srt[L];
+            if constexpr (MODE == FWD_FULL) {
+#pragma unroll
+                for (int r = 0; r < L; ++r) srt[r] = t.srt[sub][r];
+            }
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                const int el = sub * G_ + 4 * li + 4 * LPG * v;
+                float s4[4], w[4];
+                f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
+                if constexpr (MODE != FWD_KEEP)
+                    WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
+                uint32_t cv = 0u;
+                if constexpr (MODE != FWD_FULL) cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+                float o[4];
+                uint32_t nc = 0;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    float m;
+                    uint32_t code;
+                    if constexpr (MODE == FWD_KEEP) {
+                        code = (cv >> (8 * k)) & (L - 1);
+                        m = t.lv[sub][code];
+                    } else {
+                        const float x = __fadd_rn(__fdiv_rn(__fmul_rn(w[k], s4[k]), dl), za);
+                        if constexpr (MODE == FWD_REMAP) {
+                            const int c = (cv >> (8 * k)) & (L - 1);
+                            const float4 nb = t.nb[sub][c];
+                            const uint32_t packed = __float_as_uint(nb.w);
+                            float best = fabsf(__fsub_rn(x, nb.y));
+                            m = nb.y;
+                            code = c;
+                            const float dlo = fabsf(__fsub_rn(x, nb.x));
+                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
+                            const float dhi = fabsf(__fsub_rn(x, nb.z));
+                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                        } else {
+                            const int r = nearest_rank<L>(x, srt, m);
+                            code = t.cor[sub][r];
+                        }
+                    }
+                    o[k] = __fdiv_rn(__fmul_rn(dl, __fsub_rn(m, za)), s4[k]);
+                    nc |= code << (8 * k);
+                }
+                if constexpr (MODE != FWD_KEEP) *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
+                *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
+            }
+        }
+        __syncwarp();
+        if (lane == 0 && issued < it.total) {
+            awq_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, CODES, DELTA, ZA, ZB, ALPHA, out,
+                             n_in, Gr);
+            ic.next(it.n_w);
+            ++issued;
+        }
+        ring.next();
+        cc.next(it.n_w);
+    }
+}
+
+template <int Q, typename WT, int G_, int MODE>
+static cudaError_t run_awq_stream_fwd(const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes, float* what,
+                                      cudaStream_t st) {
+    using St = AwqFwdStage<Q, WT, G_, MODE>;
+    const int U = sh.n_in / St::UE;
+    const int R = rows_per_block(U);
+    const int n_rb = (int)((sh.out + R - 1) / R);
+    const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
+    auto kern = awq_stream_fwd_kernel<Q, WT, G_, MODE>;
+    int grid = 0;
+    cudaError_t e = grid_for<AwqTag<St, MODE>>(kern, dyn, n_rb, grid);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, dyn, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R, n_rb);
+    return cudaGetLastError();
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t awq_stream_fwd_g(int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                                    float* what, cudaStream_t st) {
+    if (mode == FWD_REMAP) return run_awq_stream_fwd<Q, WT, G_, FWD_REMAP>(sh, W, p, codes, what, st);
+    return run_awq_stream_fwd<Q, WT, G_, FWD_FULL>(sh, W, p, codes, what, st);
+}
+
+template <int Q, typename WT>
+static cudaError_t awq_stream_fwd(int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
+                                  float* what, cudaStream_t st) {
+    if (sh.g == 32) return awq_stream_fwd_g<Q, WT, 32>(mode, sh, W, p, codes, what, st);
+    if (sh.g == 64) return awq_stream_fwd_g<Q, WT, 64>(mode, sh, W, p, codes, what, st);
+    return awq_stream_fwd_g<Q, WT, 128>(mode, sh, W, p, codes, what, st);
+}
+
+cudaError_t awq_error(bool clear, unsigned int* flag) {
+    unsigned int v = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_awq_err, sizeof(v));
+    if (e != cudaSuccess) return e;
+    *flag = v;
+    if (clear && v != 0) {
+        const unsigned int z = 0;
+        e = cudaMemcpyToSymbol(g_awq_err, &z, sizeof(z));
+    }
+    return e;
+}
+
 // ds_A[col] = sum over the row ranges of PART[range, col], in range order.
 __global__ void __launch_bounds__(256)
 awq_colsum_kernel(const float* __restrict__ PART, float* __restrict__ DSA, int n_in, int ranges) {
@@ -302,6 +518,13 @@ static cudaError_t awq_g(bool bwd, int mode, const Shape& sh, const void* W, uq_
 template <int Q>
 static cudaError_t awq_w(bool bwd, int mode, const Shape& sh, const void* W, uq_params_awq p, uint8_t* codes,
                          float* what, const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    // Steps that map (remap, full) take the pipelined kernel on its shapes; the
+    // keep step reads no weights, and the register kernel, which holds s_A
+    // across a warp's rows, beats restaging s_A for every unit.
+    if (!bwd && mode != FWD_KEEP && stream_path_ok(sh)) {
+        if (sh.wdtype == UQ_W_BF16) return awq_stream_fwd<Q, WBF16>(mode, sh, W, p, codes, what, st);
+        return awq_stream_fwd<Q, WF32>(mode, sh, W, p, codes, what, st);
+    }
     if (sh.wdtype == UQ_W_BF16) return awq_g<Q, WBF16>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
     return awq_g<Q, WF32>(bwd, mode, sh, W, p, codes, what, gup, gr, work, st);
 }

@@ -62,6 +62,7 @@ cudaError_t launch_omni_bwd(const Shape& sh, const void* W, uq_params_omni p, co
                             uq_grads_omni gr, cudaStream_t st);
 // Reads (and optionally clears) the OmniQuant-map kernels' bounded-wait flag.
 cudaError_t omni_error(bool clear, unsigned int* flag);
+cudaError_t awq_error(bool clear, unsigned int* flag);
 cudaError_t launch_omni_scales(const Shape& sh, const void* W, const float* beta, const float* gamma, float* delta,
                                float* zo, cudaStream_t st);
 // UniQuan with AWQ's maps (uq_awq.cu); awq_ok: the group sizes it takes;
