@@ -431,6 +431,223 @@ static cudaError_t awq_stream_fwd(int mode, const Shape& sh, const void* W, uq_p
     return awq_stream_fwd_g<Q, WT, 128>(mode, sh, W, p, codes, what, st);
 }
 
+// ---------------------------------------------------------------------------
+// Pipelined backward (rows of at most kWarps work units)
+// ---------------------------------------------------------------------------
+//
+// ds_A sums down each column.  When a row holds at most kWarps work units,
+// every warp of a block owns one fixed unit (one set of columns) for the
+// whole kernel, so its ds_A partials and 1/s_A stay in registers across all
+// of its rows; at the end each (block, row slot) writes one row of partials
+// to the workspace [grid * R][in], summed in that order by awq_colsum_kernel.
+// Deterministic for a given grid.  The stage holds W, s_A of the unit's
+// columns (s slot), dL/dW^, the codes and Delta_A, z_A, z_B, alpha.
+
+constexpr int kAwqStreamBwdBlocksPerSm = 2;
+#ifndef UQ_AWQ_BWD_STAGE_BYTES
+#define UQ_AWQ_BWD_STAGE_BYTES 11520
+#endif
+
+template <int Q, typename WT, int G_>
+using AwqBwdStage = Stage<Q, WT, G_, true, true, true, UQ_AWQ_BWD_STAGE_BYTES, true>;
+
+static bool awq_stream_bwd_ok(const Shape& sh) {
+    if (!stream_path_ok(sh)) return false;
+    return sh.n_in / (sh.g == 32 ? 256 : 512) <= kWarps;
+}
+
+// Rows per block, row blocks and the grid of the pipelined backward (the
+// grid is bounded by the SM count only, so the workspace size is known).
+static void awq_stream_bwd_grid(const Shape& sh, int& R, int& n_rb, int& grid) {
+    const int U = sh.n_in / (sh.g == 32 ? 256 : 512);
+    R = rows_per_block(U);
+    n_rb = (int)((sh.out + R - 1) / R);
+    const int cap = sm_count() * kAwqStreamBwdBlocksPerSm;
+    grid = n_rb < cap ? n_rb : cap;
+}
+
+template <int Q, typename St>
+__device__ __forceinline__ void awq_bwd_issue(const Items& it, const Cursor& c, int s, uint32_t bar,
+                                              unsigned char* wsm, const void* W, const float* SA, const float* GUP,
+                                              const uint8_t* CODES, const float* DELTA, const float* ZA,
+                                              const float* ZB, const float* ALPHA, int64_t out, int n_in, int Gr) {
+    const int64_t row = it.row(c.k);
+    if (row >= out) { tma::bar_arrive(bar); return; }
+    const int64_t col0 = (int64_t)it.unit(c.j) * St::UE;
+    const int64_t e0 = row * n_in + col0;
+    const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * St::NG;
+    const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+    tma::fence_async_smem();
+    tma::bar_arrive_tx(bar, St::TX);
+    tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
+    tma::copy_g2s(d + St::OFF_S, SA + col0, St::SZ_S, bar);
+    tma::copy_g2s(d + St::OFF_G, GUP + e0, St::SZ_G, bar);
+    tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+    tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_Z, ZA + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
+    tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+}
+
+template <int Q, typename WT, int G_>
+__global__ void __launch_bounds__(kThreads, kAwqStreamBwdBlocksPerSm)
+awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, const float* __restrict__ DELTA,
+                      const float* __restrict__ ZA, const float* __restrict__ ALPHA, const float* __restrict__ ZB,
+                      const uint8_t* __restrict__ CODES, const float* __restrict__ GUP, float* __restrict__ DDELTA,
+                      float* __restrict__ DZA, float* __restrict__ DALPHA, float* __restrict__ DZB,
+                      float* __restrict__ PART, int64_t out, int n_in, int R, int n_rb) {
+    using St = AwqBwdStage<Q, WT, G_>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
+    using SR8 = SegReduce<LPG>;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) unsigned long long bars[kWarps][NST];
+    __shared__ float2 tabs[kWarps][NG][L];          // (l(c), l(c) - z_A) per group slot and code word
+    __shared__ float tau_s[kWarps][NG];
+    __shared__ float eg_s[kWarps][NG];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sub = lane / LPG, li = lane % LPG;
+    const int U = n_in / UE, Gr = n_in / G_;
+    const Items it(U, R, n_rb, warp);               // n_w <= 1: the warp's unit is it.unit(0)
+    unsigned char* wsm = smem + (size_t)warp * St::WARP_BYTES;
+
+    if (lane == 0) {
+        for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+    Cursor ic;
+    long long issued = 0;
+    if (lane == 0) {
+        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+            awq_bwd_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, GUP, CODES, DELTA, ZA, ZB,
+                                 ALPHA, out, n_in, Gr);
+            ic.next(it.n_w);
+        }
+    }
+    float rs[NV][4], dsa[NV][4];
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) { rs[v][k] = 0.f; dsa[v][k] = 0.f; }
+    bool have_rs = false;
+    Ring<NST> ring;
+    Cursor cc;
+    for (long long i = 0; i < it.total; ++i) {
+        const int s = ring.s;
+        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
+            if (lane == 0) {
+                atomicOr(&g_awq_err, 2u);
+                drain(bars[warp], i, issued);
+            }
+            return;                                      // no block barrier in this kernel
+        }
+        const int64_t row = it.row(cc.k);
+        if (row < out) {
+            const unsigned char* st = wsm + (size_t)s * St::BYTES;
+            const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
+            const float* pz = reinterpret_cast<const float*>(st + St::OFF_Z);
+            const float* pb = reinterpret_cast<const float*>(st + St::OFF_B);
+            const float* pa = reinterpret_cast<const float*>(st + St::OFF_A);
+            if (!have_rs) {                              // 1/s_A of the warp's columns, once
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    float s4[4];
+                    f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + (sub * G_ + 4 * li + 4 * LPG * v) * 4), s4);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) rs[v][k] = __fdiv_rn(1.f, s4[k]);
+                }
+                have_rs = true;
+            }
+#pragma unroll
+            for (int e = lane; e < NG * L; e += 32) {
+                const int kk = e / L, c = e % L;
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
+                const float lvc = level_of<Q>(c, a, pb[kk]);
+                tabs[warp][kk][c] = make_float2(lvc, lvc - pz[kk]);
+                if (c == 0) {
+                    float m = fabsf(a[0]);
+#pragma unroll
+                    for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
+                    tau_s[warp][kk] = m;
+                    eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, pd[kk]);
+                }
+            }
+            __syncwarp();
+            const float dl = pd[sub], za = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+            const float rdl = rcp_approx(dl);
+            float acc[8];
+#pragma unroll
+            for (int q8 = 0; q8 < 8; ++q8) acc[q8] = 0.f;
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                const int el = sub * G_ + 4 * li + 4 * LPG * v;
+                float w[4], s4[4], G[4], ws[4], m4[4], uv[4];
+                float2 mm[4];
+                bool fv[4];
+                WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
+                f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
+                f4_to(*reinterpret_cast<const float4*>(st + St::OFF_G + el * 4), G);
+                const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    ws[k] = __fmul_rn(w[k], s4[k]);
+                    mm[k] = tabs[warp][sub][(cv >> (8 * k)) & (L - 1)];
+                    m4[k] = mm[k].x;
+                }
+                shared_div_filter4(ws, dl, rdl, za, m4, tau, eg, uv, fv);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int c = (cv >> (8 * k)) & (L - 1);
+                    const bool f = fv[k];
+                    const float gs = G[k] * rs[v][k];
+                    const float mz = mm[k].y;
+                    acc[0] += gs * (mz - (f ? uv[k] : 0.f));
+                    acc[1] += f ? 0.f : gs;
+                    acc[2] += gs;
+#pragma unroll
+                    for (int j = 0; j < Q; ++j)                  // P_j: dalpha_j = Delta (2 P_j - S)
+                        if ((c >> j) & 1) acc[4 + j] += gs;
+                    dsa[v][k] += gs * ((f ? w[k] : 0.f) - dl * mz * rs[v][k]);
+                }
+            }
+            const int slot0 = SR8::run(acc, lane);
+            const float S = seg_slot2<LPG>(acc, lane);
+            if (SR8::writer(lane)) {
+                const int64_t grp = row * Gr + (int64_t)it.unit(cc.j) * NG + sub;
+#pragma unroll
+                for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
+                    const int slot = slot0 + q8;
+                    const float tot = acc[q8];
+                    if (slot == 0) DDELTA[grp] = tot;
+                    else if (slot == 1) DZA[grp] = -(dl * tot);
+                    else if (slot == 2) DZB[grp] = dl * tot;
+                    else if (slot >= 4 && slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * __fmaf_rn(2.f, tot, -S);
+                }
+            }
+        }
+        __syncwarp();                                    // stage and tables are free again
+        if (lane == 0 && issued < it.total) {
+            awq_bwd_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, GUP, CODES, DELTA, ZA, ZB,
+                                 ALPHA, out, n_in, Gr);
+            ic.next(it.n_w);
+            ++issued;
+        }
+        ring.next();
+        cc.next(it.n_w);
+    }
+    // this (block, row slot)'s ds_A partials of the warp's columns (zeros if it had no row)
+    if (it.n_w > 0) {
+        float* prow = PART + ((int64_t)blockIdx.x * R + it.row_sub) * n_in + (int64_t)it.unit(0) * UE;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int el = sub * G_ + 4 * li + 4 * LPG * v;
+            *reinterpret_cast<float4*>(prow + el) = make_float4(dsa[v][0], dsa[v][1], dsa[v][2], dsa[v][3]);
+        }
+    }
+}
+
 cudaError_t awq_error(bool clear, unsigned int* flag) {
     unsigned int v = 0;
     cudaError_t e = cudaMemcpyFromSymbol(&v, g_awq_err, sizeof(v));
@@ -469,10 +686,41 @@ static void awq_grid(const Shape& sh, int lpg, unsigned& col_blocks, int64_t& ra
 }
 
 int64_t awq_workspace_floats(const Shape& sh) {
+    if (awq_stream_bwd_ok(sh)) {
+        int R, n_rb, grid;
+        awq_stream_bwd_grid(sh, R, n_rb, grid);
+        return (int64_t)grid * R * sh.n_in;
+    }
     unsigned cb;
     int64_t ranges, rpr;
     awq_grid(sh, lanes_per_group(sh.g), cb, ranges, rpr);
     return ranges * (int64_t)sh.n_in;
+}
+
+template <int Q, typename WT, int G_>
+static cudaError_t run_awq_stream_bwd(const Shape& sh, const void* W, uq_params_awq p, const uint8_t* codes,
+                                      const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    using St = AwqBwdStage<Q, WT, G_>;
+    int R, n_rb, grid, unused = 0;
+    awq_stream_bwd_grid(sh, R, n_rb, grid);
+    const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
+    auto kern = awq_stream_bwd_kernel<Q, WT, G_>;
+    cudaError_t e = grid_for<AwqTag<St, 9>>(kern, dyn, n_rb, unused);    // shared-memory attribute (once)
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, dyn, st>>>(W, p.sa, p.delta, p.za, p.alpha, p.zb, codes, gup, gr.ddelta, gr.dza,
+                                      gr.dalpha, gr.dzb, work, sh.out, sh.n_in, R, n_rb);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    awq_colsum_kernel<<<(sh.n_in + 255) / 256, 256, 0, st>>>(work, gr.dsa, sh.n_in, grid * R);
+    return cudaGetLastError();
+}
+
+template <int Q, typename WT>
+static cudaError_t awq_stream_bwd(const Shape& sh, const void* W, uq_params_awq p, const uint8_t* codes,
+                                  const float* gup, uq_grads_awq gr, float* work, cudaStream_t st) {
+    if (sh.g == 32) return run_awq_stream_bwd<Q, WT, 32>(sh, W, p, codes, gup, gr, work, st);
+    if (sh.g == 64) return run_awq_stream_bwd<Q, WT, 64>(sh, W, p, codes, gup, gr, work, st);
+    return run_awq_stream_bwd<Q, WT, 128>(sh, W, p, codes, gup, gr, work, st);
 }
 
 template <int Q, typename WT, int LPG>
@@ -521,6 +769,10 @@ static cudaError_t awq_w(bool bwd, int mode, const Shape& sh, const void* W, uq_
     // Steps that map (remap, full) take the pipelined kernel on its shapes; the
     // keep step reads no weights, and the register kernel, which holds s_A
     // across a warp's rows, beats restaging s_A for every unit.
+    if (bwd && awq_stream_bwd_ok(sh)) {
+        if (sh.wdtype == UQ_W_BF16) return awq_stream_bwd<Q, WBF16>(sh, W, p, codes, gup, gr, work, st);
+        return awq_stream_bwd<Q, WF32>(sh, W, p, codes, gup, gr, work, st);
+    }
     if (!bwd && mode != FWD_KEEP && stream_path_ok(sh)) {
         if (sh.wdtype == UQ_W_BF16) return awq_stream_fwd<Q, WBF16>(mode, sh, W, p, codes, what, st);
         return awq_stream_fwd<Q, WF32>(mode, sh, W, p, codes, what, st);
