@@ -28,7 +28,7 @@ import math
 import torch
 import torch.nn.functional as F
 
-from . import api
+from . import api, checkpoint
 
 NAMES = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
 
@@ -139,6 +139,28 @@ class BlockReconstructor:
             self.qz[n].train_step(self.t, self.lr_F, self.lr_B, self.p, self.map_mode)
         self.t += 1
         return loss.detach()
+
+    def save(self, path):
+        """Checkpoint: Theta_IF and the codes of the seven weights and the
+        step counter (checkpoint.save_state)."""
+        checkpoint.save_state(path, {n: (self.P[n], self.codes[n]) for n in NAMES}, self.t, q=self.q, g=self.g,
+                              p=self.p, map_mode=self.map_mode, lr_F=float(self.lr_F), lr_B=float(self.lr_B))
+
+    def load(self, path):
+        """Resume from a checkpoint written by save(): loads Theta_IF, the
+        codes and the step counter, and rebuilds W^ from them without
+        mapping, so the next step() continues the saved run exactly."""
+        mats, step, meta = checkpoint.load_state(path)
+        if (meta.get("q"), meta.get("g")) != (self.q, self.g):
+            raise ValueError(f"checkpoint has q={meta.get('q')}, g={meta.get('g')}; this block has "
+                             f"q={self.q}, g={self.g}")
+        if set(mats) != set(NAMES):
+            raise ValueError(f"checkpoint holds {sorted(mats)}, expected {sorted(NAMES)}")
+        for n in NAMES:
+            checkpoint.restore_into(mats[n], self.P[n], self.codes[n])
+        for n in NAMES:
+            checkpoint.rebuild_what(self.qz[n])
+        self.t = step
 
     def state(self):
         """Host copies: ({name: params dict}, {name: codes}, {name: W^})."""
