@@ -34,6 +34,9 @@ if ROOT not in sys.path:
 
 METRIC = "quantizer fwd+bwd weights/sec and achieved HBM GB/s (% of GB300 peak) at q=3,g=128"
 RING = 16                       # parameter sets prepared before timing
+CLOCK_LEAD_S = 0.15             # untimed load before the timed steps while clocks are sampled
+CLOCK_MIN_S = 0.5               # sampling runs at least this long (about 5 samples at 100 ms)
+CLOCK_CHUNK = 16                # untimed steps between host checks of the elapsed time (even)
 
 
 # ---------------------------------------------------------------------------
@@ -78,6 +81,7 @@ class ClockSampler:
         self.gpu_id = gpu_id
 
     def start(self):
+        self.t0 = time.time()
         try:
             fd, self.path = tempfile.mkstemp(suffix=".csv")
             os.close(fd)
@@ -93,7 +97,7 @@ class ClockSampler:
     def stop(self):
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
-        time.sleep(max(0.0, 0.35 - (time.time() - self.t0)))
+        time.sleep(max(0.0, CLOCK_MIN_S - (time.time() - self.t0)))
         self.proc.terminate()
         self.proc.wait()
         sm, smax, reasons = [], [], set()
@@ -630,21 +634,40 @@ def run_gpu(args):
         gpu_id = gpu_id if gpu_id.startswith("GPU-") else "GPU-" + gpu_id
     except Exception:
         gpu_id = None
+    def load_for(seconds, t0):
+        # the same step loop, untimed, in chunks of an even number of steps
+        # (so the remap/keep alternation of the timed steps is unchanged)
+        n, t_start = 0, time.perf_counter()
+        while time.perf_counter() - t_start < seconds:
+            for i in range(CLOCK_CHUNK):
+                step(t0 + n + i)
+            torch.cuda.synchronize()
+            n += CLOCK_CHUNK
+        return n
+
+    # Clocks are sampled every 100 ms while the GPU runs the step loop: the
+    # sampler starts before an untimed lead-in, and an untimed tail after the
+    # closing barrier keeps the load on until it has run CLOCK_MIN_S, so that
+    # every sample is taken under the load of the timed steps.
     clk = ClockSampler(gpu_id)
+    clk.start()
+    lead = load_for(CLOCK_LEAD_S, args.warmup)
+    t_first = args.warmup + lead
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    clk.start()
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for t in range(args.steps):
-        step(args.warmup + t, evs[t])
+        step(t_first + t, evs[t])
     end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
+    load_for(CLOCK_MIN_S - (time.time() - clk.t0), t_first + args.steps)
     clocks = clk.stop()
+    clocks["sampled_over"] = "an untimed lead-in of the same step loop, the timed steps and an untimed tail"
     ms = start.elapsed_time(end)
     ms_max = max_over_ranks(ms, world, dev)
     secs = ms_max / 1e3
@@ -653,7 +676,7 @@ def run_gpu(args):
     fwd_ms = [e[0].elapsed_time(e[1]) for e in evs]
     bwd_ms = [e[1].elapsed_time(e[2]) for e in evs]
     bwd_bytes = roofline.bytes_per_launch("bwd", out, n_in, q, g, wbytes)
-    steps_idx = [args.warmup + t for t in range(args.steps)]
+    steps_idx = [t_first + t for t in range(args.steps)]
     step_bytes = sum(roofline.step_bytes(out, n_in, q, g, wbytes, t % wl.p == 0) for t in steps_idx)
     peaks = measured_peaks()
     peak = peaks["hbm_gbs"] if peaks else 6800.0

@@ -36,7 +36,12 @@ constexpr int kBatchRows = 8;                   // rows a warp takes at a time
 constexpr int kMaxStagesGemv = 4;
 constexpr int kLutFloats = 2 * 256 * 32;        // [byte slot][entry][lane]
 constexpr int kNibFloats = 4 * 16 * 32;         // [nibble slot][entry][lane]
-constexpr size_t kGemvFixedSmem = (size_t)(kLutFloats + kNibFloats + kTileCols) * sizeof(float);
+// x of the tile, lane-major with a padded stride of 17 floats per lane's 16
+// columns, so that the table build's reads (one lane per 16 columns) fall
+// in distinct banks
+constexpr int kXsStride = 17;
+constexpr int kXsFloats = 32 * kXsStride;
+constexpr size_t kGemvFixedSmem = (size_t)(kLutFloats + kNibFloats + kXsFloats) * sizeof(float);
 constexpr size_t kGemvSmemLimit = 227 * 1024;   // dynamic shared memory a block may opt in to
 
 // Groups of one row inside one tile: 512 / g, or 1 when a group spans whole tiles.
@@ -94,8 +99,8 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
     extern __shared__ __align__(16) float gsm[];
     float* lut = gsm;                                 // [2][256][32]
     float* nib = lut + kLutFloats;                    // [4][16][32]
-    float* xs = nib + kNibFloats;                     // [512]
-    uint32_t* stages = reinterpret_cast<uint32_t*>(xs + kTileCols);
+    float* xs = nib + kNibFloats;                     // [32][17]: lane l's columns at 17 l
+    uint32_t* stages = reinterpret_cast<uint32_t*>(xs + kXsFloats);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t = (int)(blockIdx.x % n_tiles);
     const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
@@ -177,12 +182,12 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
             cp_commit();
         }
         for (int i = threadIdx.x; i < kTileCols; i += kGemvThreads)
-            xs[i] = c0 + i < n_in ? XT::get(X, (int64_t)b * n_in + c0 + i) : 0.f;
+            xs[kXsStride * (i >> 4) + (i & 15)] = c0 + i < n_in ? XT::get(X, (int64_t)b * n_in + c0 + i) : 0.f;
         __syncthreads();
         // nibble tables: slot s = 2 k + h covers columns 16 l + 8 k + 4 h + (0..3)
         for (int e = threadIdx.x; e < kNibFloats; e += kGemvThreads) {
             const int l = e & 31, v = (e >> 5) & 15, s = e >> 9;
-            const float* xc = xs + 16 * l + 4 * s;
+            const float* xc = xs + kXsStride * l + 4 * s;
             float acc = 0.f;
 #pragma unroll
             for (int bit = 0; bit < 4; ++bit)
