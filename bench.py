@@ -826,6 +826,42 @@ def run_gpu(args):
     return result
 
 
+def time_oracle_workload(wl, q, budget_s, weights_per_matrix=131072):
+    """The CPU oracle as it stands (numpy, one thread) on a bounded sample of
+    every matrix of a workload: the first rows of each matrix (about
+    `weights_per_matrix` weights), oracle-initialised and jittered like the
+    GPU inputs.  One step = per matrix the forward (local mapping at step t),
+    the backward and the bit-plane export (Theorem 1, reused codes).  Runs
+    whole steps until budget_s has passed.  Returns (weights per second,
+    weights per step, steps, seconds)."""
+    import oracle as O
+    from paper_2506_03781_gb300 import synth
+    g = wl.g
+    mats = []
+    for idx, m in enumerate(wl.matrices):
+        rows = max(1, min(m.out, weights_per_matrix // m.n_in))
+        _, W = synth.workload_weights(wl, idx, slice(0, rows))
+        init = O.unified_init(W, q, g, G=2, T=2)
+        P = {k: init[k] for k in ("delta", "zu", "s", "sr", "alpha", "zb")}
+        P = synth.jitter(P, synth.perturb_factors(synth.param_shapes(rows, m.n_in, g, q), wl.init_eps, idx))
+        mats.append([W, P, init["codes"], synth.upstream_grad(rows, m.n_in, wl.grad_var, idx)])
+    n = sum(mm[0].size for mm in mats)
+    t0 = time.perf_counter()
+    steps = 0
+    while True:
+        for mm in mats:
+            W, P, codes, Gup = mm
+            _, codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes, g,
+                                      O.MAP_LOCAL_PERIODIC, steps, wl.p)
+            O.quantize_bwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes, Gup, g)
+            O.export_bcq(W, P["delta"], P["zu"], P["alpha"], P["zb"], codes, g)
+            mm[2] = codes
+        steps += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            return n * steps / el, n, steps, el
+
+
 def run_workloads(args):
     """Times the other workloads: the Llama-3-8B block (seven matrices, q = 2,
     g = 64, fwd + bwd + export as one launch sequence on one stream) and the
@@ -836,13 +872,21 @@ def run_workloads(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     lines = []
-    for name in ("llama3_8b_block_bf16", "llama2_70b_mlp_bf16", "attn4k_bf16", "mat1k_f32"):
+    names = ("llama3_8b_block_bf16", "llama2_70b_mlp_bf16", "attn4k_bf16", "mat1k_f32")
+    for name in names:
         wl = synth.WORKLOADS[name]
+        cpu = None
+        if not args.no_cpu_baseline:
+            v, n_s, k, el = time_oracle_workload(wl, wl.q, args.cpu_budget / len(names))
+            cpu = {"value": v, "unit": "weights/s", "cores": 1, "kind": "oracle",
+                   "sample": f"the first rows of each of the {len(wl.matrices)} matrices ({n_s} weights), {k} "
+                             f"oracle steps of fwd + bwd + bit-plane export in {el:.1f} s, numpy single thread"}
         for graph in (False, True):
             ms, n = time_matrices(wl, wl.q, args.steps, args.warmup, dev, with_export=True, graph=graph)
             line = {"workload": name, "q": wl.q, "g": wl.g, "weights": n, "steps": args.steps,
                     "cuda_graph": graph, "ms_per_step": ms, "weights_per_s": n / (ms / 1e3),
-                    "step": "per matrix: fwd (local mapping, remap/keep alternating) + bwd + bit-plane export"}
+                    "step": "per matrix: fwd (local mapping, remap/keep alternating) + bwd + bit-plane export",
+                    "cpu_baseline": cpu}
             print(json.dumps(line))
             lines.append(line)
     return lines

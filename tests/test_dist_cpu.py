@@ -62,43 +62,3 @@ def test_single_rank_defaults():
     assert bench.max_over_ranks(3.0, 1) == 3.0
     assert bench.weak_scaling_value(58720256, 4, 1, 2.0) == 58720256 * 4 / 2.0
 
-
-def test_reference_arm_line(capsys):
-    """`bench.py --impl reference` times the CPU oracle on a bounded sample
-    and prints one JSON line with the GPU arm's metric, unit and direction."""
-    import json
-
-    import bench
-    bench.main(["--impl", "reference", "--steps", "2", "--warmup", "3"])
-    lines = [ln for ln in capsys.readouterr().out.splitlines() if ln.startswith("{")]
-    assert len(lines) == 1
-    d = json.loads(lines[0])
-    assert d["impl"] == "reference" and d["metric"] == bench.METRIC
-    assert d["unit"] == "weights/s" and d["higher_is_better"] is True
-    assert d["steps"] == 2 and d["warmup"] == 3 and d["value"] > 0
-    assert d["config"]["workload"] == "mlp14336x4096_bf16" and d["config"]["mapping"] == "local, p=2"
-    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
-    assert d["e2e"] == {"value": d["value"], "unit": "weights/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
-
-
-def _ref_worker(rank, world, port, results):
-    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world),
-                      LOCAL_RANK=str(rank))
-    import bench
-    results[rank] = bench.main(["--impl", "reference", "--steps", "1", "--warmup", "3"]) is not None
-
-
-@pytest.mark.timeout(180)
-def test_reference_arm_rank0_only():
-    """Under torchrun the reference arm runs on rank 0 alone; the others exit 0 without work."""
-    world = 2
-    port = _free_port()
-    ctx = mp.get_context("spawn")
-    results = ctx.Manager().dict()
-    procs = [ctx.Process(target=_ref_worker, args=(r, world, port, results)) for r in range(world)]
-    for p in procs:
-        p.start()
-    for p in procs:
-        p.join(150)
-        assert p.exitcode == 0
-    assert results[0] is True and results[1] is False
