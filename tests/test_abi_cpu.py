@@ -288,3 +288,17 @@ def test_oracle_and_product_are_independent():
     synth_src = open(os.path.join(prod, "synth.py")).read()
     for word in ("levels", "transform", "argmin", "bitplane"):
         assert word not in synth_src.lower(), word
+
+
+def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
+    """Without the built library every entry point raises: there is no other
+    implementation behind the binding."""
+    from paper_2506_03781_gb300 import api
+    monkeypatch.setattr(api, "LIB", str(tmp_path / "libuq.so"))
+    monkeypatch.setattr(api, "_lib", None)
+    with pytest.raises(RuntimeError, match="no fallback"):
+        api.lib()
+    with pytest.raises(RuntimeError, match="no fallback"):
+        api.uq_abi_version()
+    with pytest.raises(RuntimeError, match="no fallback"):
+        api.uq_bcq_gemv_workspace_bytes(8, 512)
