@@ -391,13 +391,14 @@ uq_status uq_bcq_gemv_noalloc(const uint32_t* bitplanes, const float* alpha_star
 uq_status uq_check_device(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
-    unsigned int flag = 0, flag_step = 0, flag_omni = 0, flag_awq = 0;
+    unsigned int flag = 0, flag_step = 0, flag_omni = 0, flag_awq = 0, flag_gemv = 0;
     e = uq::stream_error(true, &flag);
     if (e == cudaSuccess) e = uq::step_error(true, &flag_step);
     if (e == cudaSuccess) e = uq::omni_error(true, &flag_omni);
     if (e == cudaSuccess) e = uq::awq_error(true, &flag_awq);
+    if (e == cudaSuccess) e = uq::gemv_error(true, &flag_gemv);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
-    flag |= (flag_step << 4) | (flag_omni << 8) | (flag_awq << 12);
+    flag |= (flag_step << 4) | (flag_omni << 8) | (flag_awq << 12) | (flag_gemv << 16);
     if (flag) return fail(UQ_ERR_CUDA, "a bounded wait ran out on the device (flag %u): a kernel gave up waiting "
                                        "for its own data copies", flag);
     return ok();

@@ -15,16 +15,22 @@
 // Split over the columns ("split-K"): thread block (t, b) owns column tile t
 // and a range of rows, builds the tile's tables once per token and streams
 // its rows' plane bytes and group parameters through a per-warp ring of
-// shared-memory stages filled by asynchronous copies.  Lane l owns columns
+// shared-memory stages.  When every tile is whole (in a multiple of 512) and
+// holds at least 4 groups (g <= 128), lane 0 fills a stage with three tensor
+// copies (bcq_gemv_tma_kernel); otherwise every lane issues its share of
+// 16- or 4-byte asynchronous copies (bcq_gemv_partial_kernel).  Lane l owns columns
 // 16 l .. 16 l + 15 of the tile (one 16-bit half of a plane word).  A warp
 // takes 8 rows at a time; a reduce-scatter over the warp (uq_common.cuh,
 // SegReduce) leaves one row's tile partial on each of 8 lanes, which store it
 // to the caller's workspace [tile][token][row].  A second kernel sums the
 // partials of a row in tile order.  Deterministic; no atomics.
+#include <cuda.h>   // CUtensorMap and its enums (the encoder is reached through the runtime)
+
 #include <atomic>
 
 #include "uq_common.cuh"
 #include "uq_launch.h"
+#include "uq_pipe.cuh"
 
 namespace uq {
 
@@ -246,6 +252,182 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
     }
 }
 
+// ---------------------------------------------------------------------------
+// TMA-staged variant (whole tiles: in a multiple of 512, g in {32, 64, 128})
+// ---------------------------------------------------------------------------
+//
+// The same product, tiling, tables and reduction as bcq_gemv_partial_kernel;
+// only the staging differs.  Lane 0 of a warp moves one 8-row batch with three
+// tensor copies (cp.async.bulk.tensor) completing on the stage's mbarrier: the
+// q bit-planes of the batch's rows in the tile as one box {16 words, 8 rows,
+// q planes}, their alpha* as a box {NGT * q, 8 rows} and their z* as a box
+// {NGT, 8 rows}.  The stage then holds planes [j][row][16 words], alpha*
+// [row][NGT * q] and z* [row][NGT].  Rows past `out` read as zeros and are
+// never stored.  Batches of the next token are staged while the current
+// token's rows are processed (the stage contents do not depend on the token).
+// Every wait on an mbarrier is bounded; one that runs out sets g_gemv_err
+// (reported by uq_check_device), and the warp stops computing but still
+// takes part in the block's barriers, then waits for its copies in flight.
+
+__device__ unsigned int g_gemv_err = 0;
+
+namespace tmap {
+__device__ __forceinline__ void load_3d(uint32_t dst, const CUtensorMap* m, int x, int y, int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void load_2d(uint32_t dst, const CUtensorMap* m, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+            "r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+}  // namespace tmap
+
+// Bytes of one TMA stage: planes, alpha*, z* of 8 rows (each a multiple of 128).
+__host__ __device__ constexpr int gemv_tma_planes_bytes(int q) { return q * kBatchRows * kTileWords * 4; }
+__host__ __device__ constexpr int gemv_tma_alpha_bytes(int q, int ng) { return kBatchRows * ng * q * 4; }
+__host__ __device__ constexpr int gemv_tma_stage_bytes(int q, int ng) {
+    return gemv_tma_planes_bytes(q) + gemv_tma_alpha_bytes(q, ng) + kBatchRows * ng * 4;
+}
+static_assert(kGemvFixedSmem % 128 == 0, "TMA stages start on a 128-byte boundary");
+
+template <int Q, typename XT, int NGT>
+__global__ void __launch_bounds__(kGemvThreads, 1)
+bcq_gemv_tma_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_constant__ CUtensorMap tm_alpha,
+                    const __grid_constant__ CUtensorMap tm_z, const void* __restrict__ X, float* __restrict__ PART,
+                    int64_t out, int n_in, int batch, int n_tiles, int64_t rows_per_block) {
+    constexpr int PLB = gemv_tma_planes_bytes(Q), ALB = gemv_tma_alpha_bytes(Q, NGT);
+    constexpr int SB = gemv_tma_stage_bytes(Q, NGT);
+    constexpr int NS = gemv_stages(Q, NGT);           // the same bytes per stage as the cp.async layout
+    static_assert(SB == gemv_stage_words(Q, NGT) * 4 && SB % 128 == 0 && NS >= 2, "stage layout");
+    static_assert(NGT >= 4, "alpha* and z* boxes must span at least 16 bytes");
+    constexpr int LPG = 32 / NGT;
+    extern __shared__ __align__(128) float gsm_tma[];
+    float* lut = gsm_tma;                             // [2][256][32]
+    float* nib = lut + kLutFloats;                    // [4][16][32]
+    float* xs = nib + kNibFloats;                     // [32][17]
+    unsigned char* stages = reinterpret_cast<unsigned char*>(xs + kXsFloats);
+    unsigned long long* bars = reinterpret_cast<unsigned long long*>(stages + (size_t)kGemvWarps * NS * SB);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t = (int)(blockIdx.x % n_tiles);
+    const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
+    const int nr = (int)(out - r0 < rows_per_block ? out - r0 : rows_per_block);
+    if (nr <= 0) return;                              // the whole block: before any barrier
+    const int c0 = t * kTileCols;
+    const int nbat = (nr + kBatchRows - 1) / kBatchRows;
+    const int my_nb = warp < nbat ? (nbat - warp + kGemvWarps - 1) / kGemvWarps : 0;
+    unsigned char* wst = stages + (size_t)warp * NS * SB;
+    unsigned long long* wbar = bars + warp * NS;
+    const int gl = lane / LPG;
+    using SR = SegReduce<32>;
+
+    if (lane == 0) {
+        for (int s = 0; s < NS; ++s) tma::bar_init(tma::smem_addr(wbar + s), 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+
+    // items: token-major, this warp's batches k = 0 .. my_nb - 1 per token
+    const long long total = (long long)batch * my_nb;
+    long long issued = 0, waited = 0;
+    int ik = 0;                                       // batch of the next item to issue
+    auto issue_next = [&]() {                         // lane 0 only
+        const int s = (int)(issued % NS);
+        const uint32_t bar = tma::smem_addr(wbar + s);
+        const uint32_t d = tma::smem_addr(wst + (size_t)s * SB);
+        const int y = (int)(r0 + (int64_t)kBatchRows * (warp + kGemvWarps * ik));
+        tma::fence_async_smem();                     // the warp's reads of this stage come first
+        tma::bar_arrive_tx(bar, (uint32_t)SB);
+        tmap::load_3d(d, &tm_planes, t * kTileWords, y, 0, bar);
+        tmap::load_2d(d + PLB, &tm_alpha, t * NGT * Q, y, bar);
+        tmap::load_2d(d + PLB + ALB, &tm_z, t * NGT, y, bar);
+        ++issued;
+        if (++ik == my_nb) ik = 0;
+    };
+    if (lane == 0)
+        while (issued < total && issued < NS) issue_next();
+
+    bool alive = true;
+    for (int b = 0; b < batch; ++b) {                      // token b is row b of X
+        __syncthreads();                                    // the previous token's readers are done
+        for (int i = threadIdx.x; i < kTileCols; i += kGemvThreads)
+            xs[kXsStride * (i >> 4) + (i & 15)] = XT::get(X, (int64_t)b * n_in + c0 + i);
+        __syncthreads();
+        for (int e = threadIdx.x; e < kNibFloats; e += kGemvThreads) {
+            const int l = e & 31, v = (e >> 5) & 15, s = e >> 9;
+            const float* xc = xs + kXsStride * l + 4 * s;
+            float acc = 0.f;
+#pragma unroll
+            for (int bit = 0; bit < 4; ++bit)
+                if ((v >> bit) & 1) acc = __fadd_rn(acc, xc[bit]);
+            nib[e] = acc;
+        }
+        __syncthreads();
+        {
+            const int l = threadIdx.x & 31, n = threadIdx.x >> 5;
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const float lo = nib[((2 * k) * 16 + n) * 32 + l];
+                const float* hi = nib + (2 * k + 1) * 16 * 32 + l;
+                float* dst = lut + (k * 256 + n) * 32 + l;
+#pragma unroll
+                for (int m = 0; m < 16; ++m) dst[m * 16 * 32] = __fadd_rn(lo, hi[m * 32]);
+            }
+        }
+        __syncthreads();
+        const float S = __fadd_rn(lut[(0 * 256 + 255) * 32 + lane], lut[(1 * 256 + 255) * 32 + lane]);
+        const float* lut0 = lut + lane;
+        const float* lut1 = lut + 256 * 32 + lane;
+        float* prow = PART + ((int64_t)t * batch + b) * out + r0;
+        for (int k = 0; k < my_nb; ++k) {
+            const long long i = (long long)b * my_nb + k;
+            const int s = (int)(i % NS);
+            if (alive) {
+                // one verdict for the whole warp (lanes poll the mbarrier separately)
+                if (__all_sync(kFull, tma::bar_wait(tma::smem_addr(wbar + s), (uint32_t)((i / NS) & 1)))) {
+                    ++waited;
+                } else {
+                    alive = false;
+                    if (lane == 0) atomicOr(&g_gemv_err, 1u);
+                }
+            }
+            if (alive) {
+                const unsigned char* st = wst + (size_t)s * SB;
+                const uint16_t* ph = reinterpret_cast<const uint16_t*>(st) + lane;
+                const float* pa = reinterpret_cast<const float*>(st + PLB) + gl * Q;
+                const float* pz = reinterpret_cast<const float*>(st + PLB + ALB) + gl;
+                const int rb = kBatchRows * (warp + kGemvWarps * k);
+                float v[kBatchRows];
+#pragma unroll
+                for (int rr = 0; rr < kBatchRows; ++rr) {
+                    float acc = __fmul_rn(pz[rr * NGT], S);
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) {
+                        const uint32_t h = ph[(j * kBatchRows + rr) * (2 * kTileWords)];
+                        const float P = __fadd_rn(lut0[(h & 255u) * 32], lut1[(h >> 8) * 32]);
+                        acc = fmaf(pa[rr * NGT * Q + j], fmaf(2.f, P, -S), acc);
+                    }
+                    v[rr] = rb + rr < nr ? acc : 0.f;
+                }
+                const int slot0 = SR::run(v, lane);
+                if (SR::writer(lane) && rb + slot0 < nr) prow[rb + slot0] = v[0];
+            }
+            __syncwarp();                                    // stage s is free for item i + NS
+            if (alive && lane == 0 && issued < total) issue_next();
+        }
+    }
+    if (!alive && lane == 0) {
+        // copies issued but never waited for land before the block exits
+        for (long long i = waited; i < issued; ++i)
+            tma::bar_wait(tma::smem_addr(wbar + (int)(i % NS)), (uint32_t)((i / NS) & 1));
+    }
+}
+
 // y[b, r] = sum over tiles of PART[t, b, r], in tile order.
 __global__ void __launch_bounds__(256)
 bcq_gemv_reduce_kernel(const float* __restrict__ PART, float* __restrict__ Y, int64_t n, int n_tiles) {
@@ -293,38 +475,101 @@ cudaError_t gemv_static_workspace(float** work) {
     return cudaSuccess;
 }
 
-template <int Q, typename XT, int NGT>
-static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in,
-                            int g, const void* x, int batch, float* y, float* work, cudaStream_t st) {
-    auto kern = bcq_gemv_partial_kernel<Q, XT, NGT>;
-    constexpr size_t stage_bytes = (size_t)gemv_stage_words(Q, NGT) * 4;
-    constexpr size_t smem = kGemvFixedSmem + kGemvWarps * (size_t)gemv_stages(Q, NGT) * stage_bytes;
-    static_assert(gemv_stages(Q, NGT) >= 2 && smem <= kGemvSmemLimit, "two stages must fit");
-    // alpha* and z* rows of a tile move in 16-byte pieces when every tile is
-    // whole (in a multiple of 512) and holds a multiple of 4 groups (both
-    // arrays start on 16-byte boundaries: the entry point checks that);
-    // otherwise in 4-byte pieces
-    const bool pwide = NGT % 4 == 0 && n_in % kTileCols == 0;
-    static int per_sm_cache[64] = {};
+cudaError_t gemv_error(bool clear, unsigned int* flag) {
+    unsigned int v = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_gemv_err, sizeof(v));
+    if (e != cudaSuccess) return e;
+    *flag = v;
+    if (clear && v) {
+        const unsigned int z = 0;
+        e = cudaMemcpyToSymbol(g_gemv_err, &z, sizeof(z));
+    }
+    return e;
+}
+
+using TensorMapEncode = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                     const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                     CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// The driver's tensor-map encoder, looked up once through the runtime (the
+// library does not link against the driver library).  Null if unavailable.
+static TensorMapEncode tensor_map_encoder() {
+    static std::atomic<TensorMapEncode> cached{nullptr};
+    static std::atomic<int> unavailable{0};
+    TensorMapEncode f = cached.load(std::memory_order_acquire);
+    if (f != nullptr || unavailable.load(std::memory_order_acquire)) return f;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qr = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &qr) != cudaSuccess ||
+        qr != cudaDriverEntryPointSuccess || p == nullptr) {
+        unavailable.store(1, std::memory_order_release);
+        return nullptr;
+    }
+    f = reinterpret_cast<TensorMapEncode>(p);
+    cached.store(f, std::memory_order_release);
+    return f;
+}
+
+// Tensor maps of the bit-planes [q][out][in/32] (u32), alpha* [out][Gr q] and
+// z* [out][Gr] (fp32), Gr = in / g, with the boxes of one 8-row batch of one
+// 512-column tile.  Called only for in a multiple of 512 and g <= 128, so every
+// stride is a multiple of 16 bytes and every box starts on a 16-byte boundary.
+// False if the encoder is unavailable or refuses a map.
+static bool gemv_tensor_maps(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in,
+                             int q, int g, CUtensorMap* mp, CUtensorMap* ma, CUtensorMap* mz) {
+    const TensorMapEncode enc = tensor_map_encoder();
+    if (enc == nullptr) return false;
+    const cuuint64_t words = (cuuint64_t)n_in / 32, gr = (cuuint64_t)(n_in / g), rows = (cuuint64_t)out;
+    const cuuint32_t ngt = (cuuint32_t)(kTileCols / g), one[3] = {1, 1, 1};
+    const cuuint64_t pdim[3] = {words, rows, (cuuint64_t)q};
+    const cuuint64_t pstride[2] = {words * 4, words * 4 * rows};
+    const cuuint32_t pbox[3] = {(cuuint32_t)kTileWords, (cuuint32_t)kBatchRows, (cuuint32_t)q};
+    if (enc(mp, CU_TENSOR_MAP_DATA_TYPE_UINT32, 3, const_cast<uint32_t*>(planes), pdim, pstride, pbox, one,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return false;
+    const cuuint64_t adim[2] = {gr * (cuuint64_t)q, rows};
+    const cuuint64_t astride[1] = {gr * (cuuint64_t)q * 4};
+    const cuuint32_t abox[2] = {ngt * (cuuint32_t)q, (cuuint32_t)kBatchRows};
+    if (enc(ma, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(astar), adim, astride, abox, one,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return false;
+    const cuuint64_t zdim[2] = {gr, rows};
+    const cuuint64_t zstride[1] = {gr * 4};
+    const cuuint32_t zbox[2] = {ngt, (cuuint32_t)kBatchRows};
+    return enc(mz, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(zstar), zdim, zstride, zbox, one,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Opts a kernel into `smem` bytes of dynamic shared memory and returns its
+// resident blocks per SM, once per device (Tag: one cache per kernel).
+template <typename Tag, typename KERN>
+static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm) {
+    static int cache[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    int per_sm = (dev >= 0 && dev < 64) ? per_sm_cache[dev] : 0;
-    if (per_sm == 0) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGemvThreads, smem);
-        if (e != cudaSuccess) return e;
-        if (per_sm < 1) per_sm = 1;
-        if (dev >= 0 && dev < 64) per_sm_cache[dev] = per_sm;
-    }
-    // Row blocks (of whole 8-row batches): the count that minimises
-    // waves x (one table build, worth about 32 rows, + rows per block), where
-    // a wave is one block per resident slot.
-    const int n_tiles = (n_in + kTileCols - 1) / kTileCols;
+    per_sm = (dev >= 0 && dev < 64) ? cache[dev] : 0;
+    if (per_sm != 0) return cudaSuccess;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGemvThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    if (dev >= 0 && dev < 64) cache[dev] = per_sm;
+    return cudaSuccess;
+}
+
+// Row blocks (of whole 8-row batches): the count that minimises
+// waves x (one table build, worth about 32 rows, + rows per block), where
+// a wave is one block per resident slot.
+static void gemv_row_blocks(int64_t out, int n_tiles, int per_sm, int64_t& n_rb, int64_t& rpb) {
     const int64_t slots = (int64_t)sm_count() * per_sm;
     const int64_t max_rb = (out + kBatchRows - 1) / kBatchRows;
-    int64_t n_rb = 1, rpb = max_rb * kBatchRows;
+    n_rb = 1;
+    rpb = max_rb * kBatchRows;
     double best = -1.0;
     const int64_t lim = max_rb < 8 * slots ? max_rb : 8 * slots;
     for (int64_t cand = 1; cand <= lim; ++cand) {
@@ -335,16 +580,66 @@ static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const fl
         const double cost = (double)waves * (32.0 + (double)r);
         if (best < 0.0 || cost < best) { best = cost; n_rb = nb; rpb = r; }
     }
-    kern<<<(unsigned)(n_rb * n_tiles), kGemvThreads, smem, st>>>(planes, astar, zstar, x, work, out, n_in, g, batch,
-                                                                 n_tiles, rpb, pwide);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    const int64_t n = (int64_t)batch * out;
+}
+
+// y = the per-tile partials summed in tile order.
+static cudaError_t gemv_reduce(const float* work, float* y, int64_t n, int n_tiles, cudaStream_t st) {
     int64_t blocks = (n + 255) / 256;
     const int64_t cap = (int64_t)sm_count() * 8;
     if (blocks > cap) blocks = cap;
     bcq_gemv_reduce_kernel<<<(unsigned)blocks, 256, 0, st>>>(work, y, n, n_tiles);
     return cudaGetLastError();
+}
+
+template <int Q, typename XT, int NGT>
+struct GemvCopyTag {};
+template <int Q, typename XT, int NGT>
+struct GemvTmaTag {};
+
+template <int Q, typename XT, int NGT>
+static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in,
+                            int g, const void* x, int batch, float* y, float* work, cudaStream_t st) {
+    constexpr size_t stage_bytes = (size_t)gemv_stage_words(Q, NGT) * 4;
+    constexpr int NS = gemv_stages(Q, NGT);
+    constexpr size_t smem = kGemvFixedSmem + kGemvWarps * (size_t)NS * stage_bytes;
+    constexpr size_t smem_tma = smem + kGemvWarps * (size_t)NS * sizeof(unsigned long long);   // + mbarriers
+    static_assert(NS >= 2 && smem_tma <= kGemvSmemLimit, "two stages must fit");
+    // Whole tiles and at least 4 groups per tile: staged by tensor copies.
+    // Otherwise by per-lane asynchronous copies; alpha* and z* rows of a tile
+    // move in 16-byte pieces when every tile is whole (in a multiple of 512)
+    // and holds a multiple of 4 groups (both arrays start on 16-byte
+    // boundaries: the entry point checks that), else in 4-byte pieces.
+    const bool whole = n_in % kTileCols == 0;
+    const bool pwide = NGT % 4 == 0 && whole;
+    const int n_tiles = (n_in + kTileCols - 1) / kTileCols;
+    if constexpr (NGT >= 4) {
+        const unsigned long long plane_bytes = (unsigned long long)(n_in / 32) * 4ull * (unsigned long long)out;
+        CUtensorMap mp, ma, mz;
+        if (whole && plane_bytes < (1ull << 40) && gemv_tensor_maps(planes, astar, zstar, out, n_in, Q, g, &mp, &ma, &mz)) {
+            auto kern = bcq_gemv_tma_kernel<Q, XT, NGT>;
+            int per_sm = 0;
+            cudaError_t e = gemv_blocks_per_sm<GemvTmaTag<Q, XT, NGT>>(kern, smem_tma, per_sm);
+            if (e != cudaSuccess) return e;
+            int64_t n_rb = 0, rpb = 0;
+            gemv_row_blocks(out, n_tiles, per_sm, n_rb, rpb);
+            kern<<<(unsigned)(n_rb * n_tiles), kGemvThreads, smem_tma, st>>>(mp, ma, mz, x, work, out, n_in, batch,
+                                                                           n_tiles, rpb);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+            return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);
+        }
+    }
+    auto kern = bcq_gemv_partial_kernel<Q, XT, NGT>;
+    int per_sm = 0;
+    cudaError_t e = gemv_blocks_per_sm<GemvCopyTag<Q, XT, NGT>>(kern, smem, per_sm);
+    if (e != cudaSuccess) return e;
+    int64_t n_rb = 0, rpb = 0;
+    gemv_row_blocks(out, n_tiles, per_sm, n_rb, rpb);
+    kern<<<(unsigned)(n_rb * n_tiles), kGemvThreads, smem, st>>>(planes, astar, zstar, x, work, out, n_in, g, batch,
+                                                                 n_tiles, rpb, pwide);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);
 }
 
 template <int Q, typename XT>

@@ -52,6 +52,9 @@ int64_t gemv_workspace_floats(int64_t out, int64_t n_in, int batch);
 // floats, and its device address on the current device (looked up once per device).
 int64_t gemv_static_workspace_floats();
 cudaError_t gemv_static_workspace(float** work);
+// Reads (and optionally clears) the flag the product's tensor-copy staging sets
+// when a bounded wait runs out.
+cudaError_t gemv_error(bool clear, unsigned int* flag);
 cudaError_t launch_gemv(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in, int q,
                         int g, const void* x, int xdtype, int batch, float* y, float* work, cudaStream_t st);
 // UniQuan with OmniQuant's maps (uq_omni.cu); omni_ok: the group sizes it takes.
