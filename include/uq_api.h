@@ -382,6 +382,12 @@ uq_status uq_export_bcq_half(const void* W, uq_wdtype wdtype, int64_t out, int64
  * deterministic, and within a small multiple of the fp32 unit roundoff of
  * sum_i (sum_j |alpha*_j| + |z*|) |x_i| of the exact product.  Shapes as
  * uq_quantize_fwd; 1 <= batch <= 64 (each token re-reads the planes).
+ * When in is a multiple of 512 and g <= 128 the call also encodes three TMA
+ * tensor maps on the host (through the runtime's driver entry point; stack
+ * memory only, nothing is allocated) and the kernel stages its rows with
+ * them; any other shape, or a driver without the encoder, takes per-thread
+ * asynchronous copies.  Only the staging differs: both run the same
+ * arithmetic in the same order.
  * Reads every input, writes y and the workspace.  A too small workspace is
  * UQ_ERR_ARG.
  */
