@@ -547,18 +547,18 @@ static bool gemv_tensor_maps(const uint32_t* planes, const float* astar, const f
 // resident blocks per SM, once per device (Tag: one cache per kernel).
 template <typename Tag, typename KERN>
 static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm) {
-    static int cache[64] = {};
+    static std::atomic<int> cache[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    per_sm = (dev >= 0 && dev < 64) ? cache[dev] : 0;
+    per_sm = (dev >= 0 && dev < 64) ? cache[dev].load(std::memory_order_relaxed) : 0;
     if (per_sm != 0) return cudaSuccess;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGemvThreads, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
-    if (dev >= 0 && dev < 64) cache[dev] = per_sm;
+    if (dev >= 0 && dev < 64) cache[dev].store(per_sm, std::memory_order_relaxed);
     return cudaSuccess;
 }
 

@@ -8,6 +8,8 @@
 // shared memory.  Every copy starts and ends on a 16-byte boundary.
 #pragma once
 
+#include <atomic>
+
 #include "uq_common.cuh"
 #include "uq_launch.h"
 
@@ -169,21 +171,23 @@ constexpr int kMaxDevices = 64;
 
 // Persistent grid: min(row blocks, SMs x resident blocks per SM).  The
 // shared-memory attribute and the occupancy of a kernel instantiation are
-// set and queried once per device (KERN is a distinct type per call site).
+// set and queried once per device (KERN is a distinct type per call site);
+// the cache is atomic, so first calls from several host threads may race
+// only to store the same value.
 template <typename Tag, typename KERN>
 static cudaError_t grid_for(KERN kern, size_t dyn, int n_rb, int& grid) {
-    static int per_sm_cache[kMaxDevices] = {0};
+    static std::atomic<int> per_sm_cache[kMaxDevices] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    int per_sm = (dev >= 0 && dev < kMaxDevices) ? per_sm_cache[dev] : 0;
+    int per_sm = (dev >= 0 && dev < kMaxDevices) ? per_sm_cache[dev].load(std::memory_order_relaxed) : 0;
     if (per_sm == 0) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
         if (e != cudaSuccess) return e;
         e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn);
         if (e != cudaSuccess) return e;
         if (per_sm < 1) per_sm = 1;
-        if (dev >= 0 && dev < kMaxDevices) per_sm_cache[dev] = per_sm;
+        if (dev >= 0 && dev < kMaxDevices) per_sm_cache[dev].store(per_sm, std::memory_order_relaxed);
     }
     const long long cap = (long long)sm_count() * per_sm;
     grid = (int)(n_rb < cap ? n_rb : cap);

@@ -346,12 +346,12 @@ static cudaError_t run_step(const Shape& sh, const void* W, uq_params p, uint8_t
     const size_t dyn = (size_t)kWarps * 2 * St::BYTES;
     auto kern = step_kernel<Q, WT, G_, MODEB>;
     // occupancy per device and cluster size (blocks per SM for csize == 1, clusters on the GPU otherwise)
-    static int cache[kMaxDevicesStep][kMaxCluster + 1] = {};
+    static std::atomic<int> cache[kMaxDevicesStep][kMaxCluster + 1] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    int* slot = (dev >= 0 && dev < kMaxDevicesStep) ? &cache[dev][csize] : nullptr;
-    int cap = slot ? *slot : 0;
+    std::atomic<int>* slot = (dev >= 0 && dev < kMaxDevicesStep) ? &cache[dev][csize] : nullptr;
+    int cap = slot ? slot->load(std::memory_order_relaxed) : 0;
 
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -381,7 +381,7 @@ static cudaError_t run_step(const Shape& sh, const void* W, uq_params p, uint8_t
             if (e != cudaSuccess) return e;
             cap = ncl < 1 ? 1 : ncl;
         }
-        if (slot) *slot = cap;
+        if (slot) slot->store(cap, std::memory_order_relaxed);
     }
     const int64_t units = csize == 1 ? n_rb : sh.out;     // row blocks, or clusters' rows
     const int64_t n_grp = units < cap ? units : cap;       // blocks (csize == 1) or clusters

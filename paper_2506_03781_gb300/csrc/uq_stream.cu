@@ -14,6 +14,8 @@
 // uq_check_device() reports, and the warp stops computing.  The backward
 // kernel's ds_r partials wait in a shared-memory ring of kRowRing row
 // blocks, summed in warp order after one block barrier per ring.
+#include <atomic>
+
 #include "uq_common.cuh"
 #include "uq_launch.h"
 #include "uq_pipe.cuh"
@@ -375,12 +377,15 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // ---------------------------------------------------------------------------
 
 int sm_count() {
-    static int cached[kMaxDevices] = {0};
+    static std::atomic<int> cached[kMaxDevices] = {};
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 1;
-    if (dev >= 0 && dev < kMaxDevices && cached[dev] > 0) return cached[dev];
+    if (dev >= 0 && dev < kMaxDevices) {
+        const int c = cached[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return 1;
-    if (dev >= 0 && dev < kMaxDevices) cached[dev] = n;
+    if (dev >= 0 && dev < kMaxDevices) cached[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 
