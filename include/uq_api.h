@@ -20,6 +20,8 @@
  * Memory.  Every pointer argument is DEVICE memory owned by the caller
  *   (except the return value of uq_last_error).  The library never allocates,
  *   frees or keeps a pointer after a call returns.
+ * Device.  Work is launched on the calling thread's current CUDA device;
+ *   every pointer and the stream must belong to that device.
  * Asynchrony.  Work is enqueued on `stream` (a cudaStream_t; NULL = the
  *   legacy default stream) and the call returns without synchronising.
  *   UQ_OK means "validated and launched"; execution errors surface on the

@@ -151,6 +151,9 @@ def _check(t, name, shape, dtype, device):
         raise TypeError(f"{name} must be a torch.Tensor")
     if t.device.type != "cuda" or (device is not None and t.device != device):
         raise ValueError(f"{name} must be on {device or 'a CUDA device'} (got {t.device})")
+    if t.device.index != torch.cuda.current_device():
+        raise ValueError(f"{name} is on {t.device} but the current device is cuda:{torch.cuda.current_device()}; "
+                         "the library launches on the current device (call it under torch.cuda.device(...))")
     if tuple(t.shape) != tuple(shape):
         raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
     if t.dtype != dtype:
@@ -651,6 +654,9 @@ class Quantizer:
         self.L = lib()
 
     def _st(self, stream):
+        if self.device.index != torch.cuda.current_device():
+            raise ValueError(f"this Quantizer's tensors are on {self.device} but the current device is "
+                             f"cuda:{torch.cuda.current_device()} (call it under torch.cuda.device(...))")
         return _stream(stream, self.device)
 
     def fwd(self, step, p_period=2, map_mode=MAP_LOCAL_PERIODIC, stream=None):
