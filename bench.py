@@ -100,23 +100,34 @@ class ClockSampler:
         time.sleep(max(0.0, CLOCK_MIN_S - (time.time() - self.t0)))
         self.proc.terminate()
         self.proc.wait()
-        sm, smax, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in open(self.path):
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                smax.append(float(parts[2]))
-            except ValueError:
-                continue
-            for n, v in zip(names, parts[5:9]):
-                if v.lower() == "active":
-                    reasons.add(n)
+        with open(self.path) as fh:
+            lines = fh.readlines()
         os.unlink(self.path)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        return parse_clock_samples(lines)
+
+
+def parse_clock_samples(lines):
+    """Clock record from `nvidia-smi --query-gpu=timestamp,<ClockSampler.FIELDS>
+    --format=csv,noheader,nounits` lines: median SM clock, the maximum SM
+    clock, and every throttle reason (of hw_slowdown, hw_thermal_slowdown,
+    sw_thermal_slowdown, sw_power_cap) seen Active in any sample.  Lines that
+    do not parse are skipped."""
+    sm, smax, reasons = [], [], set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for line in lines:
+        parts = [p.strip() for p in line.split(",")]
+        if len(parts) < 9:
+            continue
+        try:
+            sm.append(float(parts[1]))
+            smax.append(float(parts[2]))
+        except ValueError:
+            continue
+        for n, v in zip(names, parts[5:9]):
+            if v.lower() == "active":
+                reasons.add(n)
+    return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+            "reasons": sorted(reasons), "samples": len(sm)}
 
 
 # ---------------------------------------------------------------------------

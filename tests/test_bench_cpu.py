@@ -62,3 +62,21 @@ def test_oracle_timing_of_a_workload_covers_every_matrix():
     expect = sum(max(1, min(m.out, 8192 // m.n_in)) * m.n_in for m in wl.matrices)
     assert n == expect and steps >= 1 and el >= 0.05
     assert v == pytest.approx(n * steps / el)
+
+
+def test_clock_record_from_nvidia_smi_lines():
+    """The clock record of the bench line: median SM clock under load, the
+    maximum, and every throttle reason seen Active in any sample (a run with
+    hw_slowdown, hw_thermal_slowdown or sw_thermal_slowdown is rejected;
+    sw_power_cap is kept and noted)."""
+    import bench
+    ok = "2026/12/02 10:00:00.100, 2070, 2070, 900.1, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active"
+    cap = "2026/12/02 10:00:00.200, 1950, 2070, 1380.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active"
+    hot = "2026/12/02 10:00:00.300, 1500, 2070, 1390.0, 0x0000000000000040, Not Active, Active, Not Active, Not Active"
+    r = bench.parse_clock_samples([ok, ok, cap, "garbage", "", "a, b, c, d, e, f, g, h, i"])
+    assert r == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    r = bench.parse_clock_samples([ok, hot, cap])
+    assert r["reasons"] == ["hw_thermal_slowdown", "sw_power_cap"] and r["sm_mhz"] == 1950.0
+    assert bench.parse_clock_samples([]) == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+    # the query the sampler issues has exactly the fields the parser reads
+    assert bench.ClockSampler.FIELDS.count(",") == 7
