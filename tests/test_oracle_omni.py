@@ -138,3 +138,19 @@ def test_export_reproduces_the_quantizer_output(q):
     scale = np.repeat(np.abs(delta.astype(F64)) * (np.abs(pb["alpha"]).sum(-1) + np.abs(pb["zb"]) + np.abs(zo)),
                       pb["g"], axis=1)
     assert np.all(np.abs(Wt - what) <= 8 * np.finfo(F32).eps * scale)
+
+
+@pytest.mark.parametrize("wm,wM,expect_zo", [(-2.5, 0.5, 2.0), (-1.5, 1.5, 2.0), (-0.5, 2.5, 0.0), (-3.5, -0.5, 4.0)])
+def test_zero_point_rounds_half_to_even(wm, wM, expect_zo):
+    """Reading of the zero point z_O = -round(beta w_m / Delta_O): exact
+    halves go to the even integer.  With q = 2 and beta = gamma = 1,
+    Delta_O = (w_M - w_m) / 3 = 1 for these groups, so beta w_m / Delta_O = w_m
+    exactly: -2.5 -> -2 (not -3), -1.5 -> -2, -0.5 -> -0, -3.5 -> -4."""
+    g = 32
+    w = np.linspace(wm, wM, g).astype(F32)
+    w[0], w[-1] = wm, wM
+    W = w[None, :]
+    one = np.ones((1, 1), F32)
+    delta, zo = O.omni_params(W, one, one, 2, g)
+    assert delta[0, 0] == F32(1.0)
+    assert zo[0, 0] == F32(expect_zo)
