@@ -190,3 +190,40 @@ def test_half_export_rounds_to_nearest_even():
     for v32, v16 in ((a32, a16), (z32, z16)):
         for a, b in zip(v32.ravel(), v16.ravel()):
             assert struct.unpack("<H", struct.pack("<e", float(a)))[0] == int(b)
+
+
+@pytest.mark.parametrize("q", [1, 2, 3, 4])
+def test_l1_mass_is_tight_when_every_term_has_one_sign(q):
+    """The masses set the gradient tolerances, so they must not be inflated:
+    with dL/dW^ >= 0, Delta > 0 and every code bit set (c_j = +1 for all j),
+    every term of dz_B = sum Delta G and of dalpha_j = sum Delta G c_j has
+    the same sign, and the mass equals the absolute value of the sum."""
+    pb = make_problem(500 + q, q)
+    codes = np.full_like(pb["codes"], (1 << q) - 1)
+    Gup = np.abs(pb["Gup"]).astype(F32)
+    args = (pb["W"], pb["s"], pb["sr"], pb["delta"], pb["zu"], pb["alpha"], pb["zb"], codes, Gup, pb["g"])
+    gr, ms = O.quantize_bwd(*args), O.bwd_l1_mass(*args)
+    assert np.allclose(ms["dzb"], np.abs(gr["dzb"]), rtol=1e-6, atol=0)
+    assert np.allclose(ms["dalpha"], np.abs(gr["dalpha"]), rtol=1e-6, atol=0)
+
+
+def test_variant_l1_masses_are_tight_when_every_term_has_one_sign():
+    """The same for the OmniQuant and AWQ maps: with dL/dW^ >= 0 and every
+    code bit set, the masses of dz_B and dalpha equal |dz_B| and |dalpha|."""
+    from tests.test_oracle_awq import problem as awq_problem
+    from tests.test_oracle_omni import problem as omni_problem
+    q = 3
+    po = omni_problem(61, q)
+    codes = np.full_like(po["codes"], (1 << q) - 1)
+    Gup = np.abs(po["Gup"]).astype(F32)
+    args = (po["W"], po["beta"], po["gamma"], po["alpha"], po["zb"], codes, Gup, po["g"])
+    gr, ms = O.quantize_bwd_omni(*args), O.bwd_l1_mass_omni(*args)
+    assert np.allclose(ms["dzb"], np.abs(gr["dzb"]), rtol=1e-6, atol=0)
+    assert np.allclose(ms["dalpha"], np.abs(gr["dalpha"]), rtol=1e-6, atol=0)
+    pa = awq_problem(62, q)
+    codes = np.full_like(pa["codes"], (1 << q) - 1)
+    Gup = np.abs(pa["Gup"]).astype(F32)
+    args = (pa["W"], pa["sa"], pa["delta"], pa["za"], pa["alpha"], pa["zb"], codes, Gup, pa["g"])
+    gr, ms = O.quantize_bwd_awq(*args), O.bwd_l1_mass_awq(*args)
+    assert np.allclose(ms["dzb"], np.abs(gr["dzb"]), rtol=1e-6, atol=0)
+    assert np.allclose(ms["dalpha"], np.abs(gr["dalpha"]), rtol=1e-6, atol=0)
