@@ -383,7 +383,9 @@ uq_status uq_export_bcq_half(const void* W, uq_wdtype wdtype, int64_t out, int64
  * tiles are summed in order into y.  fp32 throughout, fixed order:
  * deterministic, and within a small multiple of the fp32 unit roundoff of
  * sum_i (sum_j |alpha*_j| + |z*|) |x_i| of the exact product.  Shapes as
- * uq_quantize_fwd; 1 <= batch <= 64 (each token re-reads the planes).
+ * uq_quantize_fwd, except that g must divide 512 or be a multiple of 512
+ * (32, 64, 128, 256, 512, 1024, ...; any other g, e.g. 384 or 640, is
+ * UQ_ERR_UNSUPPORTED); 1 <= batch <= 64 (each token re-reads the planes).
  * When in is a multiple of 512 and g <= 128 the call also encodes three TMA
  * tensor maps on the host (through the runtime's driver entry point; stack
  * memory only, nothing is allocated) and the kernel stages its rows with
@@ -419,8 +421,11 @@ int64_t uq_bcq_gemv_workspace_bytes(int64_t out, int64_t in, int batch);
  * no cudaFree, no library routine that allocates.
  *
  * The first call on a device looks up the scratch's device address (once,
- * with that device current) and caches it; make that first call before any
- * stream capture.  All calls share the one scratch array and it keeps the
+ * with that device current) and caches it with the identifier of the
+ * device's context; make that first call before any stream capture.  After
+ * cudaDeviceReset the device gets a new context and the array a possibly
+ * different address, so the first call in the new context looks it up again
+ * (and must also come before any capture).  All calls share the one scratch array and it keeps the
  * last call's contents: each call overwrites every word it reads before
  * reading it, so nothing needs clearing, but two calls whose work overlaps
  * on the GPU (for instance on two streams) race on it and may give wrong

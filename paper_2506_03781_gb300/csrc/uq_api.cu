@@ -60,6 +60,19 @@ uq_status cuda_status(cudaError_t e, const char* what) {
     return ok();
 }
 
+// The product cuts the columns into tiles of 512; a row's groups must either
+// tile a column tile exactly (g divides 512) or be made of whole tiles (512
+// divides g), so that every group boundary falls on a lane boundary the
+// kernels know at compile time.
+uq_status check_gemv_group(int g) {
+    if (512 % g != 0 && g % 512 != 0)
+        return fail(UQ_ERR_UNSUPPORTED,
+                    "g=%d: the BCQ product needs g to divide 512 or to be a multiple of 512 (32, 64, 128, 256, "
+                    "512, 1024, ...)",
+                    g);
+    return UQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -347,6 +360,7 @@ uq_status uq_bcq_gemv(const uint32_t* bitplanes, const float* alpha_star, const 
                       int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch, float* y, float* workspace,
                       int64_t workspace_bytes, void* stream) {
     UQ_TRY(check_shape(out, in, q, g, xdtype));
+    UQ_TRY(check_gemv_group(g));
     if (batch < 1 || batch > 64) return fail(UQ_ERR_ARG, "batch=%d must be in 1..64", batch);
     UQ_TRY(check_ptr(bitplanes, "bitplanes"));
     UQ_TRY(check_ptr(alpha_star, "alpha_star"));
@@ -367,6 +381,7 @@ uq_status uq_bcq_gemv_noalloc(const uint32_t* bitplanes, const float* alpha_star
                               int64_t out, int64_t in, int q, int g, const void* x, uq_wdtype xdtype, int batch,
                               float* y, void* stream) {
     UQ_TRY(check_shape(out, in, q, g, xdtype));
+    UQ_TRY(check_gemv_group(g));
     if (batch < 1 || batch > 64) return fail(UQ_ERR_ARG, "batch=%d must be in 1..64", batch);
     UQ_TRY(check_ptr(bitplanes, "bitplanes"));
     UQ_TRY(check_ptr(alpha_star, "alpha_star"));
@@ -399,6 +414,12 @@ uq_status uq_check_device(void* stream) {
     if (e == cudaSuccess) e = uq::gemv_error(true, &flag_gemv);
     if (e != cudaSuccess) return fail(UQ_ERR_CUDA, "uq_check_device: %s", cudaGetErrorString(e));
     flag |= (flag_step << 4) | (flag_omni << 8) | (flag_awq << 12) | (flag_gemv << 16);
+    const unsigned int drain_bits = 0x88888u;   // kDrainTimeoutBit of each kernel family
+    if (flag & drain_bits)
+        return fail(UQ_ERR_CUDA, "a bounded wait ran out on the device (flag %u): a kernel gave up waiting "
+                                 "for its own data copies, and its wait for the copies still in flight ran out "
+                                 "too, so a block may have exited with copies landing in its shared memory",
+                    flag);
     if (flag) return fail(UQ_ERR_CUDA, "a bounded wait ran out on the device (flag %u): a kernel gave up waiting "
                                        "for its own data copies", flag);
     return ok();

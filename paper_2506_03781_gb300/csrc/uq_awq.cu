@@ -316,7 +316,7 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
         if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
             if (lane == 0) {
                 atomicOr(&g_awq_err, 1u);
-                drain(bars[warp], i, issued);
+                if (!drain(bars[warp], i, issued)) atomicOr(&g_awq_err, kDrainTimeoutBit);
             }
             return;                                      // no block barrier in this kernel
         }
@@ -537,7 +537,7 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
         if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
             if (lane == 0) {
                 atomicOr(&g_awq_err, 2u);
-                drain(bars[warp], i, issued);
+                if (!drain(bars[warp], i, issued)) atomicOr(&g_awq_err, kDrainTimeoutBit);
             }
             return;                                      // no block barrier in this kernel
         }

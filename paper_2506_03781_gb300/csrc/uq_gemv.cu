@@ -27,6 +27,7 @@
 #include <cuda.h>   // CUtensorMap and its enums (the encoder is reached through the runtime)
 
 #include <atomic>
+#include <mutex>
 
 #include "uq_common.cuh"
 #include "uq_launch.h"
@@ -424,7 +425,10 @@ bcq_gemv_tma_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_
     if (!alive && lane == 0) {
         // copies issued but never waited for land before the block exits
         for (long long i = waited; i < issued; ++i)
-            tma::bar_wait(tma::smem_addr(wbar + (int)(i % NS)), (uint32_t)((i / NS) & 1));
+            if (!tma::bar_wait(tma::smem_addr(wbar + (int)(i % NS)), (uint32_t)((i / NS) & 1))) {
+                atomicOr(&g_gemv_err, kDrainTimeoutBit);   // copies may still be in flight
+                break;
+            }
     }
 }
 
@@ -452,25 +456,65 @@ static __device__ __align__(256) float g_gemv_static_work[kStaticWorkFloats];
 
 int64_t gemv_static_workspace_floats() { return kStaticWorkFloats; }
 
-// Device address of g_gemv_static_work on the current device.  The name is
-// only a host-side stand-in in host code, so the address is looked up once
-// per device with that device current, and cached.
+// Identifier of the calling thread's current CUDA context (unique for the
+// life of the process, so a context created anew after cudaDeviceReset gets
+// a new one), through the runtime's driver entry points.  False if no
+// context is current yet or the driver lacks the calls.
+static bool current_context_id(unsigned long long* id) {
+    using GetCurrent = CUresult (*)(CUcontext*);
+    using GetId = CUresult (*)(CUcontext, unsigned long long*);
+    static std::atomic<void*> get_current{nullptr}, get_id{nullptr};
+    void* fc = get_current.load(std::memory_order_acquire);
+    void* fi = get_id.load(std::memory_order_acquire);
+    if (fc == nullptr || fi == nullptr) {
+        cudaDriverEntryPointQueryResult qr = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fc, 12000, cudaEnableDefault, &qr) != cudaSuccess ||
+            qr != cudaDriverEntryPointSuccess || fc == nullptr)
+            return false;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &fi, 12000, cudaEnableDefault, &qr) != cudaSuccess ||
+            qr != cudaDriverEntryPointSuccess || fi == nullptr)
+            return false;
+        get_current.store(fc, std::memory_order_release);
+        get_id.store(fi, std::memory_order_release);
+    }
+    CUcontext ctx = nullptr;
+    if (reinterpret_cast<GetCurrent>(fc)(&ctx) != CUDA_SUCCESS || ctx == nullptr) return false;
+    return reinterpret_cast<GetId>(fi)(ctx, id) == CUDA_SUCCESS;
+}
+
+// Device address of g_gemv_static_work in the current device's context.  The
+// name is only a host-side stand-in in host code, so the address is looked up
+// with that device current (cudaGetSymbolAddress) and cached per device
+// together with the context's identifier; a new context on the device (after
+// cudaDeviceReset) is looked up again.
 cudaError_t gemv_static_workspace(float** work) {
-    static std::atomic<float*> cached[64] = {};
+    struct Entry {
+        unsigned long long ctx;
+        float* ptr;
+    };
+    static Entry cache[kMaxDevices] = {};
+    static std::mutex lock;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev >= 0 && dev < 64) {
-        float* p = cached[dev].load(std::memory_order_acquire);
-        if (p != nullptr) {
-            *work = p;
+    const bool cacheable = dev >= 0 && dev < kMaxDevices;
+    unsigned long long id = 0;
+    bool have_id = current_context_id(&id);
+    if (cacheable && have_id) {
+        std::lock_guard<std::mutex> g(lock);
+        if (cache[dev].ptr != nullptr && cache[dev].ctx == id) {
+            *work = cache[dev].ptr;
             return cudaSuccess;
         }
     }
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_gemv_static_work);
+    e = cudaGetSymbolAddress(&p, g_gemv_static_work);   // makes the device's context current if it was not
     if (e != cudaSuccess) return e;
-    if (dev >= 0 && dev < 64) cached[dev].store(static_cast<float*>(p), std::memory_order_release);
+    if (!have_id) have_id = current_context_id(&id);
+    if (cacheable && have_id) {
+        std::lock_guard<std::mutex> g(lock);
+        cache[dev] = Entry{id, static_cast<float*>(p)};
+    }
     *work = static_cast<float*>(p);
     return cudaSuccess;
 }

@@ -328,7 +328,7 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
         if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
             if (lane == 0) {
                 atomicOr(&g_omni_err, 1u);
-                drain(bars[warp], i, issued);
+                if (!drain(bars[warp], i, issued)) atomicOr(&g_omni_err, kDrainTimeoutBit);
             }
             return;                                      // no block barrier in this kernel
         }
@@ -462,7 +462,7 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
         if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
             if (lane == 0) {
                 atomicOr(&g_omni_err, 1u);
-                drain(bars[warp], i, issued);
+                if (!drain(bars[warp], i, issued)) atomicOr(&g_omni_err, kDrainTimeoutBit);
             }
             return;                                      // no block barrier in this kernel
         }

@@ -19,6 +19,10 @@ namespace uq {
 #define UQ_WAIT_HINT_NS 20000
 #endif
 constexpr uint32_t kWaitHintNs = UQ_WAIT_HINT_NS;   // suspend-time hint of one try_wait
+// Bit of a kernel family's device flag set when, after a wait ran out, the
+// bounded wait for the copies still in flight ran out too (bits 0-2 name the
+// wait that ran out first).
+constexpr unsigned int kDrainTimeoutBit = 8u;
 
 namespace tma {
 
@@ -160,11 +164,14 @@ struct Cursor {
 
 // After a wait ran out: waits (bounded again) for the copies of items
 // [waited, issued) of a warp's stage ring, so that none lands in shared
-// memory after the block has exited.  Lane 0 only.
+// memory after the block has exited.  Lane 0 only.  False if one of these
+// waits ran out as well: the block may then exit with copies still in
+// flight into its shared memory, and the caller records kDrainTimeoutBit.
 template <int NST>
-__device__ void drain(unsigned long long (&bars)[NST], long long waited, long long issued) {
+__device__ bool drain(unsigned long long (&bars)[NST], long long waited, long long issued) {
     for (long long i = waited; i < issued; ++i)
-        tma::bar_wait(tma::smem_addr(&bars[i % NST]), (uint32_t)((i / NST) & 1));
+        if (!tma::bar_wait(tma::smem_addr(&bars[i % NST]), (uint32_t)((i / NST) & 1))) return false;
+    return true;
 }
 
 constexpr int kMaxDevices = 64;

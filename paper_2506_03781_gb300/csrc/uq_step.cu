@@ -317,7 +317,10 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
     if (!alive && lane == 0) {
         // copies this warp issued but never waited for land before the block exits
         for (int64_t k = next_wait; k < next_issue; ++k)
-            tma::bar_wait(tma::smem_addr(&bars[warp][k & 1]), (uint32_t)((k >> 1) & 1));
+            if (!tma::bar_wait(tma::smem_addr(&bars[warp][k & 1]), (uint32_t)((k >> 1) & 1))) {
+                atomicOr(&g_step_err, kDrainTimeoutBit);   // copies may still be in flight
+                break;
+            }
     }
     if (csize > 1) cg::this_cluster().sync();      // no block leaves while another may read its partials
 }

@@ -212,7 +212,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
             __syncthreads();
         }
     }
-    if (!alive && lane == 0) drain(bars[warp], waited, issued);
+    if (!alive && lane == 0 && !drain(bars[warp], waited, issued)) atomicOr(&g_stream_err, kDrainTimeoutBit);
 }
 
 // ---------------------------------------------------------------------------
@@ -281,7 +281,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
             if (lane == 0) {
                 atomicOr(&g_stream_err, 1u);
-                drain(bars[warp], i, issued);
+                if (!drain(bars[warp], i, issued)) atomicOr(&g_stream_err, kDrainTimeoutBit);
             }
             return;                                      // no block barrier in this kernel
         }

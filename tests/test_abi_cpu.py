@@ -175,6 +175,8 @@ def test_train_step_accepts_the_fused_shapes(libpath, g, n_in):
 @pytest.mark.parametrize("case,expect", [
     (dict(q=0), "UNSUPPORTED"), (dict(g=48), "ARG"), (dict(n_in=200), "ARG"), (dict(out=0), "ARG"),
     (dict(batch=0), "ARG"), (dict(batch=65), "ARG"), (dict(xd=5), "ARG"),
+    (dict(g=384, n_in=1536), "UNSUPPORTED"), (dict(g=640, n_in=1280), "UNSUPPORTED"),
+    (dict(g=768, n_in=1536), "UNSUPPORTED"),
     (dict(planes=0), "ARG"), (dict(planes=FAKE + 4), "ALIGN"), (dict(a=0), "ARG"), (dict(z=FAKE + 8), "ALIGN"),
     (dict(x=0), "ARG"), (dict(y=0), "ARG"), (dict(y=FAKE + 12), "ALIGN"),
     (dict(work=0), "ARG"), (dict(work=FAKE + 4), "ALIGN"), (dict(wbytes=8 * 4 - 4), "ARG"),
@@ -188,6 +190,30 @@ def test_bcq_gemv_validation(libpath, case, expect):
                                a["batch"], a["y"], a["work"], a["wbytes"], None)
     assert st == getattr(api, "UQ_ERR_" + expect), (st, api.uq_last_error())
     assert api.uq_last_error() != ""
+
+
+@cpu_only
+@pytest.mark.parametrize("g,n_in", [(32, 512), (256, 512), (512, 1024), (1024, 3072), (2048, 2048)])
+def test_bcq_gemv_accepts_groups_that_tile_the_column_tiles(libpath, g, n_in):
+    """g dividing 512 or a multiple of 512 passes validation (only the launch
+    fails on this GPU-less machine); both product entry points agree."""
+    from paper_2506_03781_gb300 import api
+    L = api.lib()
+    st = L.uq_bcq_gemv(FAKE, FAKE + 0x1000, FAKE + 0x2000, 8, n_in, 3, g, FAKE + 0x3000, api.W_BF16, 1,
+                       FAKE + 0x4000, FAKE + 0x5000, 1 << 20, None)
+    assert st == api.UQ_ERR_CUDA, api.uq_last_error()
+    st = L.uq_bcq_gemv_noalloc(FAKE, FAKE + 0x1000, FAKE + 0x2000, 8, n_in, 3, g, FAKE + 0x3000, api.W_BF16, 1,
+                               FAKE + 0x4000, None)
+    assert st == api.UQ_ERR_CUDA, api.uq_last_error()
+
+
+@cpu_only
+@pytest.mark.parametrize("g", [384, 640, 896, 1152])
+def test_bcq_gemv_noalloc_rejects_groups_that_straddle_column_tiles(libpath, g):
+    from paper_2506_03781_gb300 import api
+    st = api.lib().uq_bcq_gemv_noalloc(FAKE, FAKE + 0x1000, FAKE + 0x2000, 8, 2 * g * 9, 3, g, FAKE + 0x3000,
+                                       api.W_BF16, 1, FAKE + 0x4000, None)
+    assert st == api.UQ_ERR_UNSUPPORTED and "divide 512" in api.uq_last_error()
 
 
 def test_bcq_gemv_workspace_size(libpath):

@@ -70,7 +70,7 @@ def check(planes, a_star, z_star, x, g, xdtype="f32", label=""):
 # 16 groups per tile take the tensor-copy staging, the others the per-lane copies
 @pytest.mark.parametrize("out,n_in,g", [(40, 256, 32), (33, 512, 64), (17, 1536, 128), (64, 4096, 128),
                                         (9, 4096 + 32 * 3, 32), (5, 8192, 256), (3, 28672, 128), (300, 1024, 512),
-                                        (24, 1024, 32), (13, 2560, 64)])
+                                        (24, 1024, 32), (13, 2560, 64), (11, 3072, 1024), (6, 4096, 2048)])
 @pytest.mark.parametrize("q", [1, 2, 3, 4])
 def test_gemv_matches_oracle(out, n_in, g, q):
     if n_in % g:

@@ -4,9 +4,10 @@ whole GPU, or where an allocation call is not allowed because it can block
 the device).  It runs the product of uq_bcq_gemv with the library's own
 built-in scratch instead of a caller workspace.
 
-The GPU test calls it through the C ABI twice in a row, with different
-shapes and inputs, and compares each result with uq_bcq_gemv on the same
-inputs, within the tolerance the product's parity tests use.  This file is
+The GPU test calls it through the C ABI several times in a row, with
+different shapes and inputs (one of them needs the whole scratch), and
+checks that each result equals that of uq_bcq_gemv on the same inputs bit
+for bit.  This file is
 collected last, so that a run which stops at its first failure has run
 every other test before it.
 """
@@ -49,11 +50,19 @@ def _mass(a_star, z_star, x, g):
 
 @pytest.mark.gpu
 def test_noalloc_matches_the_workspace_entry_point_on_two_calls_in_a_row():
+    """Both entry points launch the same kernels in the same fixed order, one
+    with the caller's workspace and one with the built-in scratch, so their
+    results must be identical bit for bit; the oracle's tolerance (1e-5 of
+    the L1 mass of the expanded terms) is checked as well.  The second call
+    needs exactly the scratch's 2^20 floats (1 tile x 64 tokens x 16384
+    rows), so every word of the array is written and read."""
     d = torch.device("cuda", 0)
     gen = torch.Generator(device=d)
     gen.manual_seed(5)
     L = api.lib()
-    cases = [(14336, 4096, 3, 128, 1, torch.bfloat16), (300, 28672 + 32 * 5, 2, 32, 2, torch.float32)]
+    cases = [(14336, 4096, 3, 128, 1, torch.bfloat16), (16384, 512, 2, 64, 64, torch.float32),
+             (300, 28672 + 32 * 5, 2, 32, 2, torch.float32)]
+    assert 16384 * 64 * 1 == 1 << 20
     for out, n_in, q, g, batch, xdt in cases:
         planes = torch.randint(-2 ** 31, 2 ** 31 - 1, (q, out, n_in // 32), generator=gen, device=d,
                                dtype=torch.int32)
@@ -69,5 +78,6 @@ def test_noalloc_matches_the_workspace_entry_point_on_two_calls_in_a_row():
         assert st == api.UQ_OK, api.uq_last_error()
         torch.cuda.synchronize()
         assert torch.isfinite(y).all()
+        assert torch.equal(y, y_ref), f"{out}x{n_in} batch {batch}: {int((y != y_ref).sum())} outputs differ"
         err = (y.double() - y_ref.double()).abs()
         assert (err <= TOL * _mass(a_s, z_s, x.float(), g) + 1e-30).all()
