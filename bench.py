@@ -945,6 +945,110 @@ def run_reference(args):
     return line
 
 
+KERNELS = ("bwd", "fwd_remap", "fwd_keep", "export", "step", "omni_bwd", "awq_bwd", "gemv")
+
+
+def run_kernel(args):
+    """Profiling driver: one kernel of the path on one problem, for ncu.
+
+    Allocates a single problem of the headline shape (14336 x 4096 bf16,
+    about 1.5 GB on the device; 8192 x 28672 planes for the BCQ product),
+    launches the named call `--launches` times after one warm-up launch on
+    one stream and prints one JSON line with the CUDA-event time per launch.
+    The launch list of a capture is therefore short and known: launch 0 is
+    the warm-up, launches 1.. are the measured ones (for `step` every call
+    alternates a remapping and a keeping forward of t + 1).
+    """
+    import torch
+    from paper_2506_03781_gb300 import api, roofline, synth
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    wl = synth.WORKLOADS["mlp14336x4096_bf16"]
+    m = wl.matrices[0]
+    q, g = args.q, wl.g
+    out, n_in = m.out, m.n_in
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 * wl.seed + q)
+    name = args.kernel
+    if name == "gemv":
+        out, n_in = 8192, 28672
+        planes = torch.randint(-2 ** 31, 2 ** 31 - 1, (q, out, n_in // 32), generator=gen, device=dev,
+                               dtype=torch.int32)
+        a_s = torch.randn(out, n_in // g, q, generator=gen, device=dev) * 0.01
+        z_s = torch.randn(out, n_in // g, generator=gen, device=dev) * 0.003
+        x = torch.randn(1, n_in, generator=gen, device=dev).to(torch.bfloat16)
+        y = torch.empty(1, out, device=dev)
+        ws = api.bcq_gemv_workspace(out, n_in, 1, dev)
+        call = lambda i: api.uq_bcq_gemv(planes, a_s, z_s, x, y, g, workspace=ws, stream=stream)
+        nbytes = roofline.bytes_per_launch("gemv", out, n_in, q, g, 2)
+    elif name in ("omni_bwd", "awq_bwd"):
+        Wd = (torch.randn(out, n_in, generator=gen, device=dev) * 0.02).to(torch.bfloat16)
+        Gr = n_in // g
+        codes = torch.randint(0, 1 << q, (out, n_in), generator=gen, device=dev, dtype=torch.uint8)
+        Gup = torch.randn(out, n_in, generator=gen, device=dev) * 0.01
+        lv = torch.tensor([2.0 ** (q - 2 - j) for j in range(q)], device=dev)
+        alpha = (lv * (1 + 0.05 * torch.randn(out, Gr, q, generator=gen, device=dev))).contiguous()
+        zb = ((1 << q) - 1) / 2 + 0.1 * torch.randn(out, Gr, generator=gen, device=dev)
+        if name == "omni_bwd":
+            P = {"beta": 0.9 + 0.1 * torch.rand(out, Gr, generator=gen, device=dev),
+                 "gamma": 0.9 + 0.1 * torch.rand(out, Gr, generator=gen, device=dev), "alpha": alpha, "zb": zb}
+            gr = {"dbeta": torch.empty(out, Gr, device=dev), "dgamma": torch.empty(out, Gr, device=dev),
+                  "dalpha": torch.empty(out, Gr, q, device=dev), "dzb": torch.empty(out, Gr, device=dev)}
+            call = lambda i: api.uq_quantize_bwd_omni(Wd, q, g, P, codes, Gup, gr, stream=stream)
+        else:
+            P = {"sa": 0.5 + torch.rand(n_in, generator=gen, device=dev),
+                 "delta": torch.full((out, Gr), 0.01, device=dev), "za": torch.full((out, Gr), 3.5, device=dev),
+                 "alpha": alpha, "zb": zb}
+            gr = {"dsa": torch.empty(n_in, device=dev), "ddelta": torch.empty(out, Gr, device=dev),
+                  "dza": torch.empty(out, Gr, device=dev), "dalpha": torch.empty(out, Gr, q, device=dev),
+                  "dzb": torch.empty(out, Gr, device=dev)}
+            ws = torch.empty(max(api.uq_awq_bwd_workspace_bytes(out, n_in, q, g) // 4, 4), device=dev)
+            call = lambda i: api.uq_quantize_bwd_awq(Wd, q, g, P, codes, Gup, gr, workspace=ws, stream=stream)
+        nbytes = roofline.bytes_per_launch(name, out, n_in, q, g, 2)
+    else:
+        raw, _ = synth.workload_weights(wl, 0)
+        Wd = api.weights_tensor(raw, dev)
+        P = api.empty_params(out, n_in, q, g, dev)
+        codes = torch.empty(out, n_in, dtype=torch.uint8, device=dev)
+        api.uq_init_params(Wd, q, g, P, codes, G=wl.G, T=wl.T)
+        for k in ("delta", "s", "sr", "alpha"):
+            P[k].mul_(1.0 + wl.init_eps * torch.randn(P[k].shape, generator=gen, device=dev))
+        Gup = torch.randn(out, n_in, generator=gen, device=dev) * float(np.sqrt(wl.grad_var))
+        what = torch.empty(out, n_in, dtype=torch.float32, device=dev)
+        qz = api.Quantizer(Wd, q, g, P, codes, what, Gup, api.empty_grads(out, n_in, q, g, dev))
+        if name == "bwd":
+            call = lambda i: qz.bwd(stream=stream)
+        elif name == "fwd_remap":
+            call = lambda i: qz.fwd(0, wl.p, stream=stream)
+        elif name == "fwd_keep":
+            call = lambda i: qz.fwd(1, wl.p, stream=stream)
+        elif name == "step":
+            call = lambda i: qz.train_step(i, p_period=wl.p, stream=stream)
+        else:
+            ex = (torch.empty(q, out, n_in // 32, dtype=torch.int32, device=dev),
+                  torch.empty(out, n_in // g, q, device=dev), torch.empty(out, n_in // g, device=dev))
+            call = lambda i: qz.export(*ex, stream=stream)
+        kind = {"export": "export_reuse", "step": "step_keep"}.get(name, name)
+        nbytes = roofline.bytes_per_launch(kind, out, n_in, q, g, 2)
+    torch.cuda.synchronize()
+    call(0)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.launches)]
+    for i in range(args.launches):
+        ev[i][0].record(stream)
+        call(1 + i)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    api.uq_check_device(stream)
+    us = [a.elapsed_time(b) * 1e3 for a, b in ev]
+    res = {"kernel": name, "shape": [out, n_in], "q": q, "g": g, "launches": args.launches, "us": us,
+           "algorithmic_bytes": nbytes, "kernel_hash": kernel_hash()}
+    print(json.dumps(res))
+    return res
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -958,10 +1062,14 @@ def main(argv=None):
     ap.add_argument("--no-sweep", action="store_true", help="skip the q sweep of the headline matrix")
     ap.add_argument("--no-block", action="store_true", help="skip the block reconstruction loop timing")
     ap.add_argument("--workloads", action="store_true", help="time the other workloads instead")
+    ap.add_argument("--kernel", choices=KERNELS, help="profiling driver: one kernel on one problem (for ncu)")
+    ap.add_argument("--launches", type=int, default=2, help="measured launches of --kernel after one warm-up")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)          # at least 3 untimed warm-up steps
     if args.impl == "reference":
         return run_reference(args)
+    if args.kernel:
+        return run_kernel(args)
     if args.workloads:
         return run_workloads(args)
     return run_gpu(args)

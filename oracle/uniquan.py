@@ -47,7 +47,7 @@ __all__ = [
     "quantize_fwd_awq", "quantize_bwd_awq", "bwd_l1_mass_awq", "export_bcq_awq",
     "unify", "codes_eq4", "pack_bitplanes", "export_bcq", "export_bcq_half",
     "bcq_dequantize", "bcq_gemv",
-    "clip_params", "greedy_init", "general_alternating", "unified_init",
+    "clip_params", "greedy_init", "general_alternating", "init_error", "unified_init",
     "rtn",
 ]
 
@@ -812,6 +812,22 @@ def general_alternating(x, zb, G, T, q, trace=False):
     return alpha, zb, codes
 
 
+def init_error(w, delta, zu, alpha, zb):
+    """Candidate error of Algorithm 2, e' = ||w - w^||^2 per group (fp64 sum).
+
+    w [NG, g] fp32 groups; delta, zu, zb [NG]; alpha [NG, q].  w^ is the
+    quantizer output under these parameters with s = s_r = 1 and the full
+    mapping (reading R10): T_F, M_B over all 2^q levels, R_B, D_R.
+    """
+    w = np.asarray(w, F32)
+    NG, g = w.shape
+    x, _ = transform_F(w, np.ones((NG, g), F32), np.asarray(delta, F32), np.asarray(zu, F32), np.ones(NG, F32))
+    lv = levels(np.asarray(alpha, F32), np.asarray(zb, F32))
+    srt, cor, _ = sorted_levels(lv)
+    what = detransform(reconstruct(map_full(x, srt, cor), lv), np.asarray(delta, F32), np.asarray(zu, F32))
+    return ((w.astype(F64) - what.astype(F64)) ** 2).sum(-1)
+
+
 def unified_init(W, q, g, G=30, T=15, clip=CLIP_FIXED_MIN, return_errors=False):
     """Unified initialization (Algorithm 2) of every group of W [out, in].
 
@@ -831,7 +847,6 @@ def unified_init(W, q, g, G=30, T=15, clip=CLIP_FIXED_MIN, return_errors=False):
     Gr = n_in // g
     NG = out * Gr
     w = W.reshape(NG, g)
-    w64 = w.astype(F64)
     wm = w.min(-1)
     wM = w.max(-1)
     ones_g = np.ones((NG, g), F32)
@@ -847,10 +862,7 @@ def unified_init(W, q, g, G=30, T=15, clip=CLIP_FIXED_MIN, return_errors=False):
         d_c, zu_c = clip_params(wm, wM, gamma, q, clip)
         x, _ = transform_F(w, ones_g, d_c, zu_c, ones_r)
         a_c, zb_c, _ = general_alternating(x, best["zb"], G, T, q)
-        lv = levels(a_c, zb_c)
-        srt, cor, _ = sorted_levels(lv)
-        what = detransform(reconstruct(map_full(x, srt, cor), lv), d_c, zu_c)
-        e = ((w64 - what.astype(F64)) ** 2).sum(-1)
+        e = init_error(w, d_c, zu_c, a_c, zb_c)
         all_errs.append(e)
         acc = e < e_best
         best["delta"] = np.where(acc, d_c, best["delta"])

@@ -132,3 +132,57 @@ def boundary_weights(P, codes, g, seed, ulps=4):
 
 def slice_rows(P, rows):
     return {k: np.ascontiguousarray(np.asarray(v)[rows]) for k, v in P.items()}
+
+
+def check_init(W, q, g, G, clip, got, got_codes, ref, errs, chosen, label=""):
+    """Unified initialization (Algorithm 2 / Algorithm 3) on the GPU against
+    the oracle, with every group checked (reading R10/R11 criteria):
+
+    * the GPU's (Delta, z_U) must be one of the oracle's clipping candidates
+      (App. E.2) for gamma_i = i/G, which identifies the GPU's gamma index;
+    * the GPU's error e' -- recomputed by the oracle's own formula
+      (oracle.init_error) from the GPU's parameters -- must be within 1e-5
+      relative of the oracle's kept error;
+    * the gamma index must be the oracle's, except where the oracle's own
+      error for the GPU's candidate is within 1e-6 relative of its best (a
+      near-tie between candidates; counted and printed);
+    * the GPU's codes must be, bit for bit, the full mapping of T_F(w)
+      (s = s_r = 1) under the GPU's own parameters, in every group, so groups
+      with identical parameters have identical codes.
+
+    got: dict of the GPU's per-group parameters shaped like ref's; errs
+    [G, NG] and chosen [out, Gr] from oracle.unified_init(return_errors).
+    Returns the fraction of groups whose parameters are bit-identical."""
+    W = np.asarray(W, F32)
+    out, n_in = W.shape
+    NG = out * (n_in // g)
+    w = W.reshape(NG, g)
+    d_gpu, z_gpu = got["delta"].reshape(NG), got["zu"].reshape(NG)
+    a_gpu, zb_gpu = got["alpha"].reshape(NG, q), got["zb"].reshape(NG)
+    same = (d_gpu == ref["delta"].reshape(NG)) & (z_gpu == ref["zu"].reshape(NG)) & \
+        (zb_gpu == ref["zb"].reshape(NG)) & (a_gpu == ref["alpha"].reshape(NG, q)).all(-1)
+    wm, wM = w.min(-1), w.max(-1)
+    match = np.zeros((G, NG), bool)
+    for i in range(1, G + 1):
+        d_c, z_c = O.clip_params(wm, wM, F32(i) / F32(G), q, clip)
+        match[i - 1] = (d_c == d_gpu) & (z_c == z_gpu)
+    assert match.any(0).all(), f"{label}: {int((~match.any(0)).sum())} groups whose Delta, z_U is no candidate"
+    gi = match.argmax(0)
+    ch = np.asarray(chosen).reshape(NG)
+    cols = np.arange(NG)
+    e_best = errs[ch, cols]
+    e_gpu = O.init_error(w, d_gpu, z_gpu, a_gpu, zb_gpu)
+    rel = np.abs(e_gpu - e_best) / np.maximum(e_best, 1e-300)
+    assert (rel <= 1e-5).all(), f"{label}: {int((rel > 1e-5).sum())} groups with e' off by more than 1e-5 " \
+                                f"(worst {rel.max():.3e})"
+    moved = gi != ch
+    near = np.abs(errs[gi, cols] - e_best) <= 1e-6 * e_best
+    assert (near | ~moved).all(), f"{label}: {int((moved & ~near).sum())} groups took another gamma without a near-tie"
+    x, _ = O.transform_F(w, np.ones((NG, g), F32), d_gpu, z_gpu, np.ones(NG, F32))
+    srt, cor, _ = O.sorted_levels(O.levels(a_gpu, zb_gpu))
+    want = O.map_full(x, srt, cor)
+    bad = np.asarray(got_codes).reshape(NG, g).astype(np.int64) != want
+    assert not bad.any(), f"{label}: {int(bad.sum())} init codes are not the full mapping of the GPU's parameters"
+    print(f"init {label}: {same.mean():.6f} of {NG} groups bit-identical, {int(moved.sum())} near-tie gamma "
+          f"choices, worst e' rel diff {rel.max():.2e}")
+    return same.mean()

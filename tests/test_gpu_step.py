@@ -77,6 +77,7 @@ def check_against_oracle(raw, W, P, codes, Gup, q, g, t, mode, p, lr_F=LR_F, lr_
                                      codes, g, mode, t + 1, p)
     mism = c1 != r_codes
     n_mis = int(mism.sum())
+    print(f"step parity {label}: {n_mis} of {c1.size} codes differ from the oracle ({n_mis / c1.size:.2e})")
     if n_mis:
         assert n_mis <= max_tie_frac * c1.size, f"{label}: {n_mis} code mismatches"
         assert_near_ties(W, ref, tol, c1, r_codes, mism, g, label)

@@ -40,7 +40,7 @@ def setup_matrix(wl, idx, rows, q=None):
     p = api.empty_params(m.out, m.n_in, q, g, d)
     codes = torch.empty(m.out, m.n_in, dtype=torch.uint8, device=d)
     api.uq_init_params(Wd, q, g, p, codes, G=wl.G, T=wl.T)
-    init_rows = O.unified_init(W[rows], q, g, G=wl.G, T=wl.T)
+    init_rows, errs, chosen = O.unified_init(W[rows], q, g, G=wl.G, T=wl.T, return_errors=True)
     full = {k: C.host(v).copy() for k, v in p.items()}
     gpu_init_rows = {k: full[k][rows].copy() for k in PK}
     gpu_codes_rows = C.host(codes)[rows].copy()
@@ -51,15 +51,15 @@ def setup_matrix(wl, idx, rows, q=None):
     fac = synth.perturb_factors(synth.param_shapes(m.out, m.n_in, g, q), wl.init_eps, (wl.seed, idx, q))
     P = synth.jitter(full, fac)
     return dict(raw=raw, W=W, Wd=Wd, P=P, codes=c_full, init_rows=init_rows, gpu_init_rows=gpu_init_rows,
-                gpu_codes_rows=gpu_codes_rows, q=q, g=g, out=m.out, n_in=m.n_in)
+                gpu_codes_rows=gpu_codes_rows, q=q, g=g, out=m.out, n_in=m.n_in, rows=rows, errs=errs,
+                chosen=chosen, G=wl.G, label=m.name)
 
 
 def init_agreement(s):
-    same = np.ones(s["init_rows"]["delta"].shape, bool)
-    for k in ("delta", "zu", "zb"):
-        same &= s["gpu_init_rows"][k] == s["init_rows"][k]
-    same &= (s["gpu_init_rows"]["alpha"] == s["init_rows"]["alpha"]).all(-1)
-    return same.mean()
+    """Every sampled group checked against the oracle (C.check_init); returns
+    the fraction of groups with bit-identical parameters."""
+    return C.check_init(s["W"][s["rows"]], s["q"], s["g"], s["G"], api.CLIP_FIXED_MIN, s["gpu_init_rows"],
+                        s["gpu_codes_rows"], s["init_rows"], s["errs"], s["chosen"], f"{s['label']} q={s['q']}")
 
 
 def run_and_compare(s, rows, steps=(0,), step_eps=0.0, seed=0, export=True, label=""):

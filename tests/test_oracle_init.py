@@ -168,3 +168,82 @@ def test_hyperparameter_defaults_follow_paper():
     assert wl.p == hp["remapping_period_p"]
     assert wl.G in hp["grid_search_iterations_G"]
     assert hp["clipping_strategy"] == "Fixed-minimum" and O.CLIP_FIXED_MIN == 0
+
+
+@pytest.mark.parametrize("q", [2, 3, 4])
+def test_singular_gram_matrix_leaves_alpha_unchanged(q):
+    """Reading R11 for the alpha step of Algorithm 3: when C^T C is exactly
+    singular, alpha keeps its value from before the round.  A group whose
+    transformed weights all equal z_B - a makes the greedy start pick
+    c_1 = -1 everywhere with alpha_1 = a, after which the residual is exactly
+    zero and every further bit is +1 with alpha_j = 0: the columns of C are
+    +-1 multiples of each other, so C^T C is singular.  Its neighbour in the
+    same batch (ordinary weights) is regular and must move.  A pseudo-inverse
+    solve, a reset of alpha or an inverted test would each change the
+    singular group's alpha and fail here (checked below for the
+    pseudo-inverse)."""
+    g, a = 64, F32(0.75)
+    zb = np.full(2, F32(((1 << q) - 1) / 2), F32)
+    x = np.empty((2, g), F32)
+    x[0] = zb[0] - a
+    x[1] = groups(90, n=1, g=g)[0] * F32(100) + zb[1]
+    a0, c0 = O.greedy_init(x, zb, q)
+    assert np.array_equal(a0[0], np.array([a] + [0.0] * (q - 1), F32))
+    C = O.signs(q, F64)[c0[0]]
+    assert np.linalg.matrix_rank(C.T @ C) < q                      # singular (integer Gram matrix)
+    a1, zb1, c1 = O.general_alternating(x, zb, 2, 1, q)
+    assert np.array_equal(a1[0], a0[0])                           # bit-identical: left unchanged
+    assert not np.array_equal(a1[1], a0[1])                       # the regular neighbour moved
+    # the minimum-norm least-squares alpha differs from the kept one
+    pinv = np.linalg.pinv(C) @ (x[0].astype(F64) - zb[0])
+    assert not np.allclose(pinv, a0[0].astype(F64))
+    # later rounds stay singular and keep alpha: T = 15 ends where the greedy start did
+    a15, _, c15 = O.general_alternating(x, zb, 2, 15, q)
+    assert np.array_equal(a15[0], a0[0])
+
+
+@pytest.mark.parametrize("clip", [O.CLIP_FIXED_MIN, O.CLIP_FIXED_MAX, O.CLIP_BALANCED])
+def test_constant_group_initializes_to_the_kept_greedy_alpha(clip):
+    """A constant weight group (w_M = w_m): T_F maps every weight to the same
+    x, so the greedy start takes alpha_1 = |x - z_B| with one sign for every
+    weight, leaves an exactly zero residual, and sets every further bit to +1
+    with alpha_j = 0.  The Gram matrix is singular in every round, so the kept
+    alpha is the greedy one, bit for bit, and every weight takes one code
+    word.  Under Fixed-minimum, x is exactly 0 (u and -z_U are the same
+    quotient), so alpha = (z_B, 0, ..., 0) = (3.5, 0, 0) and the code word is
+    0 (c_1 = -1; ties between equal levels go to the smaller code word)."""
+    q, g = 3, 128
+    W = groups(41, n=4, g=g).reshape(4, g)
+    W[1] = F32(0.0123)
+    W[2] = F32(-0.5)
+    res = O.unified_init(W, q, g, G=5, T=4, clip=clip)
+    for r in (1, 2):
+        x, _ = O.transform_F(W[r][None], np.ones((1, g), F32), res["delta"][r], res["zu"][r], np.ones(1, F32))
+        assert np.all(x == x[0, 0])
+        r0 = np.abs(x[0, 0] - F32(3.5))
+        assert np.array_equal(res["alpha"][r, 0], np.array([r0, 0.0, 0.0], F32)), res["alpha"][r]
+        assert np.all(res["codes"][r] == res["codes"][r, 0])
+        assert res["zb"][r, 0] == F32(3.5)
+        if clip == O.CLIP_FIXED_MIN:
+            assert x[0, 0] == 0 and r0 == F32(3.5) and np.all(res["codes"][r] == 0)
+
+
+def test_init_error_is_the_quantizer_error_under_full_mapping():
+    """init_error equals ||w - w^||^2 with w^ from quantize_fwd (full mapping,
+    s = s_r = 1) -- a different code path through the same definitions --
+    and is the error unified_init keeps for its chosen candidate."""
+    q, g = 3, 64
+    W = groups(42, n=6, g=g * 4).reshape(6, g * 4)
+    res, errs, chosen = O.unified_init(W, q, g, G=6, T=3, return_errors=True)
+    NG = W.size // g
+    e = O.init_error(W.reshape(NG, g), res["delta"].reshape(-1), res["zu"].reshape(-1),
+                     res["alpha"].reshape(NG, q), res["zb"].reshape(-1))
+    what, _ = O.quantize_fwd(W, res["s"], res["sr"], res["delta"], res["zu"], res["alpha"], res["zb"], None, g,
+                             mode=O.MAP_FULL)
+    direct = ((W.astype(F64) - what.astype(F64)) ** 2).reshape(NG, g).sum(-1)
+    assert np.array_equal(e, direct)
+    assert np.array_equal(e, errs[chosen.reshape(-1), np.arange(NG)])
+    # the kept candidate is the first strictly smallest error
+    assert np.all(errs[chosen.reshape(-1), np.arange(NG)] == errs.min(0))
+    first = np.argmax(errs == errs.min(0)[None], axis=0)
+    assert np.array_equal(first, chosen.reshape(-1))
