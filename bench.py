@@ -187,6 +187,83 @@ def oracle_sample_inputs(wl, q, rows, row0=0):
     return W, P, init["codes"], Gup
 
 
+def parity_sample(wl, q, rows, Wd, P_dev, codes_dev, Gup_dev, dev, stream):
+    """Parity counters of the timed kernels (part of the CPU-baseline leg).
+
+    The oracle's inputs for the first `rows` rows (its own unified
+    initialization, the seeded jitter and dL/dW^ of oracle_sample_inputs)
+    replace those rows of copies of the benchmark's device buffers; the GPU
+    then runs the timed calls over the WHOLE matrix in the timed launch
+    configuration -- the forward of a remap step (t = 0) and its backward,
+    the forward of a keep step (t = 1), and one fused step (t = 1, whose
+    forward of t + 1 remaps) -- and the sampled rows are compared with the
+    oracle: codes and W^ bit for bit (mismatches counted), gradients and
+    updated parameters as the worst ratio of error to tolerance (1e-4 of the
+    fp64 L1 mass; for the fused step lr times that plus two fp32 ulps)."""
+    import torch
+    import oracle as O
+    from paper_2506_03781_gb300 import api
+    g = wl.g
+    W, P, codes0, Gup = oracle_sample_inputs(wl, q, rows)
+    Pd = {k: v.clone() for k, v in P_dev.items()}
+    for k in Pd:
+        Pd[k][:rows].copy_(torch.from_numpy(np.ascontiguousarray(P[k])))
+    cd = codes_dev.clone()
+    cd[:rows].copy_(torch.from_numpy(codes0))
+    Gd = Gup_dev.clone()
+    Gd[:rows].copy_(torch.from_numpy(Gup))
+    what = torch.empty_like(Gd)
+    out, n_in = Gd.shape
+    gr = api.empty_grads(out, n_in, q, g, dev)
+    args = lambda Q: (W, Q["s"], Q["sr"], Q["delta"], Q["zu"], Q["alpha"], Q["zb"])
+    host = lambda t: t[:rows].cpu().numpy()
+
+    def grad_ratio(ref, mass):
+        worst = 0.0
+        for k in ("ddelta", "dzu", "dzb", "dalpha", "dsr"):
+            err = np.abs(host(gr[k]).astype(np.float64) - ref[k])
+            worst = max(worst, float((err / (1e-4 * mass[k] + 1e-30)).max()))
+        ds = ref["ds"]
+        err = np.abs(host(gr["ds"]).astype(np.float64) - ds)
+        worst = max(worst, float((err / (1e-4 * np.maximum(np.abs(ds), 1e-6 * np.abs(ds).max()))).max()))
+        return worst
+
+    res = {"rows": rows, "weights": rows * n_in,
+           "inputs": "the oracle's own init of the first rows (G=2, T=2), seeded jitter and dL/dW^; the GPU runs "
+                     "the whole matrix in the timed launch configuration"}
+    api.uq_quantize_fwd(Wd, q, g, Pd, cd, what, api.MAP_LOCAL_PERIODIC, 0, wl.p, stream=stream)
+    api.uq_quantize_bwd(Wd, q, g, Pd, cd, Gd, gr, stream=stream)
+    torch.cuda.synchronize()
+    r_what, r_codes = O.quantize_fwd(*args(P), codes0, g, O.MAP_LOCAL_PERIODIC, 0, wl.p)
+    ref = O.quantize_bwd(*args(P), r_codes, Gup, g)
+    mass = O.bwd_l1_mass(*args(P), r_codes, Gup, g)
+    res["fwd_remap"] = {"codes_mismatch": int((host(cd) != r_codes).sum()),
+                        "what_mismatch": int((host(what) != r_what).sum()),
+                        "codes_moved": int((r_codes != codes0).sum())}
+    res["bwd"] = {"grad_worst_frac_of_tol": grad_ratio(ref, mass)}
+    api.uq_quantize_fwd(Wd, q, g, Pd, cd, what, api.MAP_LOCAL_PERIODIC, 1, wl.p, stream=stream)
+    torch.cuda.synchronize()
+    k_what, _ = O.quantize_fwd(*args(P), r_codes, g, O.MAP_LOCAL_PERIODIC, 1, wl.p)
+    res["fwd_keep"] = {"codes_mismatch": int((host(cd) != r_codes).sum()),
+                       "what_mismatch": int((host(what) != k_what).sum())}
+    api.uq_train_step(Wd, q, g, Pd, cd, Gd, what, 1, stream=stream)
+    torch.cuda.synchronize()
+    new, c2, w2 = O.train_step(*args(P), r_codes, Gup, g, 1)
+    worst = 0.0
+    gname = {"delta": "ddelta", "zu": "dzu", "s": "ds", "sr": "dsr", "alpha": "dalpha", "zb": "dzb"}
+    for k in ("delta", "zu", "s", "sr", "alpha", "zb"):
+        lr = O.LR_F if k in ("delta", "zu", "s", "sr") else O.LR_B
+        gm = mass[gname[k]] if k != "s" else np.maximum(np.abs(ref["ds"]), 1e-6 * np.abs(ref["ds"]).max())
+        tol = (lr * 1e-4 * gm + 2 * np.spacing(np.abs(new[k]).astype(np.float32))
+               + np.spacing(np.abs(lr * ref[gname[k]]).astype(np.float32)))
+        err = np.abs(host(Pd[k]).astype(np.float64) - new[k])
+        worst = max(worst, float((err / tol).max()))
+    res["train_step"] = {"codes_mismatch": int((host(cd) != c2).sum()), "param_worst_frac_of_tol": worst}
+    del Pd, cd, Gd, what, gr
+    torch.cuda.empty_cache()
+    return res
+
+
 def time_oracle_step(wl, q, rows, budget_s, row0=0, barrier=None):
     """Runs oracle steps (fwd at step t + bwd) until budget_s elapses; returns
     (weights per second, steps run, seconds).  With a barrier, the timed loop
@@ -456,15 +533,18 @@ def time_link(hp, hin, hout, reps=3):
             "copy_ceiling_weights_per_s": hs.out * hs.n_in / t_both}
 
 
-def time_block_step(dev, steps=20, warmup=4, samples=4):
+def time_block_step(dev, steps=20, warmup=4, samples=4, idx_steps=64):
     """Algorithm 1 on a Llama-3-8B-shaped block (seq 2048, bf16 block
     compute, the block workload's q and g): ms per optimisation step (block
     forward + backward in torch, then uq_train_step for the seven weights),
-    the quantizer's share of it, and the share of codes a remap step moves."""
+    the quantizer's share of it, the share of codes a remap step moves, and,
+    over `idx_steps` further untimed steps, the index-change statistics of
+    the paper's Table 2 (shares of weights whose level index moves by 0, 1,
+    2, >2 in one step and over the whole run) and the loss of every step."""
     import time
     import torch
     from paper_2506_03781_gb300 import api, synth
-    from paper_2506_03781_gb300.recon import NAMES, BlockReconstructor
+    from paper_2506_03781_gb300.recon import NAMES, BlockReconstructor, index_change_shares
     wl = synth.WORKLOADS["llama3_8b_block_bf16"]
     shape = synth.BLOCKS["llama3_8b"]
     Wb = synth.block_weights(shape, wl.seed)
@@ -508,6 +588,25 @@ def time_block_step(dev, steps=20, warmup=4, samples=4):
         if remap:
             ch = sum(int((rec.codes[n] != before[n]).sum()) for n in NAMES)
             moved.append(ch / sum(rec.codes[n].numel() for n in NAMES))
+    # Table 2 (index changes) and the reconstruction-error curve (Fig. 5b): idx_steps
+    # further steps from here, the level index of every weight after each one
+    r0 = torch.cat([r.view(-1) for r in rec.ranks().values()])
+    prev, per_step, curve = r0, [], []
+    for i in range(idx_steps):
+        curve.append(rec.step(Y[i % samples], Xhd[i % samples]))
+        r = torch.cat([r.view(-1) for r in rec.ranks().values()])
+        per_step.append(index_change_shares(r, prev))
+        prev = r
+    index_change = {
+        "bins": ["0", "1", "2", ">2"],
+        "single_step_mean": [statistics.mean(s[k] for s in per_step) for k in range(4)],
+        "single_step_max_moved": max(1.0 - s[0] for s in per_step),
+        "all_steps": index_change_shares(prev, r0),
+        "steps": idx_steps,
+        "learning_rates": [rec.lr_F, rec.lr_B],
+        "paper_llama3_8b": {"single_step": [0.9997, 0.0001, 0.0, 0.0001],
+                            "all_steps_2560": [0.8930, 0.0837, 0.0136, 0.0097]},
+    }
     api.uq_check_device(stream)
     n_w = sum(rec.codes[n].numel() for n in NAMES)
     res = {"block": shape.name, "seq": shape.seq, "q": wl.q, "g": wl.g, "weights": n_w, "steps": steps,
@@ -517,6 +616,9 @@ def time_block_step(dev, steps=20, warmup=4, samples=4):
            "loss_per_epoch": [float(torch.stack(losses[k:k + samples]).mean())
                               for k in range(0, len(losses) - samples + 1, samples)],
            "init_s": init_s,
+           "index_change": index_change,
+           # loss of every step of the index-change run (the reconstruction-error curve)
+           "loss_curve": [float(v) for v in torch.stack(curve)] if curve else [],
            "paper_step_s_a100_derived": 0.25}
     del rec, Y, Xd, Xhd
     torch.cuda.empty_cache()
@@ -770,13 +872,14 @@ def run_gpu(args):
 
     result = None
     if rank == 0:
-        cpu = cpu_all = None
+        cpu = cpu_all = parity = None
         if world == 1 and not args.no_cpu_baseline:
             rows = 96
             v, n, el = time_oracle_step(wl, q, rows, args.cpu_budget)
             cpu = {"value": v, "unit": "weights/s", "cores": 1, "kind": "oracle",
                    "sample": f"first {rows} rows of {out}x{n_in} ({rows * n_in} weights), {n} oracle steps "
                              f"(local remap/keep alternating + backward) in {el:.1f} s, numpy single thread"}
+            parity = parity_sample(wl, q, rows, Wd, ring[0], codes, Gup, dev, stream)
             workers = max(1, min(cpu_cores(), out // rows))
             vp, elp = time_oracle_parallel(wl, q, rows, args.cpu_budget, workers)
             if vp is not None:
@@ -830,6 +933,7 @@ def run_gpu(args):
             "clocks": clocks,
             "cpu_baseline": cpu,
             "cpu_baseline_all_cores": cpu_all,
+            "parity": parity,
         }
         print(json.dumps(result))
     if world > 1:

@@ -326,7 +326,9 @@ uq_status uq_quantize_fwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int6
  * ds_A sums over every row of its column: per-row-range partials go to
  * `workspace` (caller-owned device memory of at least
  * uq_awq_bwd_workspace_bytes(out, in, q, g) bytes, overwritten) and are
- * summed in range order.  fp32, deterministic.  A too small workspace is
+ * summed in a fixed order (eight contiguous slices of the ranges, each in
+ * range order, then the slices in order).  fp32, deterministic.  A too
+ * small workspace is
  * UQ_ERR_ARG.
  */
 uq_status uq_quantize_bwd_awq(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,

@@ -439,7 +439,8 @@ static cudaError_t awq_stream_fwd(int mode, const Shape& sh, const void* W, uq_p
 // every warp of a block owns one fixed unit (one set of columns) for the
 // whole kernel, so its ds_A partials and 1/s_A stay in registers across all
 // of its rows; at the end each (block, row slot) writes one row of partials
-// to the workspace [grid * R][in], summed in that order by awq_colsum_kernel.
+// to the workspace [grid * R][in], summed by awq_colsum_kernel in a fixed
+// order (contiguous slices of the rows in order, then the slices in order).
 // Deterministic for a given grid.  The stage holds W, s_A of the unit's
 // columns (s slot), dL/dW^, the codes and Delta_A, z_A, z_B, alpha.
 
@@ -660,13 +661,28 @@ cudaError_t awq_error(bool clear, unsigned int* flag) {
     return e;
 }
 
-// ds_A[col] = sum over the row ranges of PART[range, col], in range order.
-__global__ void __launch_bounds__(256)
+// ds_A[col] = sum over the row ranges of PART[range, col] in a fixed order:
+// a block owns 32 columns; its 8 warps each sum one contiguous slice of the
+// ranges (ascending, one coalesced 128-byte row piece per load), and the 8
+// slice sums are added in slice order.  Deterministic, no atomics.
+constexpr int kColsumSlices = 8;
+__global__ void __launch_bounds__(32 * kColsumSlices)
 awq_colsum_kernel(const float* __restrict__ PART, float* __restrict__ DSA, int n_in, int ranges) {
-    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < n_in; c += gridDim.x * blockDim.x) {
-        float acc = 0.f;
-        for (int r = 0; r < ranges; ++r) acc += __ldg(PART + (int64_t)r * n_in + c);
-        DSA[c] = acc;
+    __shared__ float part[kColsumSlices][32];
+    const int lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
+    const int c = blockIdx.x * 32 + lane;
+    const int per = (ranges + kColsumSlices - 1) / kColsumSlices;
+    const int r0 = slice * per, r1 = r0 + per < ranges ? r0 + per : ranges;
+    float acc = 0.f;
+    if (c < n_in)
+        for (int r = r0; r < r1; ++r) acc += __ldg(PART + (int64_t)r * n_in + c);
+    part[slice][lane] = acc;
+    __syncthreads();
+    if (slice == 0 && c < n_in) {
+        float tot = part[0][lane];
+#pragma unroll
+        for (int k = 1; k < kColsumSlices; ++k) tot += part[k][lane];
+        DSA[c] = tot;
     }
 }
 
@@ -711,7 +727,7 @@ static cudaError_t run_awq_stream_bwd(const Shape& sh, const void* W, uq_params_
                                       gr.dalpha, gr.dzb, work, sh.out, sh.n_in, R, n_rb);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    awq_colsum_kernel<<<(sh.n_in + 255) / 256, 256, 0, st>>>(work, gr.dsa, sh.n_in, grid * R);
+    awq_colsum_kernel<<<(sh.n_in + 31) / 32, 32 * kColsumSlices, 0, st>>>(work, gr.dsa, sh.n_in, grid * R);
     return cudaGetLastError();
 }
 
@@ -736,8 +752,7 @@ static cudaError_t awq_lpg(bool bwd, int mode, const Shape& sh, const void* W, u
                                                              sh.n_in, sh.g, rpr);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        int blocks = (sh.n_in + 255) / 256;
-        awq_colsum_kernel<<<blocks, 256, 0, st>>>(work, gr.dsa, sh.n_in, (int)ranges);
+        awq_colsum_kernel<<<(sh.n_in + 31) / 32, 32 * kColsumSlices, 0, st>>>(work, gr.dsa, sh.n_in, (int)ranges);
         return cudaGetLastError();
     }
     if (mode == FWD_KEEP)

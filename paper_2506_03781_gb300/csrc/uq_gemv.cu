@@ -432,6 +432,238 @@ bcq_gemv_tma_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_
     }
 }
 
+// ---------------------------------------------------------------------------
+// Wide-lane variant (in a multiple of 1024, g in {32, 64, 128, 256})
+// ---------------------------------------------------------------------------
+//
+// Tiles of 1024 columns; lane l owns columns 32 l .. 32 l + 31 of the tile,
+// i.e. one whole plane word per (row, plane).  Its four bytes index four
+// lookup tables (one per 8 columns), so a plane word costs one shared load,
+// four table lookups and three adds, and the per-row work (parameters, the
+// reduction over the warp) is spread over 32 q weights per lane instead of 16 q.
+//
+// The tables of a tile take 128 KB: [pair p][entry v][slot s][lane l] floats,
+// byte slot k = 2 p + s, so that entry v sits at byte offset 256 v and lane l
+// at 4 l.  The table is placed at a shared-memory address L that is a
+// multiple of 65536: the byte address of entry v for lane l is then
+// L + 256 v + 4 l + (65536 p + 128 s), and one byte permutation (PRMT) of
+// the plane word with the per-lane constant L + 4 l puts the word's byte k
+// into bits 8..15 of that address; the constant part is the load's
+// immediate offset.  The rest of shared memory -- x of the tile (lane-major,
+// stride 33 floats: conflict-free table build), the mbarriers and the
+// stages -- fills the space below L first, then the space after the tables;
+// the host requests enough bytes for any position of the dynamic base.
+//
+// Each warp runs its own ring of NS stages; lane 0 fills a stage with three
+// tensor copies (planes {32 words, 8 rows, q}, alpha* {NGT q, 8 rows}, z*
+// {NGT, 8 rows}) completing on the stage's mbarrier.  Rows past `out` read
+// as zeros and give zero partials that are never stored, so no row needs a
+// validity test.  Waits are bounded as in bcq_gemv_tma_kernel.
+
+constexpr int kWideCols = 1024;                   // columns per tile: 32 lanes x 32
+constexpr int kWideWords = kWideCols / 32;        // plane words per tile and row
+constexpr uint32_t kWideLutBytes = 4u * 256u * 32u * 4u;
+constexpr int kWideXsStride = 33;
+constexpr int kWideXsBytes = 32 * kWideXsStride * 4;
+constexpr int kWideMaxWarps = 16;
+constexpr int kWideStages = 2;
+constexpr int kWideHeadBytes = align_up(kWideXsBytes + kWideMaxWarps * kWideStages * 8, 128);   // x + mbarriers
+constexpr int kSmemOptIn = 227 * 1024;
+constexpr int kWideLutRows = 64;                  // a table build costs about as much as 64 rows
+
+// Groups of one row inside one wide tile.
+__host__ __device__ constexpr int wide_tile_groups(int g) { return kWideCols / g; }
+// Bytes of one stage: 8 rows x (q planes x 32 words + the tile's alpha* and z*).
+__host__ __device__ constexpr int wide_stage_bytes(int q, int ngt) {
+    return kBatchRows * (q * kWideWords + ngt * (q + 1)) * 4;
+}
+// Slack for the part of the space below the tables that cannot be used (at
+// most one stage, or the head when the gap is smaller than the head).
+__host__ __device__ constexpr int wide_slack(int q, int ngt) {
+    return (wide_stage_bytes(q, ngt) > kWideHeadBytes ? wide_stage_bytes(q, ngt) : kWideHeadBytes) + 128;
+}
+// Warps per block: as many as fit two stages each next to the tables (at most 16).
+__host__ __device__ constexpr int wide_warps(int q, int ngt) {
+    return (int)((kSmemOptIn - (int)kWideLutBytes - kWideHeadBytes - wide_slack(q, ngt)) /
+                 (kWideStages * wide_stage_bytes(q, ngt))) > kWideMaxWarps
+               ? kWideMaxWarps
+               : (int)((kSmemOptIn - (int)kWideLutBytes - kWideHeadBytes - wide_slack(q, ngt)) /
+                       (kWideStages * wide_stage_bytes(q, ngt)));
+}
+__host__ __device__ constexpr int wide_smem_bytes(int q, int ngt) {
+    return (int)kWideLutBytes + kWideHeadBytes + wide_slack(q, ngt) +
+           wide_warps(q, ngt) * kWideStages * wide_stage_bytes(q, ngt);
+}
+
+// Index of the lowest set bit of n (1 <= n <= 15).
+__host__ __device__ constexpr int low_bit(int n) { return (n & 1) ? 0 : (n & 2) ? 1 : (n & 4) ? 2 : 3; }
+
+__device__ __forceinline__ uint32_t lds_u32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ float lds_f32(uint32_t a) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a));
+    return v;
+}
+
+template <int Q, typename XT, int NGT>
+__global__ void __launch_bounds__(kWideMaxWarps * 32, 1)
+bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_constant__ CUtensorMap tm_alpha,
+                     const __grid_constant__ CUtensorMap tm_z, const void* __restrict__ X, float* __restrict__ PART,
+                     int64_t out, int n_in, int batch, int n_tiles, int64_t rows_per_block) {
+    constexpr int NW = wide_warps(Q, NGT);
+    constexpr int NS = kWideStages;
+    constexpr int SB = wide_stage_bytes(Q, NGT);
+    constexpr int PLB = Q * kBatchRows * kWideWords * 4;       // planes of a stage
+    constexpr int ALB = kBatchRows * NGT * Q * 4;              // alpha* of a stage
+    constexpr int DYN = wide_smem_bytes(Q, NGT);
+    constexpr int LPG = 32 / NGT;                              // lanes per group
+    static_assert(NW >= 4 && SB % 128 == 0 && DYN <= kSmemOptIn, "wide layout");
+    static_assert(NGT >= 4 && (NGT * Q * 4) % 16 == 0, "alpha* and z* boxes must span a multiple of 16 bytes");
+    extern __shared__ __align__(128) unsigned char wsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t = (int)(blockIdx.x % n_tiles);
+    const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
+    const int nr = (int)(out - r0 < rows_per_block ? out - r0 : rows_per_block);
+    if (nr <= 0) return;                                       // the whole block: before any barrier
+
+    // shared-memory layout (uniform over the block)
+    const uint32_t D = tma::smem_addr(wsm);
+    const uint32_t L = (D + 0xFFFFu) & ~0xFFFFu;
+    uint32_t lo = (D + 127u) & ~127u, hi = L + kWideLutBytes;
+    uint32_t head;
+    if (L >= lo + (uint32_t)kWideHeadBytes) { head = lo; lo += kWideHeadBytes; }
+    else { head = hi; hi += kWideHeadBytes; }
+    const uint32_t n_gap = L > lo ? (L - lo) / SB : 0u;
+    if (hi + ((uint32_t)(NW * NS) > n_gap ? (uint32_t)(NW * NS) - n_gap : 0u) * SB > D + DYN) {
+        if (threadIdx.x == 0) atomicOr(&g_gemv_err, 4u);       // cannot happen: the host sized DYN for any D
+        return;
+    }
+    float* xs = reinterpret_cast<float*>(wsm + (head - D));
+    float* lut = reinterpret_cast<float*>(wsm + (L - D));
+    const uint32_t bar0 = head + (uint32_t)kWideXsBytes + (uint32_t)(warp * NS * 8);
+    static_assert(NS == 2, "two stages per warp, held in two registers");
+    const uint32_t i0 = (uint32_t)(warp * NS), i1 = i0 + 1u;
+    const uint32_t st0 = i0 < n_gap ? lo + i0 * SB : hi + (i0 - n_gap) * SB;
+    const uint32_t st1 = i1 < n_gap ? lo + i1 * SB : hi + (i1 - n_gap) * SB;
+
+    const int c0 = t * kWideCols;
+    const int nbat = (nr + kBatchRows - 1) / kBatchRows;
+    const int my_nb = warp < nbat ? (nbat - warp + NW - 1) / NW : 0;
+    const uint32_t lane_base = L + 4u * (uint32_t)lane;        // bits 8..15 are zero
+    const int gl = lane / LPG;                                 // this lane's group within the tile
+    using SR = SegReduce<32>;
+
+    if (lane == 0) {
+#pragma unroll
+        for (int s = 0; s < NS; ++s) tma::bar_init(bar0 + 8u * s, 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+
+    const int total = batch * my_nb;                           // items: token-major, this warp's batches
+    int issued = 0, waited = 0, ik = 0;
+    auto issue_next = [&]() {                                  // lane 0 only
+        const int s = issued & 1;
+        const uint32_t bar = bar0 + 8u * s;
+        const uint32_t d = s ? st1 : st0;
+        const int y = (int)(r0 + (int64_t)kBatchRows * (warp + NW * ik));
+        tma::fence_async_smem();                               // the warp's reads of this stage come first
+        tma::bar_arrive_tx(bar, (uint32_t)SB);
+        tmap::load_3d(d, &tm_planes, t * kWideWords, y, 0, bar);
+        tmap::load_2d(d + PLB, &tm_alpha, t * NGT * Q, y, bar);
+        tmap::load_2d(d + PLB + ALB, &tm_z, t * NGT, y, bar);
+        ++issued;
+        if (++ik == my_nb) ik = 0;
+    };
+    if (lane == 0)
+        while (issued < total && issued < NS) issue_next();
+
+    bool alive = true;
+    for (int b = 0; b < batch; ++b) {                          // token b is row b of X
+        __syncthreads();                                       // the previous token's readers are done
+        for (int i = threadIdx.x; i < kWideCols; i += NW * 32)
+            xs[kWideXsStride * (i >> 5) + (i & 31)] = XT::get(X, (int64_t)b * n_in + c0 + i);
+        __syncthreads();
+        // tables: item (lane l, slot k, high nibble m) writes entries 16 m + n, n = 0..15
+        for (int it = threadIdx.x; it < 2048; it += NW * 32) {
+            const int l = it & 31, k = (it >> 5) & 3, m = it >> 7;
+            const float* xc = xs + kWideXsStride * l + 8 * k;
+            float x[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) x[i] = xc[i];
+            float lo4[16];
+            lo4[0] = 0.f;
+#pragma unroll
+            for (int n = 1; n < 16; ++n) lo4[n] = __fadd_rn(lo4[n & (n - 1)], x[low_bit(n)]);
+            float h = (m & 1) ? x[4] : 0.f;
+            h = (m & 2) ? __fadd_rn(h, x[5]) : h;
+            h = (m & 4) ? __fadd_rn(h, x[6]) : h;
+            h = (m & 8) ? __fadd_rn(h, x[7]) : h;
+            float* dst = lut + (k >> 1) * 16384 + (k & 1) * 32 + l + 16 * m * 64;
+#pragma unroll
+            for (int n = 0; n < 16; ++n) dst[n * 64] = __fadd_rn(lo4[n], h);
+        }
+        __syncthreads();
+        // S = the sum of this lane's 32 x values (entry 255 of each slot)
+        const float S = __fadd_rn(__fadd_rn(lds_f32(lane_base + 255u * 256u), lds_f32(lane_base + 255u * 256u + 128u)),
+                                  __fadd_rn(lds_f32(lane_base + 65536u + 255u * 256u),
+                                            lds_f32(lane_base + 65536u + 255u * 256u + 128u)));
+        float* prow = PART + ((int64_t)t * batch + b) * out + r0;
+        for (int k = 0; k < my_nb; ++k) {
+            const int i = b * my_nb + k;
+            const int s = i & 1;
+            const uint32_t sa = s ? st1 : st0;
+            if (alive) {
+                // one verdict for the whole warp (lanes poll the mbarrier separately)
+                if (__all_sync(kFull, tma::bar_wait(bar0 + 8u * s, (uint32_t)((i >> 1) & 1)))) {
+                    ++waited;
+                } else {
+                    alive = false;
+                    if (lane == 0) atomicOr(&g_gemv_err, 1u);
+                }
+            }
+            if (alive) {
+                const uint32_t pw = sa + 4u * (uint32_t)lane;                          // this lane's plane words
+                const uint32_t pa = sa + PLB + 4u * (uint32_t)(gl * Q);               // its group's alpha*
+                const uint32_t pz = sa + PLB + ALB + 4u * (uint32_t)gl;               // and z*
+                float v[kBatchRows];
+#pragma unroll
+                for (int rr = 0; rr < kBatchRows; ++rr) {
+                    float acc = __fmul_rn(lds_f32(pz + 4u * (uint32_t)(rr * NGT)), S);
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) {
+                        const uint32_t w = lds_u32(pw + 4u * (uint32_t)((j * kBatchRows + rr) * kWideWords));
+                        const float t0 = lds_f32(__byte_perm(w, lane_base, 0x7604));
+                        const float t1 = lds_f32(__byte_perm(w, lane_base, 0x7614) + 128u);
+                        const float t2 = lds_f32(__byte_perm(w, lane_base, 0x7624) + 65536u);
+                        const float t3 = lds_f32(__byte_perm(w, lane_base, 0x7634) + 65536u + 128u);
+                        const float P = __fadd_rn(__fadd_rn(t0, t1), __fadd_rn(t2, t3));
+                        acc = fmaf(lds_f32(pa + 4u * (uint32_t)(rr * NGT * Q + j)), fmaf(2.f, P, -S), acc);
+                    }
+                    v[rr] = acc;
+                }
+                const int rb = kBatchRows * (warp + NW * k);
+                const int slot0 = SR::run(v, lane);
+                if (SR::writer(lane) && rb + slot0 < nr) prow[rb + slot0] = v[0];
+            }
+            __syncwarp();                                      // stage s is free for item i + NS
+            if (alive && lane == 0 && issued < total) issue_next();
+        }
+    }
+    if (!alive && lane == 0) {
+        // copies issued but never waited for land before the block exits
+        for (int i = waited; i < issued; ++i)
+            if (!tma::bar_wait(bar0 + 8u * (i & 1), (uint32_t)((i >> 1) & 1))) {
+                atomicOr(&g_gemv_err, kDrainTimeoutBit);       // copies may still be in flight
+                break;
+            }
+    }
+}
+
 // y[b, r] = sum over tiles of PART[t, b, r], in tile order.
 __global__ void __launch_bounds__(256)
 bcq_gemv_reduce_kernel(const float* __restrict__ PART, float* __restrict__ Y, int64_t n, int n_tiles) {
@@ -556,18 +788,19 @@ static TensorMapEncode tensor_map_encoder() {
 
 // Tensor maps of the bit-planes [q][out][in/32] (u32), alpha* [out][Gr q] and
 // z* [out][Gr] (fp32), Gr = in / g, with the boxes of one 8-row batch of one
-// 512-column tile.  Called only for in a multiple of 512 and g <= 128, so every
-// stride is a multiple of 16 bytes and every box starts on a 16-byte boundary.
+// tile of `tile_cols` columns (512 or 1024).  Called only for in a multiple of
+// tile_cols and at least 4 groups per tile, so every stride is a multiple of
+// 16 bytes and every box starts on a 16-byte boundary.
 // False if the encoder is unavailable or refuses a map.
 static bool gemv_tensor_maps(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in,
-                             int q, int g, CUtensorMap* mp, CUtensorMap* ma, CUtensorMap* mz) {
+                             int q, int g, int tile_cols, CUtensorMap* mp, CUtensorMap* ma, CUtensorMap* mz) {
     const TensorMapEncode enc = tensor_map_encoder();
     if (enc == nullptr) return false;
     const cuuint64_t words = (cuuint64_t)n_in / 32, gr = (cuuint64_t)(n_in / g), rows = (cuuint64_t)out;
-    const cuuint32_t ngt = (cuuint32_t)(kTileCols / g), one[3] = {1, 1, 1};
+    const cuuint32_t ngt = (cuuint32_t)(tile_cols / g), one[3] = {1, 1, 1};
     const cuuint64_t pdim[3] = {words, rows, (cuuint64_t)q};
     const cuuint64_t pstride[2] = {words * 4, words * 4 * rows};
-    const cuuint32_t pbox[3] = {(cuuint32_t)kTileWords, (cuuint32_t)kBatchRows, (cuuint32_t)q};
+    const cuuint32_t pbox[3] = {(cuuint32_t)(tile_cols / 32), (cuuint32_t)kBatchRows, (cuuint32_t)q};
     if (enc(mp, CU_TENSOR_MAP_DATA_TYPE_UINT32, 3, const_cast<uint32_t*>(planes), pdim, pstride, pbox, one,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
@@ -590,7 +823,7 @@ static bool gemv_tensor_maps(const uint32_t* planes, const float* astar, const f
 // Opts a kernel into `smem` bytes of dynamic shared memory and returns its
 // resident blocks per SM, once per device (Tag: one cache per kernel).
 template <typename Tag, typename KERN>
-static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm) {
+static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm, int threads = kGemvThreads) {
     static std::atomic<int> cache[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -599,7 +832,7 @@ static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm) {
     if (per_sm != 0) return cudaSuccess;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGemvThreads, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     if (dev >= 0 && dev < 64) cache[dev].store(per_sm, std::memory_order_relaxed);
@@ -609,7 +842,8 @@ static cudaError_t gemv_blocks_per_sm(KERN kern, size_t smem, int& per_sm) {
 // Row blocks (of whole 8-row batches): the count that minimises
 // waves x (one table build, worth about 32 rows, + rows per block), where
 // a wave is one block per resident slot.
-static void gemv_row_blocks(int64_t out, int n_tiles, int per_sm, int64_t& n_rb, int64_t& rpb) {
+static void gemv_row_blocks(int64_t out, int n_tiles, int per_sm, int64_t& n_rb, int64_t& rpb,
+                            double table_rows = 32.0) {
     const int64_t slots = (int64_t)sm_count() * per_sm;
     const int64_t max_rb = (out + kBatchRows - 1) / kBatchRows;
     n_rb = 1;
@@ -621,7 +855,7 @@ static void gemv_row_blocks(int64_t out, int n_tiles, int per_sm, int64_t& n_rb,
         r = (r + kBatchRows - 1) / kBatchRows * kBatchRows;
         const int64_t nb = (out + r - 1) / r;
         const int64_t waves = (nb * n_tiles + slots - 1) / slots;
-        const double cost = (double)waves * (32.0 + (double)r);
+        const double cost = (double)waves * (table_rows + (double)r);
         if (best < 0.0 || cost < best) { best = cost; n_rb = nb; rpb = r; }
     }
 }
@@ -659,7 +893,7 @@ static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const fl
     if constexpr (NGT >= 4) {
         const unsigned long long plane_bytes = (unsigned long long)(n_in / 32) * 4ull * (unsigned long long)out;
         CUtensorMap mp, ma, mz;
-        if (whole && plane_bytes < (1ull << 40) && gemv_tensor_maps(planes, astar, zstar, out, n_in, Q, g, &mp, &ma, &mz)) {
+        if (whole && plane_bytes < (1ull << 40) && gemv_tensor_maps(planes, astar, zstar, out, n_in, Q, g, kTileCols, &mp, &ma, &mz)) {
             auto kern = bcq_gemv_tma_kernel<Q, XT, NGT>;
             int per_sm = 0;
             cudaError_t e = gemv_blocks_per_sm<GemvTmaTag<Q, XT, NGT>>(kern, smem_tma, per_sm);
@@ -686,9 +920,53 @@ static cudaError_t run_gemv(const uint32_t* planes, const float* astar, const fl
     return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);
 }
 
+template <int Q, typename XT, int NGT>
+struct GemvWideTag {};
+
+// The wide-lane product (in a multiple of 1024, NGT = 1024 / g groups per
+// tile).  Returns cudaErrorNotSupported, having launched nothing, when the
+// shape or the driver does not allow it; the caller then takes the 512-column
+// kernels.
+template <int Q, typename XT, int NGT>
+static cudaError_t run_gemv_wide(const uint32_t* planes, const float* astar, const float* zstar, int64_t out,
+                                 int n_in, int g, const void* x, int batch, float* y, float* work, cudaStream_t st) {
+    if constexpr (wide_warps(Q, NGT) >= 4) {
+        constexpr int NW = wide_warps(Q, NGT);
+        constexpr int DYN = wide_smem_bytes(Q, NGT);
+        const unsigned long long plane_bytes = (unsigned long long)(n_in / 32) * 4ull * (unsigned long long)out;
+        if (n_in % kWideCols != 0 || plane_bytes >= (1ull << 40)) return cudaErrorNotSupported;
+        CUtensorMap mp, ma, mz;
+        if (!gemv_tensor_maps(planes, astar, zstar, out, n_in, Q, g, kWideCols, &mp, &ma, &mz))
+            return cudaErrorNotSupported;
+        auto kern = bcq_gemv_wide_kernel<Q, XT, NGT>;
+        int per_sm = 0;
+        cudaError_t e = gemv_blocks_per_sm<GemvWideTag<Q, XT, NGT>>(kern, DYN, per_sm, NW * 32);
+        if (e != cudaSuccess) return e;
+        const int n_tiles = n_in / kWideCols;
+        int64_t n_rb = 0, rpb = 0;
+        gemv_row_blocks(out, n_tiles, per_sm, n_rb, rpb, (double)kWideLutRows);
+        kern<<<(unsigned)(n_rb * n_tiles), NW * 32, DYN, st>>>(mp, ma, mz, x, work, out, n_in, batch, n_tiles, rpb);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);
+    } else {
+        return cudaErrorNotSupported;
+    }
+}
+
 template <int Q, typename XT>
 static cudaError_t gemv_g(const uint32_t* planes, const float* astar, const float* zstar, int64_t out, int n_in, int g,
                           const void* x, int batch, float* y, float* work, cudaStream_t st) {
+    if (n_in % kWideCols == 0 && g <= 256) {
+        cudaError_t e = cudaErrorNotSupported;
+        switch (wide_tile_groups(g)) {
+            case 32: e = run_gemv_wide<Q, XT, 32>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st); break;
+            case 16: e = run_gemv_wide<Q, XT, 16>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st); break;
+            case 8: e = run_gemv_wide<Q, XT, 8>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st); break;
+            default: e = run_gemv_wide<Q, XT, 4>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st); break;
+        }
+        if (e != cudaErrorNotSupported) return e;
+    }
     switch (gemv_tile_groups(g)) {
         case 16: return run_gemv<Q, XT, 16>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st);
         case 8: return run_gemv<Q, XT, 8>(planes, astar, zstar, out, n_in, g, x, batch, y, work, st);

@@ -66,6 +66,40 @@ def block_forward(X, W, shape):
     return X1 + F.linear(F.silu(F.linear(h2, W["gate_proj"])) * F.linear(h2, W["up_proj"]), W["down_proj"])
 
 
+def level_ranks(alpha, zb, codes, g):
+    """Index of every weight's level among its group's 2^q levels, as
+    Algorithm 4 indexes them: the levels l(c) = c_1 a_1 + ... + c_q a_q + z_B
+    (fp32, summed left to right) sorted ascending, equal levels in code-word
+    order.  The index-change statistics of the paper's Table 2 compare these
+    ranks between steps.  alpha [out, in/g, q], zb [out, in/g], codes
+    [out, in] uint8 (bits at or above q ignored) -> uint8 ranks [out, in].
+    Device tensors in, device tensor out; a report, outside the quantizer."""
+    out, n_in = codes.shape
+    q = alpha.shape[-1]
+    L = 1 << q
+    cw = torch.arange(L, device=codes.device)
+    lv = None
+    for j in range(q):
+        cj = (((cw >> j) & 1) * 2 - 1).to(torch.float32)           # c_j of every code word
+        term = alpha[..., j:j + 1] * cj                              # exact: c_j = +-1
+        lv = term if lv is None else lv + term
+    lv = lv + zb[..., None]
+    order = torch.sort(lv, dim=-1, stable=True).indices              # ties keep code-word order
+    rank_of_code = torch.empty_like(order)
+    rank_of_code.scatter_(-1, order, cw.expand_as(order).contiguous())
+    c = (codes.view(out, n_in // g, g).long() & (L - 1))
+    return torch.gather(rank_of_code, -1, c).view(out, n_in).to(torch.uint8)
+
+
+def index_change_shares(r_a, r_b):
+    """Shares of weights whose level index moved by 0, 1, 2 and more than 2
+    between two rank arrays (the four columns of Table 2)."""
+    d = (r_a.to(torch.int16) - r_b.to(torch.int16)).abs()
+    n = d.numel()
+    c0, c1, c2 = int((d == 0).sum()), int((d == 1).sum()), int((d == 2).sum())
+    return [c0 / n, c1 / n, c2 / n, (n - c0 - c1 - c2) / n]
+
+
 class BlockReconstructor:
     """The quantizer state of one block and the steps of Algorithm 1.
 
@@ -139,6 +173,10 @@ class BlockReconstructor:
             self.qz[n].train_step(self.t, self.lr_F, self.lr_B, self.p, self.map_mode)
         self.t += 1
         return loss.detach()
+
+    def ranks(self):
+        """{name: level index of every weight} under the current parameters (level_ranks)."""
+        return {n: level_ranks(self.P[n]["alpha"], self.P[n]["zb"], self.codes[n], self.g) for n in NAMES}
 
     def save(self, path):
         """Checkpoint: Theta_IF and the codes of the seven weights and the

@@ -66,8 +66,10 @@ def check(planes, a_star, z_star, x, g, xdtype="f32", label=""):
     return y
 
 
-# in: one ragged tile, several tiles, a non-multiple of 512; whole tiles with 4, 8 and
-# 16 groups per tile take the tensor-copy staging, the others the per-lane copies
+# in: one ragged tile, several tiles, a non-multiple of 512.  In a multiple of 1024 with
+# g <= 256 takes the wide-lane kernel (1024-column tiles, 4 to 32 groups per tile); other
+# whole 512-column tiles with 4, 8 and 16 groups per tile the tensor-copy staging, the
+# rest the per-lane copies
 @pytest.mark.parametrize("out,n_in,g", [(40, 256, 32), (33, 512, 64), (17, 1536, 128), (64, 4096, 128),
                                         (9, 4096 + 32 * 3, 32), (5, 8192, 256), (3, 28672, 128), (300, 1024, 512),
                                         (24, 1024, 32), (13, 2560, 64), (11, 3072, 1024), (6, 4096, 2048)])
@@ -88,11 +90,14 @@ def test_gemv_batches_and_bf16_activations(batch, xdtype):
     check(planes, a_star, z_star, x, 128, xdtype, label=f"batch {batch} {xdtype}")
 
 
-def test_gemv_many_rows():
-    """Many more rows than one wave of row blocks."""
-    planes, a_star, z_star = random_export(9000, 512, 2, 64, seed=9)
-    x = np.random.default_rng(0).standard_normal((1, 512)).astype(F32)
-    check(planes, a_star, z_star, x, 64, label="9000 rows")
+@pytest.mark.parametrize("out,n_in,g,q", [(9000, 512, 64, 2), (9001, 2048, 64, 2), (2053, 3072, 32, 4),
+                                          (1, 1024, 256, 1), (7, 1024, 128, 3)])
+def test_gemv_many_rows(out, n_in, g, q):
+    """Many more rows than one wave of row blocks, a ragged last batch of
+    rows, and single-row and single-tile products, on both kernels."""
+    planes, a_star, z_star = random_export(out, n_in, q, g, seed=9 + out)
+    x = np.random.default_rng(0).standard_normal((2, n_in)).astype(F32)
+    check(planes, a_star, z_star, x, g, label=f"{out} rows {n_in} g{g} q{q}")
 
 
 def test_gemv_deterministic():

@@ -65,8 +65,14 @@ def param_tolerances(W, P, codes, Gup, g, lr_F, lr_B):
     return ref, tol
 
 
+# Code mismatches allowed per case: every one must also be a near-tie (assert_near_ties).
+# Measured over the 109 cases of this file: 1 mismatch in 7,088,640 codes (1.4e-7); the worst
+# single case had 1 of 86,016 (1.16e-5).  The cap is four times that worst case.
+MAX_TIE_FRAC = 5e-5
+
+
 def check_against_oracle(raw, W, P, codes, Gup, q, g, t, mode, p, lr_F=LR_F, lr_B=LR_B, label="",
-                         max_tie_frac=1e-4):
+                         max_tie_frac=MAX_TIE_FRAC):
     newP, c1, w1 = gpu_step(raw, P, codes, Gup, q, g, t, mode, p, lr_F, lr_B)
     ref, tol = param_tolerances(W, P, codes, Gup, g, lr_F, lr_B)
     for k in PK:
