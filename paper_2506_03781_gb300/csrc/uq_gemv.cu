@@ -490,9 +490,17 @@ __host__ __device__ constexpr int wide_warps(int q, int ngt) {
                : (int)((kSmemOptIn - (int)kWideLutBytes - kWideHeadBytes - wide_slack(q, ngt)) /
                        (kWideStages * wide_stage_bytes(q, ngt)));
 }
+// Dynamic shared memory to request.  The tables start at the first multiple
+// of 65536 at or above the dynamic base D, so they end by D + 192 KB at the
+// latest; when the head and the stages do not fit in the space below them,
+// the rest follows the tables with at most wide_slack of that space unused.
 __host__ __device__ constexpr int wide_smem_bytes(int q, int ngt) {
     return (int)kWideLutBytes + kWideHeadBytes + wide_slack(q, ngt) +
-           wide_warps(q, ngt) * kWideStages * wide_stage_bytes(q, ngt);
+                       wide_warps(q, ngt) * kWideStages * wide_stage_bytes(q, ngt) >
+                   (int)kWideLutBytes + 65536
+               ? (int)kWideLutBytes + kWideHeadBytes + wide_slack(q, ngt) +
+                     wide_warps(q, ngt) * kWideStages * wide_stage_bytes(q, ngt)
+               : (int)kWideLutBytes + 65536;
 }
 
 // Index of the lowest set bit of n (1 <= n <= 15).

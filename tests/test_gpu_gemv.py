@@ -51,6 +51,7 @@ def gpu_gemv(planes, a_star, z_star, x, g, xdtype="f32"):
     ws = torch.full((api.uq_bcq_gemv_workspace_bytes(planes.shape[1], x.shape[1], x.shape[0]) // 4,), float("nan"),
                     device=d)
     api.uq_bcq_gemv(pd, ad, zd, xd, y, g, workspace=ws)
+    api.uq_check_device()                         # no pipeline wait ran out, no layout refused
     return C.host(y)
 
 
