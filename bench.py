@@ -572,10 +572,10 @@ def time_block_step(dev, steps=20, warmup=4, samples=4, idx_steps=64):
     # the quantizer alone: the seven fused steps of one optimisation step
     q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     q0.record(stream)
+    qgrads = {n: (torch.randn(rec.what_c[n].shape, device=dev) * 1e-7).to(torch.bfloat16) for n in NAMES} \
+        if rec.bf16_io else None
     for i in range(steps):
-        for n in NAMES:
-            rec.qz[n].train_step(rec.t, rec.lr_F, rec.lr_B, rec.p, rec.map_mode)
-        rec.t += 1
+        rec.quantizer_step(qgrads)
     q1.record(stream)
     torch.cuda.synchronize()
     qms = q0.elapsed_time(q1) / steps

@@ -255,6 +255,24 @@ uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                         uq_map map, int64_t step, int p_period, float* W_hat, void* stream);
 
 /*
+ * uq_train_step_bf16 -- uq_train_step for a block computed in bf16 (the
+ * reconstruction loop of Algorithm 1 back-propagates through the block in
+ * its compute type): the same step, parameters and codes bit for bit as
+ * uq_train_step given the same dL_dWhat values, except that
+ *   dL_dWhat: [out, in] bf16 bits (uint16), read exactly (each value is the
+ *     fp32 number those bits denote);
+ *   W_hat: [out, in] bf16 bits (uint16), written with W^ of step + 1 as
+ *     computed in fp32 by uq_train_step, rounded to the nearest bf16 (ties
+ *     to even).
+ * So the caller's block consumes W^ and produces dL/dW^ in its own type
+ * without a conversion pass over the weights.  Arguments, shapes and errors
+ * otherwise as uq_train_step.
+ */
+uq_status uq_train_step_bf16(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
+                             uq_params params, uint8_t* codes, const uint16_t* dL_dWhat, float lr_F, float lr_B,
+                             uq_map map, int64_t step, int p_period, uint16_t* W_hat, void* stream);
+
+/*
  * uq_quantize_fwd_omni -- the UniQuan quantizer with OmniQuant's maps
  * (App. E, extensibility) in place of FlexRound's:
  *   T_O(w) = w / Delta_O + z_O,  D_O(w~) = Delta_O (w~ - z_O),

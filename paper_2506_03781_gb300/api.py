@@ -34,7 +34,8 @@ OMNI_GRAD_NAMES = ("dbeta", "dgamma", "dalpha", "dzb")
 AWQ_PARAM_NAMES = ("sa", "delta", "za", "alpha", "zb")
 AWQ_GRAD_NAMES = ("dsa", "ddelta", "dza", "dalpha", "dzb")
 GRAD_NAMES = ("ddelta", "dzu", "ds", "dsr", "dalpha", "dzb")
-ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_export_bcq",
+ENTRY_POINTS = ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_train_step", "uq_train_step_bf16",
+                "uq_export_bcq",
                 "uq_quantize_bwd_ex", "uq_export_bcq_half",
                 "uq_quantize_fwd_omni", "uq_quantize_bwd_omni", "uq_omni_scales",
                 "uq_quantize_fwd_awq", "uq_quantize_bwd_awq", "uq_awq_bwd_workspace_bytes", "uq_bcq_gemv",
@@ -107,6 +108,8 @@ def lib() -> ctypes.CDLL:
         f32 = ctypes.c_float
         L.uq_train_step.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, f32, f32, i32, i64, i32, vp,
                                     vp]
+        L.uq_train_step_bf16.argtypes = [vp, i32, i64, i64, i32, i32, uq_params, vp, vp, f32, f32, i32, i64, i32,
+                                         vp, vp]
         for name in ("uq_init_params", "uq_quantize_fwd", "uq_quantize_bwd", "uq_export_bcq"):
             getattr(L, name).restype = ctypes.c_int
         L.uq_last_error.argtypes = []
@@ -268,6 +271,20 @@ def uq_train_step(W, q, g, params, codes, dL_dWhat, W_hat, step, lr_F=LR_THETA_F
         _check(codes, "codes", (out, n_in), torch.uint8, dev),
         _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.float32, dev), float(lr_F), float(lr_B), map_mode, step,
         p_period, _check(W_hat, "W_hat", (out, n_in), torch.float32, dev), _stream(stream, dev))
+    _raise(st)
+
+
+def uq_train_step_bf16(W, q, g, params, codes, dL_dWhat, W_hat, step, lr_F=LR_THETA_F, lr_B=LR_THETA_B,
+                       map_mode=MAP_LOCAL_PERIODIC, p_period=2, stream=None):
+    """uq_train_step with bf16 ``dL_dWhat`` (read exactly) and bf16 ``W_hat``
+    (W^ of ``step + 1`` rounded to nearest even), for a block computed in bf16."""
+    out, n_in = _dims(W, g)
+    dev = W.device
+    st = lib().uq_train_step_bf16(
+        W.data_ptr(), _wdtype(W), out, n_in, q, g, _params(params, out, n_in, q, g, dev),
+        _check(codes, "codes", (out, n_in), torch.uint8, dev),
+        _check(dL_dWhat, "dL_dWhat", (out, n_in), torch.bfloat16, dev), float(lr_F), float(lr_B), map_mode, step,
+        p_period, _check(W_hat, "W_hat", (out, n_in), torch.bfloat16, dev), _stream(stream, dev))
     _raise(st)
 
 

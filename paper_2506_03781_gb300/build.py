@@ -18,7 +18,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libuq.so")
-SOURCES = ["uq_api.cu", "uq_fwd.cu", "uq_bwd.cu", "uq_export.cu", "uq_init.cu", "uq_stream.cu", "uq_step.cu", "uq_gemv.cu", "uq_omni.cu", "uq_awq.cu"]
+SOURCES = ["uq_api.cu", "uq_fwd.cu", "uq_bwd.cu", "uq_export.cu", "uq_init.cu", "uq_stream.cu", "uq_step.cu", "uq_step_bf16.cu", "uq_gemv.cu", "uq_omni.cu", "uq_awq.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include")]
 

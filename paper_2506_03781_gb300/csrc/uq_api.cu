@@ -221,6 +221,35 @@ uq_status uq_train_step(const void* W, uq_wdtype wdtype, int64_t out, int64_t in
                        "uq_train_step");
 }
 
+uq_status uq_train_step_bf16(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g, uq_params p,
+                             uint8_t* codes, const uint16_t* dL_dWhat, float lr_F, float lr_B, uq_map map,
+                             int64_t step, int p_period, uint16_t* W_hat, void* stream) {
+    UQ_TRY(check_shape(out, in, q, g, wdtype));
+    if (map != UQ_MAP_FULL && map != UQ_MAP_LOCAL_PERIODIC) return fail(UQ_ERR_ARG, "unknown mapping %d", (int)map);
+    if (p_period < 1) return fail(UQ_ERR_ARG, "p_period=%d must be >= 1", p_period);
+    if (step < 0 || step == INT64_MAX) return fail(UQ_ERR_ARG, "step=%lld must be in [0, 2^63 - 1)", (long long)step);
+    const uq::Shape sh{out, (int)in, q, g, (int)wdtype};
+    if (!uq::step_path_ok(sh))
+        return fail(UQ_ERR_UNSUPPORTED,
+                    "the fused step handles g in {32, 64, 128} with in a multiple of %d and at most %d (g=%d in=%lld)",
+                    g == 32 ? 256 : 512, g == 32 ? 16384 : 32768, g, (long long)in);
+    UQ_TRY(check_ptr(W, "W"));
+    UQ_TRY(check_ptr(p.delta, "params.delta"));
+    UQ_TRY(check_ptr(p.zu, "params.zu"));
+    UQ_TRY(check_ptr(p.s, "params.s"));
+    UQ_TRY(check_ptr(p.sr, "params.sr"));
+    UQ_TRY(check_ptr(p.alpha, "params.alpha"));
+    UQ_TRY(check_ptr(p.zb, "params.zb"));
+    UQ_TRY(check_ptr(codes, "codes"));
+    UQ_TRY(check_ptr(dL_dWhat, "dL_dWhat"));
+    UQ_TRY(check_ptr(W_hat, "W_hat"));
+    const int64_t next = step + 1;
+    const int mode = map == UQ_MAP_FULL ? uq::FWD_FULL : (next % p_period == 0 ? uq::FWD_REMAP : uq::FWD_KEEP);
+    return cuda_status(
+        uq::launch_step_bf16(sh, W, p, codes, dL_dWhat, lr_F, lr_B, mode, W_hat, (cudaStream_t)stream),
+        "uq_train_step_bf16");
+}
+
 uq_status uq_quantize_fwd_omni(const void* W, uq_wdtype wdtype, int64_t out, int64_t in, int q, int g,
                                uq_params_omni p, uint8_t* codes, uq_map map, int64_t step, int p_period,
                                float* W_hat, void* stream) {
@@ -409,6 +438,11 @@ uq_status uq_check_device(void* stream) {
     unsigned int flag = 0, flag_step = 0, flag_omni = 0, flag_awq = 0, flag_gemv = 0;
     e = uq::stream_error(true, &flag);
     if (e == cudaSuccess) e = uq::step_error(true, &flag_step);
+    if (e == cudaSuccess) {
+        unsigned int flag_step_bf16 = 0;
+        e = uq::step_bf16_error(true, &flag_step_bf16);
+        flag_step |= flag_step_bf16;
+    }
     if (e == cudaSuccess) e = uq::omni_error(true, &flag_omni);
     if (e == cudaSuccess) e = uq::awq_error(true, &flag_awq);
     if (e == cudaSuccess) e = uq::gemv_error(true, &flag_gemv);

@@ -45,6 +45,10 @@ cudaError_t launch_step(const Shape& sh, const void* W, uq_params p, uint8_t* co
                         float lr_b, int mode, float* what, cudaStream_t st);
 // Reads (and optionally clears) the fused step kernel's bounded-wait flag.
 cudaError_t step_error(bool clear, unsigned int* flag);
+// The fused step with bf16 dL/dW^ and W^ (uq_step_bf16.cu), and its flag.
+cudaError_t launch_step_bf16(const Shape& sh, const void* W, uq_params p, uint8_t* codes, const uint16_t* gup,
+                             float lr_f, float lr_b, int mode, uint16_t* what, cudaStream_t st);
+cudaError_t step_bf16_error(bool clear, unsigned int* flag);
 // BCQ matrix-vector product from the exported bit-planes (uq_gemv.cu); `work`
 // holds gemv_workspace_floats(out, in, batch) floats of per-tile partials.
 int64_t gemv_workspace_floats(int64_t out, int64_t n_in, int batch);

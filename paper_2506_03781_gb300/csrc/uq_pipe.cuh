@@ -95,7 +95,9 @@ constexpr int kMaxStages = 16;
 // staged; HAS_G: dL/dW^ is staged; HAS_C: code words are staged.  The group
 // parameters (Delta, z_U, z_B, alpha of the unit's NG groups) always are.
 // HAS_S: s is staged with the weights (by default exactly when they are).
-template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET, bool HAS_S = HAS_X>
+// GBYTES: bytes of one staged dL/dW^ element (4 for fp32, 2 for bf16).
+template <int Q, typename WT, int G_, bool HAS_X, bool HAS_G, bool HAS_C, int BUDGET, bool HAS_S = HAS_X,
+          int GBYTES = 4>
 struct Stage {
     static constexpr int LPG = G_ <= 64 ? 4 : 8;
     static constexpr int NG = 32 / LPG;                  // groups per unit
@@ -104,7 +106,8 @@ struct Stage {
     static constexpr int WBYTES = sizeof(typename WT::raw) / 4;
     static constexpr int SZ_W = HAS_X ? UE * WBYTES : 0;
     static constexpr int SZ_S = HAS_S ? UE * 4 : 0;
-    static constexpr int SZ_G = HAS_G ? UE * 4 : 0;
+    static constexpr int GB = GBYTES;
+    static constexpr int SZ_G = HAS_G ? UE * GBYTES : 0;
     static constexpr int SZ_C = HAS_C ? UE : 0;
     static constexpr int SZ_P = NG * 4, SZ_A = NG * Q * 4;
     static constexpr int OFF_W = 0;

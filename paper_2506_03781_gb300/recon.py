@@ -115,7 +115,11 @@ class BlockReconstructor:
         self.lr_F, self.lr_B = lr_F, lr_B
         self.device = torch.device(device)
         self.dtype = compute_dtype
+        # A bf16 block takes W^ and gives dL/dW^ in bf16 straight from the fused
+        # step (uq_train_step_bf16): no conversion pass over the weights per step.
+        self.bf16_io = compute_dtype == torch.bfloat16
         self.W, self.P, self.codes, self.what, self.G, self.qz = {}, {}, {}, {}, {}, {}
+        self.what_c = {}
         for m in shape.matrices():
             n = m.name
             Wd = api.weights_tensor(weights[n], self.device)
@@ -125,6 +129,8 @@ class BlockReconstructor:
             self.what[n] = torch.empty(m.out, m.n_in, dtype=torch.float32, device=self.device)
             self.G[n] = torch.zeros(m.out, m.n_in, dtype=torch.float32, device=self.device)
             self.qz[n] = api.Quantizer(Wd, q, g, self.P[n], self.codes[n], self.what[n], self.G[n])
+            if self.bf16_io:
+                self.what_c[n] = torch.empty(m.out, m.n_in, dtype=torch.bfloat16, device=self.device)
             if init:
                 api.uq_init_params(Wd, q, g, self.P[n], self.codes[n], G=G, T=T)
         # unquantized weights in the compute dtype, for the targets
@@ -145,7 +151,27 @@ class BlockReconstructor:
     def _forward0(self):
         for n in NAMES:
             self.qz[n].fwd(0, self.p, self.map_mode)
+        self._sync_compute_copy()
         self.t = 0
+
+    def _sync_compute_copy(self):
+        # the bf16 W^ the block reads, from the fp32 W^ of a separate forward
+        # (step 0 or a resume; every later W^ comes from the fused step in bf16)
+        if self.bf16_io:
+            for n in NAMES:
+                self.what_c[n].copy_(self.what[n])
+
+    def quantizer_step(self, grads=None):
+        """The fused steps of the seven weights (backward of step t, SGD, forward
+        of t + 1), then t += 1.  grads: {name: dL/dW^} in bf16 for a bf16 block
+        (uq_train_step_bf16); otherwise the fp32 buffers self.G are used."""
+        for n in NAMES:
+            if self.bf16_io:
+                api.uq_train_step_bf16(self.W[n], self.q, self.g, self.P[n], self.codes[n], grads[n],
+                                       self.what_c[n], self.t, self.lr_F, self.lr_B, self.map_mode, self.p)
+            else:
+                self.qz[n].train_step(self.t, self.lr_F, self.lr_B, self.p, self.map_mode)
+        self.t += 1
 
     @torch.no_grad()
     def targets(self, X):
@@ -156,22 +182,32 @@ class BlockReconstructor:
         """One optimisation step on one sample; returns the loss of W^_t
         (a 0-d tensor on the device, no synchronisation)."""
         leaves = {}
-        for n in NAMES:
-            leaf = self.what[n].detach().requires_grad_(True)
-            self.G[n].zero_()
-            leaf.grad = self.G[n]                       # back-propagation accumulates into dL/dW^
-            leaves[n] = leaf
-        Wc = {n: leaves[n].to(self.dtype) for n in NAMES}
+        if self.bf16_io:
+            # W^ is already bf16; autograd hands back dL/dW^ in bf16
+            for n in NAMES:
+                leaves[n] = self.what_c[n].detach().requires_grad_(True)
+            Wc = leaves
+        else:
+            for n in NAMES:
+                leaf = self.what[n].detach().requires_grad_(True)
+                self.G[n].zero_()
+                leaf.grad = self.G[n]                   # back-propagation accumulates into dL/dW^
+                leaves[n] = leaf
+            Wc = {n: leaves[n].to(self.dtype) for n in NAMES}
         out = block_forward(Xh.to(self.dtype), Wc, self.shape)
         loss = (out.float() - Y.float()).pow(2).mean()
         loss.backward()
+        grads = None
+        if self.bf16_io:
+            grads = {n: leaves[n].grad.contiguous() for n in NAMES}
+        else:
+            for n in NAMES:
+                gr = leaves[n].grad
+                if gr.data_ptr() != self.G[n].data_ptr():   # autograd replaced the buffer instead of adding into it
+                    self.G[n].copy_(gr)
         for n in NAMES:
-            gr = leaves[n].grad
-            if gr.data_ptr() != self.G[n].data_ptr():   # autograd replaced the buffer instead of adding into it
-                self.G[n].copy_(gr)
             leaves[n].grad = None
-            self.qz[n].train_step(self.t, self.lr_F, self.lr_B, self.p, self.map_mode)
-        self.t += 1
+        self.quantizer_step(grads)
         return loss.detach()
 
     def ranks(self):
@@ -198,9 +234,12 @@ class BlockReconstructor:
             checkpoint.restore_into(mats[n], self.P[n], self.codes[n])
         for n in NAMES:
             checkpoint.rebuild_what(self.qz[n])
+        self._sync_compute_copy()
         self.t = step
 
     def state(self):
-        """Host copies: ({name: params dict}, {name: codes}, {name: W^})."""
+        """Host copies: ({name: params dict}, {name: codes}, {name: W^}); W^ is
+        the block's copy (bf16 values as fp32 for a bf16 block)."""
+        what = {n: (self.what_c[n].float() if self.bf16_io else self.what[n]).cpu().numpy() for n in NAMES}
         return ({n: {k: v.cpu().numpy() for k, v in self.P[n].items()} for n in NAMES},
-                {n: self.codes[n].cpu().numpy() for n in NAMES}, {n: self.what[n].cpu().numpy() for n in NAMES})
+                {n: self.codes[n].cpu().numpy() for n in NAMES}, what)

@@ -370,3 +370,31 @@ def test_llama2_70b_down_proj_step_sampled_rows():
     wl = synth.WORKLOADS["llama2_70b_mlp_bf16"]
     idx = [i for i, m in enumerate(wl.matrices) if m.n_in == 28672][0]
     full_size_step(wl, idx, sample_rows(wl.matrices[idx].out, 12, 17), 1, "70b down")
+
+
+@pytest.mark.parametrize("out,n_in,g", [(64, 512, 128), (21, 768, 32), (37, 4096, 128), (6, 14336, 128)])
+@pytest.mark.parametrize("q", [2, 3])
+def test_step_bf16_io_equals_the_fp32_step(out, n_in, g, q):
+    """uq_train_step_bf16 reads dL/dW^ as bf16 and writes W^ as bf16: given
+    dL/dW^ values that bf16 represents exactly, its parameters and codes
+    equal uq_train_step's bit for bit, and its W^ is the fp32 step's W^
+    rounded to nearest even (torch's fp32 -> bf16 conversion), for a
+    remapping and a keeping forward of t + 1 and rows split over a cluster."""
+    raw, W, P, codes, Gup = C.make_inputs(out, n_in, q, g, seed=60 + out + q)
+    _, Gb = synth.bf16_round(Gup)                 # values exact in bf16
+    d = C.dev()
+    Wd = api.weights_tensor(raw, d)
+    for t in (0, 1):
+        pa, pb = C.to_dev(P), C.to_dev(P)
+        ca = torch.from_numpy(np.ascontiguousarray(codes)).to(d)
+        cb = ca.clone()
+        Ga = torch.from_numpy(np.ascontiguousarray(Gb)).to(d)
+        wa = torch.full((out, n_in), float("nan"), device=d)
+        wb = torch.full((out, n_in), float("nan"), device=d).to(torch.bfloat16)
+        api.uq_train_step(Wd, q, g, pa, ca, Ga, wa, t)
+        api.uq_train_step_bf16(Wd, q, g, pb, cb, Ga.to(torch.bfloat16), wb, t)
+        api.uq_check_device(None)
+        for k in PK:
+            assert torch.equal(pa[k], pb[k]), (k, t)
+        assert torch.equal(ca, cb), t
+        assert torch.equal(wa.to(torch.bfloat16), wb), (t, int((wa.to(torch.bfloat16) != wb).sum()))
