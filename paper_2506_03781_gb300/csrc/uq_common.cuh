@@ -330,6 +330,98 @@ __device__ __forceinline__ void bwd_vec4(const float w[4], const float s4[4], co
     }
 }
 
+// ---------------------------------------------------------------------------
+// Local remap step (Algorithm 4) from the reciprocal, with a proof
+// ---------------------------------------------------------------------------
+//
+// On a remap step the code word c of an element is kept unless the level
+// below it (rank r - 1) or above it (rank r + 1) is strictly nearer to the
+// IEEE value x = fl(fl(w / den) + z_U) (the tie rules of the exact path).
+// Per group slot k and code word c, unit_remap_iv stores iv = (a, b, w^, 0):
+//   a = mid(l_lo, l_c) + m_lo, b = mid(l_c, l_hi) - m_hi  (fp32), with
+//   mid(p, q) = 0.5 (p + q) and m = 2^-18 (|mid| + |z_U| + M) + 2^-126,
+//   M = max |level| of the group; a = -inf when l_lo == l_c and b = +inf
+//   when l_hi == l_c (equal levels never win: ties keep c);
+//   w^ = Delta (l_c - z_U), the output of a kept code.
+// remap_vec4 forms x' = fl(fl(w r) + z_U) from the reciprocal estimate r of
+// den (as bwd_vec4 does; |x' - x| <= 2^-21 |x'| + 2^-22 |z_U| + 2^-148) and
+// keeps the codes of a vector of 4 elements when every x' lies in (a, b)
+// and every |den| < 2^125.  Then each x lies more than m / 2 from the
+// midpoint on a finite side, where the fp32 distances to the two levels
+// differ by more than m - 2^-22 M > 0, or beyond the level on that side
+// (the far level is then never strictly nearer: rounding is monotonic); so
+// the exact path keeps c as well.  Every other vector -- an element near a
+// midpoint, a den out of range, an infinity or a NaN (all comparisons
+// false) -- takes the exact path: transform_x and the three distances.
+template <int Q, int NS>
+__device__ __forceinline__ void unit_remap_iv(const MapTab<Q, NS>& t, float4 (*iv)[1 << Q], int lane,
+                                              const float* pd, const float* pz) {
+    constexpr int L = 1 << Q;
+    constexpr int E = NS * L;
+#pragma unroll
+    for (int e = lane; e < E; e += 32) {
+        const int k = e / L, c = e % L;
+        const int r = t.rk[k][c];
+        const int rl = r > 0 ? r - 1 : 0, rh = r < L - 1 ? r + 1 : L - 1;
+        const float y = t.lv[k][c], lo = t.srt[k][rl], hi = t.srt[k][rh];
+        const float zu = pz[k];
+        const float M = fmaxf(fabsf(t.srt[k][0]), fabsf(t.srt[k][L - 1]));
+        const float base = __fadd_rn(fabsf(zu), M);
+        const float ml = __fmul_rn(0.5f, __fadd_rn(lo, y));
+        const float mh = __fmul_rn(0.5f, __fadd_rn(y, hi));
+        const float a = lo == y ? -__int_as_float(0x7f800000)
+                                : __fadd_rn(ml, __fmaf_rn(__fadd_rn(fabsf(ml), base), 0x1p-18f, 0x1p-126f));
+        const float b = hi == y ? __int_as_float(0x7f800000)
+                                : __fsub_rn(mh, __fmaf_rn(__fadd_rn(fabsf(mh), base), 0x1p-18f, 0x1p-126f));
+        iv[k][c] = make_float4(a, b, __fmul_rn(pd[k], __fsub_rn(y, zu)), 0.f);
+    }
+    __syncwarp();
+}
+
+// Remap step of 4 consecutive elements of group slot `sub`: W^ into o[],
+// returns the 4 new code words packed as bytes (bits above q cleared).
+template <int Q, int NS>
+__device__ __forceinline__ uint32_t remap_vec4(const float w[4], const float s4[4], uint32_t cv,
+                                               const MapTab<Q, NS>& t, const float4 (*iv)[1 << Q], int sub,
+                                               float dl, float sr, float zu, float o[4]) {
+    constexpr int L = 1 << Q;
+    bool sure = true;
+    uint32_t nc = 0;
+#pragma unroll
+    for (int kq = 0; kq < 4; ++kq) {
+        const int c = (cv >> (8 * kq)) & (L - 1);
+        const float4 v = iv[sub][c];
+        const float den = __fmul_rn(__fmul_rn(dl, s4[kq]), sr);
+        const float x = __fadd_rn(__fmul_rn(w[kq], rcp_approx(den)), zu);
+        sure = sure & (x > v.x) & (x < v.y) & (fabsf(den) < 0x1p125f);
+        o[kq] = v.z;
+        nc |= uint32_t(c) << (8 * kq);
+    }
+    if (!sure) {
+        nc = 0;
+#pragma unroll
+        for (int kq = 0; kq < 4; ++kq) {
+            const int c = (cv >> (8 * kq)) & (L - 1);
+            const int r = t.rk[sub][c];
+            const int rl = r > 0 ? r - 1 : 0, rh = r < L - 1 ? r + 1 : L - 1;
+            float uu;
+            const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
+            float m = t.lv[sub][c];
+            float best = fabsf(__fsub_rn(x, m));
+            uint32_t code = c;
+            const float lo = t.srt[sub][rl];
+            const float dlo = fabsf(__fsub_rn(x, lo));
+            if (dlo < best) { best = dlo; m = lo; code = t.cor[sub][rl]; }
+            const float hi = t.srt[sub][rh];
+            const float dhi = fabsf(__fsub_rn(x, hi));
+            if (dhi < best) { m = hi; code = t.cor[sub][rh]; }
+            o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
+            nc |= code << (8 * kq);
+        }
+    }
+    return nc;
+}
+
 // Filter decisions of 4 elements whose x = nu / dv + z share the divisor dv
 // (OmniQuant's Delta_O, AWQ's Delta_A; App. E): u = nu / dv from r =
 // rcp_approx(dv) where the margin test above proves the decision equal to

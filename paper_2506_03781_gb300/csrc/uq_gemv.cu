@@ -108,6 +108,8 @@ bcq_gemv_partial_kernel(const uint32_t* __restrict__ PLANES, const float* __rest
     float* nib = lut + kLutFloats;                    // [4][16][32]
     float* xs = nib + kNibFloats;                     // [32][17]: lane l's columns at 17 l
     uint32_t* stages = reinterpret_cast<uint32_t*>(xs + kXsFloats);
+    // the tile sum (a programmatic dependent) may be scheduled now; it waits for this grid's results
+    asm volatile("griddepcontrol.launch_dependents;");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t = (int)(blockIdx.x % n_tiles);
     const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
@@ -314,6 +316,8 @@ bcq_gemv_tma_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_
     float* xs = nib + kNibFloats;                     // [32][17]
     unsigned char* stages = reinterpret_cast<unsigned char*>(xs + kXsFloats);
     unsigned long long* bars = reinterpret_cast<unsigned long long*>(stages + (size_t)kGemvWarps * NS * SB);
+    // the tile sum (a programmatic dependent) may be scheduled now; it waits for this grid's results
+    asm volatile("griddepcontrol.launch_dependents;");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int t = (int)(blockIdx.x % n_tiles);
     const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
@@ -469,6 +473,11 @@ constexpr int kWideMaxWarps = 16;
 constexpr int kWideStages = 2;
 constexpr int kWideHeadBytes = align_up(kWideXsBytes + kWideMaxWarps * kWideStages * 8, 128);   // x + mbarriers
 constexpr int kSmemOptIn = 227 * 1024;
+// A table build costs about as much as 64 rows.  Row blocks run over all the
+// tiles side by side (block b takes tile b mod n_tiles), so the blocks in flight
+// stream the same rows and DRAM pages: an equal split of (tile, row) pairs
+// over every SM, tile-major, measured slower (33.1 vs 29.7 us on 8192 x 28672).
+constexpr int kWideLutRows = 64;
 
 // Groups of one row inside one wide tile.
 __host__ __device__ constexpr int wide_tile_groups(int g) { return kWideCols / g; }
@@ -520,7 +529,7 @@ template <int Q, typename XT, int NGT>
 __global__ void __launch_bounds__(kWideMaxWarps * 32, 1)
 bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid_constant__ CUtensorMap tm_alpha,
                      const __grid_constant__ CUtensorMap tm_z, const void* __restrict__ X, float* __restrict__ PART,
-                     int64_t out, int n_in, int batch, int n_tiles, int64_t chunk) {
+                     int64_t out, int n_in, int batch, int n_tiles, int64_t rows_per_block) {
     constexpr int NW = wide_warps(Q, NGT);
     constexpr int NS = kWideStages;
     constexpr int SB = wide_stage_bytes(Q, NGT);
@@ -531,14 +540,13 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
     static_assert(NW >= 4 && SB % 128 == 0 && DYN <= kSmemOptIn, "wide layout");
     static_assert(NGT >= 4 && (NGT * Q * 4) % 16 == 0, "alpha* and z* boxes must span a multiple of 16 bytes");
     extern __shared__ __align__(128) unsigned char wsm[];
+    // the tile sum (a programmatic dependent) may be scheduled now; it waits for this grid's results
+    asm volatile("griddepcontrol.launch_dependents;");
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // This block's run of (tile, row) pairs, tile-major: [f0, f1).  It may
-    // span tiles; each maximal piece within one tile is a segment, with its
-    // own table build.
-    const int64_t total_rt = (int64_t)n_tiles * out;
-    const int64_t f0 = (int64_t)blockIdx.x * chunk;
-    const int64_t f1 = f0 + chunk < total_rt ? f0 + chunk : total_rt;
-    if (f0 >= f1) return;                                      // the whole block: before any barrier
+    const int t = (int)(blockIdx.x % n_tiles);
+    const int64_t r0 = (int64_t)(blockIdx.x / n_tiles) * rows_per_block;
+    const int nr = (int)(out - r0 < rows_per_block ? out - r0 : rows_per_block);
+    if (nr <= 0) return;                                       // the whole block: before any barrier
 
     // shared-memory layout (uniform over the block)
     const uint32_t D = tma::smem_addr(wsm);
@@ -560,32 +568,13 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
     const uint32_t st0 = i0 < n_gap ? lo + i0 * SB : hi + (i0 - n_gap) * SB;
     const uint32_t st1 = i1 < n_gap ? lo + i1 * SB : hi + (i1 - n_gap) * SB;
 
+    const int c0 = t * kWideCols;
+    const int nbat = (nr + kBatchRows - 1) / kBatchRows;
+    const int my_nb = warp < nbat ? (nbat - warp + NW - 1) / NW : 0;
     const uint32_t lane_base = L + 4u * (uint32_t)lane;        // bits 8..15 are zero
     const int gl = lane / LPG;                                 // this lane's group within the tile
     using SR = SegReduce<32>;
-    // a segment starting at flat index f: tile t, first row r, rows nr, this warp's batches nb
-    struct Seg {
-        int t, nb;
-        int64_t r, end;
-        int nr;
-    };
-    auto seg_at = [&](int64_t f) {
-        Seg g;
-        g.t = (int)(f / out);
-        g.r = f - (int64_t)g.t * out;
-        const int64_t te = (int64_t)(g.t + 1) * out;
-        g.end = f1 < te ? f1 : te;
-        g.nr = (int)(g.end - f);
-        const int nbat = (g.nr + kBatchRows - 1) / kBatchRows;
-        g.nb = warp < nbat ? (nbat - warp + NW - 1) / NW : 0;
-        return g;
-    };
-    int per_token = 0;                                         // this warp's batches over the segments
-    for (int64_t f = f0; f < f1;) {
-        const Seg g = seg_at(f);
-        per_token += g.nb;
-        f = g.end;
-    }
+
     if (lane == 0) {
 #pragma unroll
         for (int s = 0; s < NS; ++s) tma::bar_init(bar0 + 8u * s, 1);
@@ -593,109 +582,94 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
     }
     __syncwarp();
 
-    // items in order: token, segment, this warp's batch k of the segment (rows
-    // r + 8 (warp + NW k)); lane 0 issues them NS ahead of the computation
-    const int total = batch * per_token;
+    const int total = batch * my_nb;                           // items: token-major, this warp's batches
     int issued = 0, waited = 0, ik = 0;
-    int64_t if_ = f0;                                          // issue cursor: segment start, batch
-    Seg ig = seg_at(f0);
-    auto issue_next = [&]() {                                  // lane 0 only; issued < total
-        while (ik == ig.nb) {                                  // next segment (token) with batches here
-            if_ = ig.end < f1 ? ig.end : f0;
-            ig = seg_at(if_);
-            ik = 0;
-        }
+    auto issue_next = [&]() {                                  // lane 0 only
         const int s = issued & 1;
         const uint32_t bar = bar0 + 8u * s;
         const uint32_t d = s ? st1 : st0;
-        const int y = (int)(ig.r + (int64_t)kBatchRows * (warp + NW * ik));
+        const int y = (int)(r0 + (int64_t)kBatchRows * (warp + NW * ik));
         tma::fence_async_smem();                               // the warp's reads of this stage come first
         tma::bar_arrive_tx(bar, (uint32_t)SB);
-        tmap::load_3d(d, &tm_planes, ig.t * kWideWords, y, 0, bar);
-        tmap::load_2d(d + PLB, &tm_alpha, ig.t * NGT * Q, y, bar);
-        tmap::load_2d(d + PLB + ALB, &tm_z, ig.t * NGT, y, bar);
+        tmap::load_3d(d, &tm_planes, t * kWideWords, y, 0, bar);
+        tmap::load_2d(d + PLB, &tm_alpha, t * NGT * Q, y, bar);
+        tmap::load_2d(d + PLB + ALB, &tm_z, t * NGT, y, bar);
         ++issued;
-        ++ik;
+        if (++ik == my_nb) ik = 0;
     };
     if (lane == 0)
         while (issued < total && issued < NS) issue_next();
 
     bool alive = true;
-    int i = 0;                                                 // item being computed
     for (int b = 0; b < batch; ++b) {                          // token b is row b of X
-        for (int64_t f = f0; f < f1;) {
-            const Seg sg = seg_at(f);
-            f = sg.end;
-            const int c0 = sg.t * kWideCols;
-            __syncthreads();                                   // the previous segment's readers are done
-            for (int e = threadIdx.x; e < kWideCols; e += NW * 32)
-                xs[kWideXsStride * (e >> 5) + (e & 31)] = XT::get(X, (int64_t)b * n_in + c0 + e);
-            __syncthreads();
-            // tables: item (lane l, slot k, high nibble m) writes entries 16 m + n, n = 0..15
-            for (int it = threadIdx.x; it < 2048; it += NW * 32) {
-                const int l = it & 31, k = (it >> 5) & 3, m = it >> 7;
-                const float* xc = xs + kWideXsStride * l + 8 * k;
-                float x[8];
+        __syncthreads();                                       // the previous token's readers are done
+        for (int i = threadIdx.x; i < kWideCols; i += NW * 32)
+            xs[kWideXsStride * (i >> 5) + (i & 31)] = XT::get(X, (int64_t)b * n_in + c0 + i);
+        __syncthreads();
+        // tables: item (lane l, slot k, high nibble m) writes entries 16 m + n, n = 0..15
+        for (int it = threadIdx.x; it < 2048; it += NW * 32) {
+            const int l = it & 31, k = (it >> 5) & 3, m = it >> 7;
+            const float* xc = xs + kWideXsStride * l + 8 * k;
+            float x[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) x[e] = xc[e];
-                float lo4[16];
-                lo4[0] = 0.f;
+            for (int i = 0; i < 8; ++i) x[i] = xc[i];
+            float lo4[16];
+            lo4[0] = 0.f;
 #pragma unroll
-                for (int n = 1; n < 16; ++n) lo4[n] = __fadd_rn(lo4[n & (n - 1)], x[low_bit(n)]);
-                float h = (m & 1) ? x[4] : 0.f;
-                h = (m & 2) ? __fadd_rn(h, x[5]) : h;
-                h = (m & 4) ? __fadd_rn(h, x[6]) : h;
-                h = (m & 8) ? __fadd_rn(h, x[7]) : h;
-                float* dst = lut + (k >> 1) * 16384 + (k & 1) * 32 + l + 16 * m * 64;
+            for (int n = 1; n < 16; ++n) lo4[n] = __fadd_rn(lo4[n & (n - 1)], x[low_bit(n)]);
+            float h = (m & 1) ? x[4] : 0.f;
+            h = (m & 2) ? __fadd_rn(h, x[5]) : h;
+            h = (m & 4) ? __fadd_rn(h, x[6]) : h;
+            h = (m & 8) ? __fadd_rn(h, x[7]) : h;
+            float* dst = lut + (k >> 1) * 16384 + (k & 1) * 32 + l + 16 * m * 64;
 #pragma unroll
-                for (int n = 0; n < 16; ++n) dst[n * 64] = __fadd_rn(lo4[n], h);
-            }
-            __syncthreads();
-            // S = the sum of this lane's 32 x values (entry 255 of each slot)
-            const float S =
-                __fadd_rn(__fadd_rn(lds_f32(lane_base + 255u * 256u), lds_f32(lane_base + 255u * 256u + 128u)),
-                          __fadd_rn(lds_f32(lane_base + 65536u + 255u * 256u),
-                                    lds_f32(lane_base + 65536u + 255u * 256u + 128u)));
-            float* prow = PART + ((int64_t)sg.t * batch + b) * out + sg.r;
-            for (int k = 0; k < sg.nb; ++k, ++i) {
-                const int s = i & 1;
-                const uint32_t sa = s ? st1 : st0;
-                if (alive) {
-                    // one verdict for the whole warp (lanes poll the mbarrier separately)
-                    if (__all_sync(kFull, tma::bar_wait(bar0 + 8u * s, (uint32_t)((i >> 1) & 1)))) {
-                        ++waited;
-                    } else {
-                        alive = false;
-                        if (lane == 0) atomicOr(&g_gemv_err, 1u);
-                    }
+            for (int n = 0; n < 16; ++n) dst[n * 64] = __fadd_rn(lo4[n], h);
+        }
+        __syncthreads();
+        // S = the sum of this lane's 32 x values (entry 255 of each slot)
+        const float S = __fadd_rn(__fadd_rn(lds_f32(lane_base + 255u * 256u), lds_f32(lane_base + 255u * 256u + 128u)),
+                                  __fadd_rn(lds_f32(lane_base + 65536u + 255u * 256u),
+                                            lds_f32(lane_base + 65536u + 255u * 256u + 128u)));
+        float* prow = PART + ((int64_t)t * batch + b) * out + r0;
+        for (int k = 0; k < my_nb; ++k) {
+            const int i = b * my_nb + k;
+            const int s = i & 1;
+            const uint32_t sa = s ? st1 : st0;
+            if (alive) {
+                // one verdict for the whole warp (lanes poll the mbarrier separately)
+                if (__all_sync(kFull, tma::bar_wait(bar0 + 8u * s, (uint32_t)((i >> 1) & 1)))) {
+                    ++waited;
+                } else {
+                    alive = false;
+                    if (lane == 0) atomicOr(&g_gemv_err, 1u);
                 }
-                if (alive) {
-                    const uint32_t pw = sa + 4u * (uint32_t)lane;                      // this lane's plane words
-                    const uint32_t pa = sa + PLB + 4u * (uint32_t)(gl * Q);           // its group's alpha*
-                    const uint32_t pz = sa + PLB + ALB + 4u * (uint32_t)gl;           // and z*
-                    float v[kBatchRows];
-#pragma unroll
-                    for (int rr = 0; rr < kBatchRows; ++rr) {
-                        float acc = __fmul_rn(lds_f32(pz + 4u * (uint32_t)(rr * NGT)), S);
-#pragma unroll
-                        for (int j = 0; j < Q; ++j) {
-                            const uint32_t w = lds_u32(pw + 4u * (uint32_t)((j * kBatchRows + rr) * kWideWords));
-                            const float t0 = lds_f32(__byte_perm(w, lane_base, 0x7604));
-                            const float t1 = lds_f32(__byte_perm(w, lane_base, 0x7614) + 128u);
-                            const float t2 = lds_f32(__byte_perm(w, lane_base, 0x7624) + 65536u);
-                            const float t3 = lds_f32(__byte_perm(w, lane_base, 0x7634) + 65536u + 128u);
-                            const float P = __fadd_rn(__fadd_rn(t0, t1), __fadd_rn(t2, t3));
-                            acc = fmaf(lds_f32(pa + 4u * (uint32_t)(rr * NGT * Q + j)), fmaf(2.f, P, -S), acc);
-                        }
-                        v[rr] = acc;
-                    }
-                    const int rb = kBatchRows * (warp + NW * k);
-                    const int slot0 = SR::run(v, lane);
-                    if (SR::writer(lane) && rb + slot0 < sg.nr) prow[rb + slot0] = v[0];
-                }
-                __syncwarp();                                  // stage s is free for item i + NS
-                if (alive && lane == 0 && issued < total) issue_next();
             }
+            if (alive) {
+                const uint32_t pw = sa + 4u * (uint32_t)lane;                          // this lane's plane words
+                const uint32_t pa = sa + PLB + 4u * (uint32_t)(gl * Q);               // its group's alpha*
+                const uint32_t pz = sa + PLB + ALB + 4u * (uint32_t)gl;               // and z*
+                float v[kBatchRows];
+#pragma unroll
+                for (int rr = 0; rr < kBatchRows; ++rr) {
+                    float acc = __fmul_rn(lds_f32(pz + 4u * (uint32_t)(rr * NGT)), S);
+#pragma unroll
+                    for (int j = 0; j < Q; ++j) {
+                        const uint32_t w = lds_u32(pw + 4u * (uint32_t)((j * kBatchRows + rr) * kWideWords));
+                        const float t0 = lds_f32(__byte_perm(w, lane_base, 0x7604));
+                        const float t1 = lds_f32(__byte_perm(w, lane_base, 0x7614) + 128u);
+                        const float t2 = lds_f32(__byte_perm(w, lane_base, 0x7624) + 65536u);
+                        const float t3 = lds_f32(__byte_perm(w, lane_base, 0x7634) + 65536u + 128u);
+                        const float P = __fadd_rn(__fadd_rn(t0, t1), __fadd_rn(t2, t3));
+                        acc = fmaf(lds_f32(pa + 4u * (uint32_t)(rr * NGT * Q + j)), fmaf(2.f, P, -S), acc);
+                    }
+                    v[rr] = acc;
+                }
+                const int rb = kBatchRows * (warp + NW * k);
+                const int slot0 = SR::run(v, lane);
+                if (SR::writer(lane) && rb + slot0 < nr) prow[rb + slot0] = v[0];
+            }
+            __syncwarp();                                      // stage s is free for item i + NS
+            if (alive && lane == 0 && issued < total) issue_next();
         }
     }
     if (!alive && lane == 0) {
@@ -711,6 +685,10 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
 // y[b, r] = sum over tiles of PART[t, b, r], in tile order.
 __global__ void __launch_bounds__(256)
 bcq_gemv_reduce_kernel(const float* __restrict__ PART, float* __restrict__ Y, int64_t n, int n_tiles) {
+    // Launched as a programmatic dependent of the product kernel: it may start
+    // while that kernel still runs, and waits here until the product grid has
+    // completed and its partials are visible.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         float acc = 0.f;
         for (int t = 0; t < n_tiles; ++t) acc += __ldg(PART + (int64_t)t * n + i);
@@ -905,12 +883,24 @@ static void gemv_row_blocks(int64_t out, int n_tiles, int per_sm, int64_t& n_rb,
 }
 
 // y = the per-tile partials summed in tile order.
+// The tile sum is launched with programmatic stream serialization, so its
+// launch overlaps the end of the product kernel (it waits for that grid's
+// results with griddepcontrol.wait before reading them).
 static cudaError_t gemv_reduce(const float* work, float* y, int64_t n, int n_tiles, cudaStream_t st) {
     int64_t blocks = (n + 255) / 256;
     const int64_t cap = (int64_t)sm_count() * 8;
     if (blocks > cap) blocks = cap;
-    bcq_gemv_reduce_kernel<<<(unsigned)blocks, 256, 0, st>>>(work, y, n, n_tiles);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, bcq_gemv_reduce_kernel, work, y, n, n_tiles);
 }
 
 template <int Q, typename XT, int NGT>
@@ -986,14 +976,10 @@ static cudaError_t run_gemv_wide(const uint32_t* planes, const float* astar, con
         int per_sm = 0;
         cudaError_t e = gemv_blocks_per_sm<GemvWideTag<Q, XT, NGT>>(kern, DYN, per_sm, NW * 32);
         if (e != cudaSuccess) return e;
-        // one block per resident slot, each with an equal run of (tile, row) pairs
         const int n_tiles = n_in / kWideCols;
-        const int64_t total = (int64_t)n_tiles * out;
-        const int64_t slots = (int64_t)sm_count() * per_sm;
-        int64_t chunk = (total + slots - 1) / slots;
-        chunk = (chunk + kBatchRows - 1) / kBatchRows * kBatchRows;
-        const int64_t blocks = (total + chunk - 1) / chunk;
-        kern<<<(unsigned)blocks, NW * 32, DYN, st>>>(mp, ma, mz, x, work, out, n_in, batch, n_tiles, chunk);
+        int64_t n_rb = 0, rpb = 0;
+        gemv_row_blocks(out, n_tiles, per_sm, n_rb, rpb, (double)kWideLutRows);
+        kern<<<(unsigned)(n_rb * n_tiles), NW * 32, DYN, st>>>(mp, ma, mz, x, work, out, n_in, batch, n_tiles, rpb);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);

@@ -232,6 +232,8 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ MapTab<Q, NG> tabs[kWarps];
+    constexpr int NIV = mode == FWD_REMAP ? NG : 1;              // remap intervals only on remap steps
+    __shared__ float4 ivs[kWarps][NIV][L];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
@@ -301,8 +303,12 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
             }
             __syncwarp();
-            if constexpr (mode == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
-            else if constexpr (mode == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            if constexpr (mode == FWD_REMAP) {
+                unit_sort<Q, NG, false>(t, lane);
+                unit_remap_iv<Q, NG>(t, ivs[warp], lane, pd, pz);
+            } else if constexpr (mode == FWD_FULL) {
+                unit_sort<Q, NG, false>(t, lane);
+            }
             const float dl = pd[sub], zu = pz[sub];
             const float sr = need_x ? __ldg(SR + row) : 0.f;
             const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
@@ -329,23 +335,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
                     if constexpr (mode == FWD_REMAP) {
-#pragma unroll
-                        for (int kq = 0; kq < 4; ++kq) {
-                            const int c = (cv >> (8 * kq)) & (L - 1);
-                            const float4 nb = t.nb[sub][c];
-                            float uu;
-                            const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
-                            const uint32_t packed = __float_as_uint(nb.w);
-                            float best = fabsf(__fsub_rn(x, nb.y));
-                            float m = nb.y;
-                            uint32_t code = c;
-                            const float dlo = fabsf(__fsub_rn(x, nb.x));
-                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
-                            const float dhi = fabsf(__fsub_rn(x, nb.z));
-                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
-                            o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
-                            nc |= code << (8 * kq);
-                        }
+                        nc = remap_vec4<Q, NG>(w, s4, cv, t, ivs[warp], sub, dl, sr, zu, o);
                     } else {
 #pragma unroll
                         for (int kq = 0; kq < 4; ++kq) {

@@ -186,3 +186,30 @@ def check_init(W, q, g, G, clip, got, got_codes, ref, errs, chosen, label=""):
     print(f"init {label}: {same.mean():.6f} of {NG} groups bit-identical, {int(moved.sum())} near-tie gamma "
           f"choices, worst e' rel diff {rel.max():.2e}")
     return same.mean()
+
+
+def midpoint_weights(P, codes, g, seed, ulps=4):
+    """fp32 weights whose x = T_F(w) lies within `ulps` relative ulps of the
+    midpoint between each element's level and one of its two rank neighbours
+    (Algorithm 4's candidates d - 1, d + 1), about a tenth of them exactly on
+    it, so every local remap decision is taken by a hair or by the tie rule.
+    Built from the oracle's levels and sorted order; codes are the given ones."""
+    out, n_in = P["s"].shape
+    Gr = n_in // g
+    q = P["alpha"].shape[-1]
+    L = 1 << q
+    lv = O.levels(P["alpha"], P["zb"])
+    srt, _, rank_of_code = O.sorted_levels(lv)
+    c = (np.asarray(codes).reshape(out, Gr, g).astype(np.int64)) & (L - 1)
+    r = np.take_along_axis(rank_of_code, c, axis=-1)
+    rng = np.random.default_rng(seed)
+    rn = np.clip(r + rng.choice([-1, 1], r.shape), 0, L - 1)
+    l_c = np.take_along_axis(lv, c, axis=-1).astype(np.float64)
+    l_n = np.take_along_axis(srt, rn, axis=-1).astype(np.float64)
+    mid = 0.5 * (l_c + l_n)
+    k = rng.integers(-ulps, ulps + 1, mid.shape)
+    k[rng.random(mid.shape) < 0.1] = 0
+    x = mid + k * 2.0 ** -23 * np.abs(mid)
+    den = (np.asarray(P["delta"], np.float64)[..., None] * np.asarray(P["s"], np.float64).reshape(out, Gr, g)
+           * np.asarray(P["sr"], np.float64)[:, None, None])
+    return ((x - np.asarray(P["zu"], np.float64)[..., None]) * den).astype(F32).reshape(out, n_in)

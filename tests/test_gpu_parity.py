@@ -205,6 +205,23 @@ def test_exact_decision_ties_are_bit_exact():
     C.assert_fwd_equal(what, codes, r_what, r_codes, "exact ties")
 
 
+@pytest.mark.parametrize("q,g,n_in", [(1, 32, 1024), (2, 64, 1024), (3, 128, 2048), (4, 128, 1024), (3, 256, 1024)])
+def test_remap_near_level_midpoints_is_bit_exact(q, g, n_in):
+    """Every element within 4 ulps of the midpoint between its level and a
+    rank neighbour (some exactly on it): the remap step's codes and W^ must
+    be the oracle's bit for bit, whichever way the kernel forms x (the
+    pipelined kernels decide from the reciprocal only inside a proven
+    interval and fall back to the IEEE quotient and the three distances)."""
+    out = 24
+    _, W0, P, codes0, _ = C.make_inputs(out, n_in, q, g, seed=800 + 10 * q + g, wdtype="f32")
+    W = C.midpoint_weights(P, codes0, g, seed=q + g)
+    what, codes = C.gpu_fwd(W, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(what, codes, r_what, r_codes, f"midpoints q={q} g={g}")
+    assert (r_codes != codes0).mean() > 0.05         # many decisions go to the neighbour
+
+
 def test_deterministic_and_in_bounds():
     """Two identical calls give identical bits; outputs written into the middle
     of larger buffers leave the sentinel margins untouched."""

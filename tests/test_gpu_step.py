@@ -398,3 +398,21 @@ def test_step_bf16_io_equals_the_fp32_step(out, n_in, g, q):
             assert torch.equal(pa[k], pb[k]), (k, t)
         assert torch.equal(ca, cb), t
         assert torch.equal(wa.to(torch.bfloat16), wb), (t, int((wa.to(torch.bfloat16) != wb).sum()))
+
+
+@pytest.mark.parametrize("out,n_in,g,q", [(24, 1024, 128, 3), (16, 768, 32, 2), (6, 14336, 128, 4)])
+def test_step_remap_near_level_midpoints_is_bit_exact(out, n_in, g, q):
+    """With zero learning rates the update leaves every parameter unchanged,
+    so the forward of t + 1 remaps with the levels the weights were aimed at:
+    every element within 4 ulps of a midpoint between its level and a rank
+    neighbour.  Codes and W^ must be the oracle's bit for bit (phase B takes
+    the reciprocal only inside a proven interval, else the IEEE path)."""
+    _, W0, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=900 + out + q, wdtype="f32")
+    W = C.midpoint_weights(P, codes0, g, seed=out + q)
+    newP, c1, w1 = gpu_step(W, P, codes0, Gup, q, g, 1, O.MAP_LOCAL_PERIODIC, 2, lr_F=0.0, lr_B=0.0)
+    for k in PK:
+        assert np.array_equal(newP[k], P[k]), k
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 2, 2)
+    C.assert_fwd_equal(w1, c1, r_what, r_codes, f"step midpoints q={q} g={g}")
+    assert (r_codes != codes0).mean() > 0.05
