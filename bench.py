@@ -340,6 +340,61 @@ def time_oracle_parallel(wl, q, rows, budget_s, workers):
 # GPU run
 # ---------------------------------------------------------------------------
 
+def time_slabs(wl, q, steps, warmup, dev, seed=0, graph=True):
+    """time_matrices with the matrices of one input width stored as row ranges
+    of one slab (api.RowSlabs): per step one forward, one backward and one
+    export per width instead of per matrix (the Llama-3-8B block: 2 widths,
+    7 matrices)."""
+    import torch
+    from paper_2506_03781_gb300 import api, synth
+    g = wl.g
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 * wl.seed + q + 7 * seed)
+    slabs = api.RowSlabs({m.name: (m.out, m.n_in) for m in wl.matrices}, q, g,
+                         torch.bfloat16 if wl.wdtype == "bf16" else torch.float32, dev, with_export=True)
+    for idx, m in enumerate(wl.matrices):
+        raw, _ = synth.workload_weights(wl, idx)
+        slabs.view(m.name)["W"].copy_(api.weights_tensor(raw, dev))
+    slabs.init_params(G=wl.G, T=wl.T)
+    for d in slabs.slabs.values():
+        for k in ("delta", "s", "sr", "alpha"):
+            d["params"][k].mul_(1.0 + wl.init_eps * torch.randn(d["params"][k].shape, generator=gen, device=dev))
+        d["dL_dWhat"].copy_(torch.randn(d["dL_dWhat"].shape, generator=gen, device=dev) * float(np.sqrt(wl.grad_var)))
+
+    def step(t):
+        slabs.fwd(t, wl.p)
+        slabs.bwd()
+        slabs.export()
+
+    for t in range(warmup):
+        step(t)
+    torch.cuda.synchronize()
+    graphs = None
+    if graph:
+        side = torch.cuda.Stream(dev)
+        graphs = []
+        for t in (0, 1):
+            cg = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(cg, stream=side):
+                step(t)
+            graphs.append(cg)
+        torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(steps):
+        if graphs is not None:
+            graphs[(warmup + t) % wl.p != 0].replay()
+        else:
+            step(warmup + t)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    n = sum(m.out * m.n_in for m in wl.matrices)
+    del slabs, graphs
+    torch.cuda.empty_cache()
+    return e0.elapsed_time(e1) / steps, n, 3 * len({m.n_in for m in wl.matrices})
+
+
 def time_matrices(wl, q, steps, warmup, dev, with_export=False, seed=0, graph=False):
     """Times `steps` optimisation steps over every matrix of a workload, all
     launches back to back on one stream: per matrix the forward (local
@@ -1001,6 +1056,15 @@ def run_workloads(args):
             line = {"workload": name, "q": wl.q, "g": wl.g, "weights": n, "steps": args.steps,
                     "cuda_graph": graph, "ms_per_step": ms, "weights_per_s": n / (ms / 1e3),
                     "step": "per matrix: fwd (local mapping, remap/keep alternating) + bwd + bit-plane export",
+                    "cpu_baseline": cpu}
+            print(json.dumps(line))
+            lines.append(line)
+        if len({m.n_in for m in wl.matrices}) < len(wl.matrices):
+            ms, n, launches = time_slabs(wl, wl.q, args.steps, args.warmup, dev)
+            line = {"workload": name, "q": wl.q, "g": wl.g, "weights": n, "steps": args.steps,
+                    "cuda_graph": True, "ms_per_step": ms, "weights_per_s": n / (ms / 1e3),
+                    "step": f"grouped: the matrices of each input width as one row slab, fwd + bwd + bit-plane "
+                            f"export per width ({launches} calls per step)",
                     "cpu_baseline": cpu}
             print(json.dumps(line))
             lines.append(line)

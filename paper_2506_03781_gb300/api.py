@@ -492,6 +492,82 @@ def uq_bcq_gemv_noalloc(bitplanes, alpha_star, zb_star, x, y, g, stream=None):
     _raise(st)
 
 
+class RowSlabs:
+    """Several weight matrices quantized with one launch per input width.
+
+    Rows are independent (groups lie inside rows and s_r is per row), so the
+    matrices that share a number of columns are stored as consecutive row
+    ranges of one slab: W, Theta_IF, the codes, W^, dL/dW^ (and, on request,
+    the gradients and the export outputs) are one [sum of rows, in] tensor
+    per width, and every matrix's tensors are row views into them.  One call
+    per width then runs the forward, backward, fused step or export of all
+    its matrices with the persistent grid filled (a Llama-3-8B block's
+    1024-row k and v projections alone would leave most of the GPU idle),
+    and the results are bit for bit those of one call per matrix.  The views
+    of a matrix start on 16-byte boundaries when every matrix before it in
+    the slab has a multiple of 4 rows (true of the model shapes).
+
+    shapes: {name: (out, in)} in the order the matrices are laid out.
+    """
+
+    def __init__(self, shapes, q, g, w_dtype=torch.bfloat16, device="cuda", with_grads=True, with_export=False):
+        self.q, self.g, self.device = q, g, torch.device(device)
+        self.rows, widths = {}, {}
+        for name, (out, n_in) in shapes.items():
+            r0 = widths.get(n_in, 0)
+            self.rows[name] = (n_in, r0, r0 + out)
+            widths[n_in] = r0 + out
+        self.slabs = {}
+        for n_in, total in widths.items():
+            d = {"W": torch.empty(total, n_in, dtype=w_dtype, device=self.device),
+                 "params": empty_params(total, n_in, q, g, self.device),
+                 "codes": torch.empty(total, n_in, dtype=torch.uint8, device=self.device),
+                 "W_hat": torch.empty(total, n_in, dtype=torch.float32, device=self.device),
+                 "dL_dWhat": torch.zeros(total, n_in, dtype=torch.float32, device=self.device),
+                 "grads": empty_grads(total, n_in, q, g, self.device) if with_grads else None}
+            if with_export:
+                d["export"] = (torch.empty(q, total, n_in // 32, dtype=torch.int32, device=self.device),
+                               torch.empty(total, n_in // g, q, dtype=torch.float32, device=self.device),
+                               torch.empty(total, n_in // g, dtype=torch.float32, device=self.device))
+            d["qz"] = Quantizer(d["W"], q, g, d["params"], d["codes"], d["W_hat"], d["dL_dWhat"], d["grads"])
+            self.slabs[n_in] = d
+
+    def view(self, name):
+        """The matrix's tensors: row views of its slab (W, params, codes,
+        W_hat, dL_dWhat, grads, export)."""
+        n_in, r0, r1 = self.rows[name]
+        d = self.slabs[n_in]
+        v = {k: d[k][r0:r1] for k in ("W", "codes", "W_hat", "dL_dWhat")}
+        v["params"] = {k: t[r0:r1] for k, t in d["params"].items()}
+        v["grads"] = None if d["grads"] is None else {k: t[r0:r1] for k, t in d["grads"].items()}
+        if "export" in d:
+            planes, a_s, z_s = d["export"]
+            v["export"] = (planes[:, r0:r1], a_s[r0:r1], z_s[r0:r1])
+        return v
+
+    def init_params(self, G=30, T=15, clip=CLIP_FIXED_MIN, stream=None):
+        """Unified initialization of every matrix (one call per width)."""
+        for d in self.slabs.values():
+            uq_init_params(d["W"], self.q, self.g, d["params"], d["codes"], G=G, T=T, clip=clip, stream=stream)
+
+    def fwd(self, step, p_period=2, map_mode=MAP_LOCAL_PERIODIC, stream=None):
+        for d in self.slabs.values():
+            d["qz"].fwd(step, p_period, map_mode, stream)
+
+    def bwd(self, stream=None):
+        for d in self.slabs.values():
+            d["qz"].bwd(stream)
+
+    def train_step(self, step, lr_F=LR_THETA_F, lr_B=LR_THETA_B, p_period=2, map_mode=MAP_LOCAL_PERIODIC,
+                   stream=None):
+        for d in self.slabs.values():
+            d["qz"].train_step(step, lr_F, lr_B, p_period, map_mode, stream)
+
+    def export(self, mode=EXPORT_REUSE_CODES, stream=None):
+        for d in self.slabs.values():
+            d["qz"].export(*d["export"], mode=mode, stream=stream)
+
+
 # ---------------------------------------------------------------------------
 # buffer helpers
 # ---------------------------------------------------------------------------
