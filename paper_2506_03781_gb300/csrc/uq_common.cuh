@@ -345,14 +345,16 @@ __device__ __forceinline__ void bwd_vec4(const float w[4], const float s4[4], co
 //   w^ = Delta (l_c - z_U), the output of a kept code.
 // remap_vec4 forms x' = fl(fl(w r) + z_U) from the reciprocal estimate r of
 // den (as bwd_vec4 does; |x' - x| <= 2^-21 |x'| + 2^-22 |z_U| + 2^-148) and
-// keeps the codes of a vector of 4 elements when every x' lies in (a, b)
-// and every |den| < 2^125.  Then each x lies more than m / 2 from the
+// keeps an element's code when its x' lies in (a, b) and |den| < 2^125
+// (for the same element slot of every lane of the warp: the verdict is
+// taken per warp).  Then each x lies more than m / 2 from the
 // midpoint on a finite side, where the fp32 distances to the two levels
 // differ by more than m - 2^-22 M > 0, or beyond the level on that side
 // (the far level is then never strictly nearer: rounding is monotonic); so
-// the exact path keeps c as well.  Every other vector -- an element near a
-// midpoint, a den out of range, an infinity or a NaN (all comparisons
-// false) -- takes the exact path: transform_x and the three distances.
+// the exact path keeps c as well.  Every other element slot -- an element
+// near a midpoint, one whose code moves, a den out of range, an infinity or
+// a NaN (all comparisons false) -- takes the exact path: transform_x and
+// the three distances.
 template <int Q, int NS>
 __device__ __forceinline__ void unit_remap_iv(const MapTab<Q, NS>& t, float4 (*iv)[1 << Q], int lane,
                                               const float* pd, const float* pz) {
@@ -380,35 +382,32 @@ __device__ __forceinline__ void unit_remap_iv(const MapTab<Q, NS>& t, float4 (*i
 
 // Remap step of 4 consecutive elements of group slot `sub`: W^ into o[],
 // returns the 4 new code words packed as bytes (bits above q cleared).
+// Every lane of the warp must call it (the fallback verdicts are warp-wide).
 template <int Q, int NS>
 __device__ __forceinline__ uint32_t remap_vec4(const float w[4], const float s4[4], uint32_t cv,
                                                const MapTab<Q, NS>& t, const float4 (*iv)[1 << Q], int sub,
                                                float dl, float sr, float zu, float o[4]) {
     constexpr int L = 1 << Q;
-    bool sure = true;
     uint32_t nc = 0;
 #pragma unroll
     for (int kq = 0; kq < 4; ++kq) {
         const int c = (cv >> (8 * kq)) & (L - 1);
         const float4 v = iv[sub][c];
         const float den = __fmul_rn(__fmul_rn(dl, s4[kq]), sr);
-        const float x = __fadd_rn(__fmul_rn(w[kq], rcp_approx(den)), zu);
-        sure = sure & (x > v.x) & (x < v.y) & (fabsf(den) < 0x1p125f);
+        const float xa = __fadd_rn(__fmul_rn(w[kq], rcp_approx(den)), zu);
+        const bool sure = (xa > v.x) & (xa < v.y) & (fabsf(den) < 0x1p125f);
+        uint32_t code = c;
         o[kq] = v.z;
-        nc |= uint32_t(c) << (8 * kq);
-    }
-    if (!sure) {
-        nc = 0;
-#pragma unroll
-        for (int kq = 0; kq < 4; ++kq) {
-            const int c = (cv >> (8 * kq)) & (L - 1);
+        // One verdict per element slot and warp: the warp redoes element kq of
+        // its lanes with the exact path when any of them is unsure (the exact
+        // path gives the same result where the interval already decided).
+        if (__any_sync(kFull, !sure)) {
             const int r = t.rk[sub][c];
             const int rl = r > 0 ? r - 1 : 0, rh = r < L - 1 ? r + 1 : L - 1;
             float uu;
             const float x = transform_x(w[kq], s4[kq], dl, sr, zu, uu);
             float m = t.lv[sub][c];
             float best = fabsf(__fsub_rn(x, m));
-            uint32_t code = c;
             const float lo = t.srt[sub][rl];
             const float dlo = fabsf(__fsub_rn(x, lo));
             if (dlo < best) { best = dlo; m = lo; code = t.cor[sub][rl]; }
@@ -416,8 +415,8 @@ __device__ __forceinline__ uint32_t remap_vec4(const float w[4], const float s4[
             const float dhi = fabsf(__fsub_rn(x, hi));
             if (dhi < best) { m = hi; code = t.cor[sub][rh]; }
             o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
-            nc |= code << (8 * kq);
         }
+        nc |= code << (8 * kq);
     }
     return nc;
 }
