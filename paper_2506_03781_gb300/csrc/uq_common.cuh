@@ -337,6 +337,8 @@ __device__ __forceinline__ void bwd_vec4(const float w[4], const float s4[4], co
 // On a remap step the code word c of an element is kept unless the level
 // below it (rank r - 1) or above it (rank r + 1) is strictly nearer to the
 // IEEE value x = fl(fl(w / den) + z_U) (the tie rules of the exact path).
+// Used by the pipelined forward; the fused step keeps the exact path (the
+// interval test made its register-bound kernel no faster).
 // Per group slot k and code word c, unit_remap_iv stores iv = (a, b, w^, 0):
 //   a = mid(l_lo, l_c) + m_lo, b = mid(l_c, l_hi) - m_hi  (fp32), with
 //   mid(p, q) = 0.5 (p + q) and m = 2^-18 (|mid| + |z_U| + M) + 2^-126,

@@ -66,14 +66,9 @@ namespace cg = cooperative_groups;
 constexpr int kMaxCluster = 8;     // portable cluster size limit
 
 template <int Q, int NG>
-struct StepTabB {
-    MapTab<Q, NG> m;               // levels, sorted order
-    float4 iv[NG][1 << Q];         // remap intervals (unit_remap_iv)
-};
-template <int Q, int NG>
 union StepTab {
     float2 a[NG][1 << Q];          // phase A: (l(c), l(c) - z_U) per group slot and code word
-    StepTabB<Q, NG> b;             // phase B
+    MapTab<Q, NG> b;               // phase B: levels, sorted order, local-mapping neighbours
 };
 
 __device__ __forceinline__ void step_sync(int csize) {
@@ -270,21 +265,17 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                 float a[Q];
 #pragma unroll
                 for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
-                t.b.m.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+                t.b.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
             }
             __syncwarp();
-            if constexpr (MODEB == FWD_REMAP) {
-                unit_sort<Q, NG, false>(t.b.m, lane);
-                unit_remap_iv<Q, NG>(t.b.m, t.b.iv, lane, pd, pz);
-            } else if constexpr (MODEB == FWD_FULL) {
-                unit_sort<Q, NG, false>(t.b.m, lane);
-            }
+            if constexpr (MODEB == FWD_REMAP) unit_sort<Q, NG, true>(t.b, lane);
+            else if constexpr (MODEB == FWD_FULL) unit_sort<Q, NG, false>(t.b, lane);
             const float dl = pd[sub], zu = pz[sub];
             const int64_t ebase = row * n_in + (int64_t)unit * UE;
             float srt[L];
             if constexpr (MODEB == FWD_FULL) {
 #pragma unroll
-                for (int r = 0; r < L; ++r) srt[r] = t.b.m.srt[sub][r];
+                for (int r = 0; r < L; ++r) srt[r] = t.b.srt[sub][r];
             }
 #pragma unroll
             for (int v = 0; v < NV; ++v) {
@@ -295,7 +286,7 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
 #pragma unroll
                     for (int kq = 0; kq < 4; ++kq) {
                         const int c = (cv >> (8 * kq)) & (L - 1);
-                        o[kq] = __fmul_rn(dl, __fsub_rn(t.b.m.lv[sub][c], zu));
+                        o[kq] = __fmul_rn(dl, __fsub_rn(t.b.lv[sub][c], zu));
                     }
                 } else {
                     float w[4], s4[4];
@@ -303,7 +294,23 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                     WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
                     if constexpr (MODEB == FWD_REMAP) {
-                        nc = remap_vec4<Q, NG>(w, s4, cv, t.b.m, t.b.iv, sub, dl, sr_new, zu, o);
+#pragma unroll
+                        for (int kq = 0; kq < 4; ++kq) {
+                            const int c = (cv >> (8 * kq)) & (L - 1);
+                            const float4 nb = t.b.nb[sub][c];
+                            float uu;
+                            const float x = transform_x(w[kq], s4[kq], dl, sr_new, zu, uu);
+                            const uint32_t packed = __float_as_uint(nb.w);
+                            float best = fabsf(__fsub_rn(x, nb.y));
+                            float m = nb.y;
+                            uint32_t code = c;
+                            const float dlo = fabsf(__fsub_rn(x, nb.x));
+                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
+                            const float dhi = fabsf(__fsub_rn(x, nb.z));
+                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                            o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
+                            nc |= code << (8 * kq);
+                        }
                     } else {
 #pragma unroll
                         for (int kq = 0; kq < 4; ++kq) {
@@ -311,7 +318,7 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                             const float x = transform_x(w[kq], s4[kq], dl, sr_new, zu, uu);
                             const int r = nearest_rank<L>(x, srt, m);
                             o[kq] = __fmul_rn(dl, __fsub_rn(m, zu));
-                            nc |= uint32_t(t.b.m.cor[sub][r]) << (8 * kq);
+                            nc |= uint32_t(t.b.cor[sub][r]) << (8 * kq);
                         }
                     }
                     *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
