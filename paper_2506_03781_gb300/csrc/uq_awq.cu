@@ -288,6 +288,8 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ MapTab<Q, NG> tabs[kWarps];
+    constexpr int NIV = MODE == FWD_REMAP ? NG : 1;              // remap intervals only on remap steps
+    __shared__ float4 ivs[kWarps][NIV][L];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
@@ -336,8 +338,12 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
                 t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
             }
             __syncwarp();
-            if constexpr (MODE == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
-            else if constexpr (MODE == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            if constexpr (MODE == FWD_REMAP) {
+                unit_sort<Q, NG, false>(t, lane);
+                unit_remap_iv<Q, NG>(t, ivs[warp], lane, pd, pz);
+            } else if constexpr (MODE == FWD_FULL) {
+                unit_sort<Q, NG, false>(t, lane);
+            }
             const float dl = pd[sub], za = pz[sub];
             const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
             float srt[L];
@@ -356,33 +362,32 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
                 if constexpr (MODE != FWD_FULL) cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
                 float o[4];
                 uint32_t nc = 0;
+                if constexpr (MODE == FWD_REMAP) {
+                    // x = (w s_A) / Delta_A + z_A: the interval test on the numerator w s_A
+                    // with s = s_r = 1; W^ = (Delta_A (l - z_A)) / s_A
+                    const float one[4] = {1.f, 1.f, 1.f, 1.f};
+                    float nu[4];
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float m;
-                    uint32_t code;
-                    if constexpr (MODE == FWD_KEEP) {
-                        code = (cv >> (8 * k)) & (L - 1);
-                        m = t.lv[sub][code];
-                    } else {
-                        const float x = __fadd_rn(__fdiv_rn(__fmul_rn(w[k], s4[k]), dl), za);
-                        if constexpr (MODE == FWD_REMAP) {
-                            const int c = (cv >> (8 * k)) & (L - 1);
-                            const float4 nb = t.nb[sub][c];
-                            const uint32_t packed = __float_as_uint(nb.w);
-                            float best = fabsf(__fsub_rn(x, nb.y));
-                            m = nb.y;
-                            code = c;
-                            const float dlo = fabsf(__fsub_rn(x, nb.x));
-                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
-                            const float dhi = fabsf(__fsub_rn(x, nb.z));
-                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                    for (int k = 0; k < 4; ++k) nu[k] = __fmul_rn(w[k], s4[k]);
+                    nc = remap_vec4<Q, NG>(nu, one, cv, t, ivs[warp], sub, dl, 1.f, za, o);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) o[k] = __fdiv_rn(o[k], s4[k]);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        float m;
+                        uint32_t code;
+                        if constexpr (MODE == FWD_KEEP) {
+                            code = (cv >> (8 * k)) & (L - 1);
+                            m = t.lv[sub][code];
                         } else {
+                            const float x = __fadd_rn(__fdiv_rn(__fmul_rn(w[k], s4[k]), dl), za);
                             const int r = nearest_rank<L>(x, srt, m);
                             code = t.cor[sub][r];
                         }
+                        o[k] = __fdiv_rn(__fmul_rn(dl, __fsub_rn(m, za)), s4[k]);
+                        nc |= code << (8 * k);
                     }
-                    o[k] = __fdiv_rn(__fmul_rn(dl, __fsub_rn(m, za)), s4[k]);
-                    nc |= code << (8 * k);
                 }
                 if constexpr (MODE != FWD_KEEP) *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);

@@ -300,6 +300,9 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ MapTab<Q, NG> tabs[kWarps];
+    constexpr int NIV = MODE == FWD_REMAP ? NG : 1;              // remap intervals only on remap steps
+    __shared__ float4 ivs[kWarps][NIV][L];
+    __shared__ float dzs[kWarps][2][NIV];                        // Delta_O, z_O per group slot
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
@@ -362,8 +365,16 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 t.lv[kk][c] = level_of<Q>(c, a, pb[kk]);
             }
             __syncwarp();
-            if constexpr (MODE == FWD_REMAP) unit_sort<Q, NG, true>(t, lane);
-            else if constexpr (MODE == FWD_FULL) unit_sort<Q, NG, false>(t, lane);
+            if constexpr (MODE == FWD_REMAP) {
+                if (li == 0) {
+                    dzs[warp][0][sub] = dl;
+                    dzs[warp][1][sub] = zo;
+                }
+                unit_sort<Q, NG, false>(t, lane);
+                unit_remap_iv<Q, NG>(t, ivs[warp], lane, dzs[warp][0], dzs[warp][1]);
+            } else if constexpr (MODE == FWD_FULL) {
+                unit_sort<Q, NG, false>(t, lane);
+            }
             const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
             float srt[L];
             if constexpr (MODE == FWD_FULL) {
@@ -377,33 +388,26 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 if constexpr (MODE != FWD_FULL) cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
                 float o[4];
                 uint32_t nc = 0;
+                if constexpr (MODE == FWD_REMAP) {
+                    // x = w / Delta_O + z_O: the interval test with s = s_r = 1
+                    const float one[4] = {1.f, 1.f, 1.f, 1.f};
+                    nc = remap_vec4<Q, NG>(w[v], one, cv, t, ivs[warp], sub, dl, 1.f, zo, o);
+                } else {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float m;
-                    uint32_t code;
-                    if constexpr (MODE == FWD_KEEP) {
-                        code = (cv >> (8 * k)) & (L - 1);
-                        m = t.lv[sub][code];
-                    } else {
-                        const float x = __fadd_rn(__fdiv_rn(w[v][k], dl), zo);
-                        if constexpr (MODE == FWD_REMAP) {
-                            const int c = (cv >> (8 * k)) & (L - 1);
-                            const float4 nb = t.nb[sub][c];
-                            const uint32_t packed = __float_as_uint(nb.w);
-                            float best = fabsf(__fsub_rn(x, nb.y));
-                            m = nb.y;
-                            code = c;
-                            const float dlo = fabsf(__fsub_rn(x, nb.x));
-                            if (dlo < best) { best = dlo; m = nb.x; code = packed & 0xffu; }
-                            const float dhi = fabsf(__fsub_rn(x, nb.z));
-                            if (dhi < best) { m = nb.z; code = (packed >> 8) & 0xffu; }
+                    for (int k = 0; k < 4; ++k) {
+                        float m;
+                        uint32_t code;
+                        if constexpr (MODE == FWD_KEEP) {
+                            code = (cv >> (8 * k)) & (L - 1);
+                            m = t.lv[sub][code];
                         } else {
+                            const float x = __fadd_rn(__fdiv_rn(w[v][k], dl), zo);
                             const int r = nearest_rank<L>(x, srt, m);
                             code = t.cor[sub][r];
                         }
+                        o[k] = __fmul_rn(dl, __fsub_rn(m, zo));
+                        nc |= code << (8 * k);
                     }
-                    o[k] = __fmul_rn(dl, __fsub_rn(m, zo));
-                    nc |= code << (8 * k);
                 }
                 if constexpr (MODE != FWD_KEEP) *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);

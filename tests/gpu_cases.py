@@ -188,6 +188,27 @@ def check_init(W, q, g, G, clip, got, got_codes, ref, errs, chosen, label=""):
     return same.mean()
 
 
+def midpoint_targets(alpha, zb, codes, g, seed, ulps=4):
+    """fp64 targets x [out, in/g, g]: for each element, the midpoint between its
+    level and one of its two rank neighbours (Algorithm 4's d - 1, d + 1),
+    moved by up to `ulps` relative ulps (a tenth exactly on it)."""
+    q = np.asarray(alpha).shape[-1]
+    L = 1 << q
+    out, Gr = np.asarray(zb).shape
+    lv = O.levels(alpha, zb)
+    srt, _, rank_of_code = O.sorted_levels(lv)
+    c = (np.asarray(codes).reshape(out, Gr, g).astype(np.int64)) & (L - 1)
+    r = np.take_along_axis(rank_of_code, c, axis=-1)
+    rng = np.random.default_rng(seed)
+    rn = np.clip(r + rng.choice([-1, 1], r.shape), 0, L - 1)
+    l_c = np.take_along_axis(lv, c, axis=-1).astype(np.float64)
+    l_n = np.take_along_axis(srt, rn, axis=-1).astype(np.float64)
+    mid = 0.5 * (l_c + l_n)
+    k = rng.integers(-ulps, ulps + 1, mid.shape)
+    k[rng.random(mid.shape) < 0.1] = 0
+    return mid + k * 2.0 ** -23 * np.abs(mid)
+
+
 def midpoint_weights(P, codes, g, seed, ulps=4):
     """fp32 weights whose x = T_F(w) lies within `ulps` relative ulps of the
     midpoint between each element's level and one of its two rank neighbours
@@ -213,3 +234,34 @@ def midpoint_weights(P, codes, g, seed, ulps=4):
     den = (np.asarray(P["delta"], np.float64)[..., None] * np.asarray(P["s"], np.float64).reshape(out, Gr, g)
            * np.asarray(P["sr"], np.float64)[:, None, None])
     return ((x - np.asarray(P["zu"], np.float64)[..., None]) * den).astype(F32).reshape(out, n_in)
+
+
+def omni_midpoint_weights(W, P, codes, g, seed, ulps=4):
+    """OmniQuant's maps: weights whose x = w / Delta_O + z_O lies at level
+    midpoints (midpoint_targets).  Every group keeps its smallest and largest
+    weight, so Delta_O and z_O (functions of w_m, w_M) are unchanged; the
+    other weights move to a target when it lies strictly inside (w_m, w_M)."""
+    W = np.asarray(W, F32)
+    out, n_in = W.shape
+    Gr = n_in // g
+    d, zo = O.omni_params(W, P["beta"], P["gamma"], P["alpha"].shape[-1], g)
+    x = midpoint_targets(P["alpha"], P["zb"], codes, g, seed, ulps)
+    Wg = W.reshape(out, Gr, g).copy()
+    cand = ((x - np.asarray(zo, np.float64)[..., None]) * np.asarray(d, np.float64)[..., None]).astype(F32)
+    lo, hi = Wg.min(-1, keepdims=True), Wg.max(-1, keepdims=True)
+    ok = (cand > lo) & (cand < hi) & (Wg != lo) & (Wg != hi)    # the extremes stay
+    Wn = np.where(ok, cand, Wg).reshape(out, n_in)
+    d2, z2 = O.omni_params(Wn, P["beta"], P["gamma"], P["alpha"].shape[-1], g)
+    assert np.array_equal(d2, d) and np.array_equal(z2, zo)
+    return Wn, ok.mean()
+
+
+def awq_midpoint_weights(P, codes, g, seed, ulps=4):
+    """AWQ's maps: weights whose x = (w s_A) / Delta_A + z_A lies at level
+    midpoints (midpoint_targets)."""
+    out, Gr = np.asarray(P["zb"]).shape
+    n_in = Gr * g
+    x = midpoint_targets(P["alpha"], P["zb"], codes, g, seed, ulps)
+    w = ((x - np.asarray(P["za"], np.float64)[..., None]) * np.asarray(P["delta"], np.float64)[..., None]
+         / np.asarray(P["sa"], np.float64).reshape(1, Gr, g))
+    return w.astype(F32).reshape(out, n_in)

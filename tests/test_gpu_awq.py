@@ -137,3 +137,22 @@ def test_awq_backward_rejects_a_small_workspace():
         api.uq_quantize_bwd_awq(Wd, 2, 64, dev_params(P), torch.from_numpy(codes).cuda(), torch.from_numpy(Gup).cuda(),
                                 gr, workspace=torch.empty(4, device=C.dev()))
     assert e.value.status == api.UQ_ERR_ARG
+
+
+@pytest.mark.parametrize("q,g,n_in", [(1, 32, 1024), (2, 64, 1024), (3, 128, 2048), (4, 128, 1024)])
+def test_awq_remap_near_level_midpoints_is_bit_exact(q, g, n_in):
+    """Weights aimed within 4 ulps of the midpoints between each element's
+    level and a rank neighbour: the remap step's codes and W^ are the
+    oracle's bit for bit (the pipelined forward decides from the reciprocal
+    of Delta_A only inside a proven interval)."""
+    out = 24
+    _, _, P, codes, _ = inputs(out, n_in, q, g, seed=600 + q + g, wdtype="f32")
+    W = C.awq_midpoint_weights(P, codes, g, seed=q + g)
+    Wd = api.weights_tensor(W, C.dev())
+    cd = torch.from_numpy(codes.copy()).cuda()
+    what = torch.full((out, n_in), float("nan"), device=C.dev())
+    api.uq_quantize_fwd_awq(Wd, q, g, dev_params(P), cd, what, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd_awq(W, P["sa"], P["delta"], P["za"], P["alpha"], P["zb"], codes, g,
+                                         O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(C.host(what), C.host(cd), r_what, r_codes, f"awq midpoints q={q} g={g}")
+    assert (r_codes != codes).mean() > 0.05

@@ -143,3 +143,24 @@ def test_omni_unsupported_group_size_raises():
         api.uq_quantize_fwd_omni(Wd, 2, 1024, dev_params(P), torch.from_numpy(codes).cuda(),
                                  torch.empty(4, 2048, device=C.dev()))
     assert e.value.status == api.UQ_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("q,g,n_in", [(1, 32, 1024), (2, 64, 1024), (3, 128, 2048), (4, 128, 1024)])
+def test_omni_remap_near_level_midpoints_is_bit_exact(q, g, n_in):
+    """Weights aimed within 4 ulps of the midpoints between each element's
+    level and a rank neighbour (the group's extremes kept, so Delta_O and z_O
+    do not move): the remap step's codes and W^ are the oracle's bit for bit
+    (the pipelined forward decides from the reciprocal of Delta_O only inside
+    a proven interval)."""
+    out = 24
+    _, W0, P, codes, _ = inputs(out, n_in, q, g, seed=500 + q + g, wdtype="f32")
+    W, moved_share = C.omni_midpoint_weights(W0, P, codes, g, seed=q + g)
+    assert moved_share > 0.5
+    Wd = api.weights_tensor(W, C.dev())
+    cd = torch.from_numpy(codes.copy()).cuda()
+    what = torch.full((out, n_in), float("nan"), device=C.dev())
+    api.uq_quantize_fwd_omni(Wd, q, g, dev_params(P), cd, what, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd_omni(W, P["beta"], P["gamma"], P["alpha"], P["zb"], codes, g,
+                                          O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(C.host(what), C.host(cd), r_what, r_codes, f"omni midpoints q={q} g={g}")
+    assert (r_codes != codes).mean() > 0.05
