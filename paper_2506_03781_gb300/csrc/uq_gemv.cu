@@ -537,7 +537,9 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
     constexpr int ALB = kBatchRows * NGT * Q * 4;              // alpha* of a stage
     constexpr int DYN = wide_smem_bytes(Q, NGT);
     constexpr int LPG = 32 / NGT;                              // lanes per group
-    static_assert(NW >= 4 && SB % 128 == 0 && DYN <= kSmemOptIn, "wide layout");
+    // every tensor-copy destination (stage, alpha*, z*) on a 128-byte boundary
+    static_assert(NW >= 4 && SB % 128 == 0 && PLB % 128 == 0 && ALB % 128 == 0 && DYN <= kSmemOptIn,
+                  "wide layout");
     static_assert(NGT >= 4 && (NGT * Q * 4) % 16 == 0, "alpha* and z* boxes must span a multiple of 16 bytes");
     extern __shared__ __align__(128) unsigned char wsm[];
     // the tile sum (a programmatic dependent) may be scheduled now; it waits for this grid's results
