@@ -53,6 +53,42 @@ export_kernel(const void* __restrict__ W, const float* __restrict__ DELTA, const
         ZSTAR[grp] = OT::cvt(__fmul_rn(d, __fsub_rn(__ldg(ZB + grp), __ldg(ZU + grp))));
     }
 
+    if constexpr (!EQ4) {
+        if ((words & 3) == 0) {
+            // Four words per thread (128 columns): eight 16-byte loads of code
+            // bytes in flight, one 16-byte store of four words per plane.
+            const int quads = words >> 2;
+            const int64_t qstep_rows = nthr / quads;
+            const int qstep_cols = (int)(nthr - qstep_rows * quads);
+            int64_t qrow = tid / quads;
+            int qcol = (int)(tid - qrow * quads);
+            for (int64_t ch = tid; ch < out * quads; ch += nthr) {
+                const uint4* src = reinterpret_cast<const uint4*>(CODES + qrow * n_in + (int64_t)qcol * 128);
+                uint4 a[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) a[k] = __ldg(src + k);
+#pragma unroll
+                for (int j = 0; j < Q; ++j) {
+                    uint32_t wq[4];
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const uint4 x = a[2 * h], y = a[2 * h + 1];
+                        wq[h] = gather_bit(x.x & kMask, j) | (gather_bit(x.y & kMask, j) << 4) |
+                                (gather_bit(x.z & kMask, j) << 8) | (gather_bit(x.w & kMask, j) << 12) |
+                                (gather_bit(y.x & kMask, j) << 16) | (gather_bit(y.y & kMask, j) << 20) |
+                                (gather_bit(y.z & kMask, j) << 24) | (gather_bit(y.w & kMask, j) << 28);
+                    }
+                    *reinterpret_cast<uint4*>(PLANES + ((int64_t)j * out + qrow) * words + (int64_t)qcol * 4) =
+                        make_uint4(wq[0], wq[1], wq[2], wq[3]);
+                }
+                qrow += qstep_rows;
+                qcol += qstep_cols;
+                if (qcol >= quads) { qcol -= quads; ++qrow; }
+            }
+            return;
+        }
+    }
+
     // (row, wcol) of chunk ch = row * words + wcol, advanced by nthr chunks
     // per iteration without dividing inside the loop.
     const int64_t step_rows = nthr / words;
@@ -129,7 +165,8 @@ static int export_grid(int64_t work) {
 template <int Q, typename WT, bool EQ4, typename OT>
 static cudaError_t run_export(const Shape& sh, const void* W, uq_params p, const uint8_t* codes, uint32_t* planes,
                               typename OT::T* astar, typename OT::T* zstar, cudaStream_t st) {
-    const int grid = export_grid(sh.out * (int64_t)(sh.n_in / 32));
+    const int64_t words = sh.n_in / 32;
+    const int grid = export_grid(sh.out * (!EQ4 && (words & 3) == 0 ? words / 4 : words));
     export_kernel<Q, WT, EQ4, OT><<<grid, kThreads, 0, st>>>(W, p.delta, p.zu, p.alpha, p.zb, codes, planes, astar,
                                                              zstar, sh.out, sh.n_in, sh.g);
     return cudaGetLastError();
