@@ -302,26 +302,12 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
         tma::bar_init_fence();
     }
     __syncwarp();
-    Cursor ic;
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            awq_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, CODES, DELTA, ZA, ZB, ALPHA, out,
-                             n_in, Gr);
-            ic.next(it.n_w);
-        }
-    }
-    Ring<NST> ring;
-    Cursor cc;
-    for (long long i = 0; i < it.total; ++i) {
-        const int s = ring.s;
-        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
-            if (lane == 0) {
-                atomicOr(&g_awq_err, 1u);
-                if (!drain(bars[warp], i, issued)) atomicOr(&g_awq_err, kDrainTimeoutBit);
-            }
-            return;                                      // no block barrier in this kernel
-        }
+    auto issue = [&](const Cursor& c, int s) {          // lane 0 only
+        awq_issue<Q, St>(it, c, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, CODES, DELTA, ZA, ZB, ALPHA, out, n_in,
+                         Gr);
+    };
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_awq_err, 1u, issue,
+                                  [&](const Cursor& cc, int s) {
         const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -393,16 +379,8 @@ awq_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
             }
         }
-        __syncwarp();
-        if (lane == 0 && issued < it.total) {
-            awq_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, CODES, DELTA, ZA, ZB, ALPHA, out,
-                             n_in, Gr);
-            ic.next(it.n_w);
-            ++issued;
-        }
-        ring.next();
-        cc.next(it.n_w);
-    }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
 }
 
 template <int Q, typename WT, int G_, int MODE>
@@ -521,32 +499,18 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
         tma::bar_init_fence();
     }
     __syncwarp();
-    Cursor ic;
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            awq_bwd_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, GUP, CODES, DELTA, ZA, ZB,
-                                 ALPHA, out, n_in, Gr);
-            ic.next(it.n_w);
-        }
-    }
+    auto issue = [&](const Cursor& c, int s) {          // lane 0 only
+        awq_bwd_issue<Q, St>(it, c, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, GUP, CODES, DELTA, ZA, ZB, ALPHA,
+                             out, n_in, Gr);
+    };
     float rs[NV][4], dsa[NV][4];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
         for (int k = 0; k < 4; ++k) { rs[v][k] = 0.f; dsa[v][k] = 0.f; }
     bool have_rs = false;
-    Ring<NST> ring;
-    Cursor cc;
-    for (long long i = 0; i < it.total; ++i) {
-        const int s = ring.s;
-        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
-            if (lane == 0) {
-                atomicOr(&g_awq_err, 2u);
-                if (!drain(bars[warp], i, issued)) atomicOr(&g_awq_err, kDrainTimeoutBit);
-            }
-            return;                                      // no block barrier in this kernel
-        }
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_awq_err, 2u, issue,
+                                  [&](const Cursor& cc, int s) {
         const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -633,16 +597,8 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
                 }
             }
         }
-        __syncwarp();                                    // stage and tables are free again
-        if (lane == 0 && issued < it.total) {
-            awq_bwd_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, SA, GUP, CODES, DELTA, ZA, ZB,
-                                 ALPHA, out, n_in, Gr);
-            ic.next(it.n_w);
-            ++issued;
-        }
-        ring.next();
-        cc.next(it.n_w);
-    }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
     // this (block, row slot)'s ds_A partials of the warp's columns (zeros if it had no row)
     if (it.n_w > 0) {
         float* prow = PART + ((int64_t)blockIdx.x * R + it.row_sub) * n_in + (int64_t)it.unit(0) * UE;

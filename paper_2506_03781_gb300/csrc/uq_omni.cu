@@ -315,26 +315,12 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
         tma::bar_init_fence();
     }
     __syncwarp();
-    Cursor ic;
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            omni_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, nullptr, CODES, BETA, GAMMA, ZB, ALPHA,
-                           out, n_in, Gr);
-            ic.next(it.n_w);
-        }
-    }
-    Ring<NST> ring;
-    Cursor cc;
-    for (long long i = 0; i < it.total; ++i) {
-        const int s = ring.s;
-        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
-            if (lane == 0) {
-                atomicOr(&g_omni_err, 1u);
-                if (!drain(bars[warp], i, issued)) atomicOr(&g_omni_err, kDrainTimeoutBit);
-            }
-            return;                                      // no block barrier in this kernel
-        }
+    auto issue = [&](const Cursor& c, int s) {          // lane 0 only
+        omni_issue<Q, St>(it, c, s, tma::smem_addr(&bars[warp][s]), wsm, W, nullptr, CODES, BETA, GAMMA, ZB, ALPHA,
+                          out, n_in, Gr);
+    };
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_omni_err, 1u, issue,
+                                  [&](const Cursor& cc, int s) {
         const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -413,16 +399,8 @@ omni_stream_fwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
             }
         }
-        __syncwarp();
-        if (lane == 0 && issued < it.total) {
-            omni_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, nullptr, CODES, BETA, GAMMA, ZB, ALPHA,
-                           out, n_in, Gr);
-            ic.next(it.n_w);
-            ++issued;
-        }
-        ring.next();
-        cc.next(it.n_w);
-    }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
 }
 
 template <int Q, typename WT, int G_>
@@ -450,26 +428,12 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
         tma::bar_init_fence();
     }
     __syncwarp();
-    Cursor ic;
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            omni_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, GUP, CODES, BETA, GAMMA, ZB, ALPHA, out,
-                           n_in, Gr);
-            ic.next(it.n_w);
-        }
-    }
-    Ring<NST> ring;
-    Cursor cc;
-    for (long long i = 0; i < it.total; ++i) {
-        const int s = ring.s;
-        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
-            if (lane == 0) {
-                atomicOr(&g_omni_err, 1u);
-                if (!drain(bars[warp], i, issued)) atomicOr(&g_omni_err, kDrainTimeoutBit);
-            }
-            return;                                      // no block barrier in this kernel
-        }
+    auto issue = [&](const Cursor& c, int s) {          // lane 0 only
+        omni_issue<Q, St>(it, c, s, tma::smem_addr(&bars[warp][s]), wsm, W, GUP, CODES, BETA, GAMMA, ZB, ALPHA, out,
+                          n_in, Gr);
+    };
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_omni_err, 1u, issue,
+                                  [&](const Cursor& cc, int s) {
         const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -564,16 +528,8 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
                 for (int j = 0; j < Q; ++j) DALPHA[grp * Q + j] = dl * __fmaf_rn(2.f, sg[4 + j], -sg[2]);
             }
         }
-        __syncwarp();                                    // stage, tables and sums are free again
-        if (lane == 0 && issued < it.total) {
-            omni_issue<Q, St>(it, ic, s, tma::smem_addr(&bars[warp][s]), wsm, W, GUP, CODES, BETA, GAMMA, ZB, ALPHA, out,
-                           n_in, Gr);
-            ic.next(it.n_w);
-            ++issued;
-        }
-        ring.next();
-        cc.next(it.n_w);
-    }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
 }
 
 template <int Q, typename WT, int G_, int MODE>

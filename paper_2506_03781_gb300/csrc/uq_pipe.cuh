@@ -177,6 +177,49 @@ __device__ bool drain(unsigned long long (&bars)[NST], long long waited, long lo
     return true;
 }
 
+// The per-warp pipeline over a warp's work items, in Items/Cursor order:
+// lane 0 keeps the copies of NST items in flight -- issue(cursor, stage)
+// arms the stage's mbarrier and starts them -- and the warp waits (bounded)
+// for each item in turn, runs body(cursor, stage) on it and refills the
+// stage.  A wait that runs out sets `bit` in *flag, waits (bounded) for the
+// copies still in flight and returns false; for use in kernels without
+// block barriers.  Shared by the pipelined forwards and the OmniQuant and
+// AWQ backwards, which differ only in what they stage and compute.
+template <int NST, typename Issue, typename Body>
+__device__ __forceinline__ bool pipe_run(const Items& it, unsigned long long (&bars)[NST], int lane,
+                                         unsigned int* flag, unsigned int bit, Issue&& issue, Body&& body) {
+    Cursor ic;                                   // next item to issue (lane 0)
+    long long issued = 0;
+    if (lane == 0) {
+        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+            issue(ic, s);
+            ic.next(it.n_w);
+        }
+    }
+    Ring<NST> ring;
+    Cursor cc;                                   // item being computed
+    for (long long i = 0; i < it.total; ++i) {
+        const int s = ring.s;
+        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[s]), ring.parity))) {
+            if (lane == 0) {
+                atomicOr(flag, bit);
+                if (!drain(bars, i, issued)) atomicOr(flag, kDrainTimeoutBit);
+            }
+            return false;
+        }
+        body(static_cast<const Cursor&>(cc), s);
+        __syncwarp();                            // the stage is free again
+        if (lane == 0 && issued < it.total) {
+            issue(ic, s);
+            ic.next(it.n_w);
+            ++issued;
+        }
+        ring.next();
+        cc.next(it.n_w);
+    }
+    return true;
+}
+
 constexpr int kMaxDevices = 64;
 
 // Persistent grid: min(row blocks, SMs x resident blocks per SM).  The

@@ -267,26 +267,9 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
     };
-    Cursor ic;
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            issue(ic, s);
-            ic.next(it.n_w);
-        }
-    }
 
-    Ring<NST> ring;
-    Cursor cc;                                            // item being computed
-    for (long long i = 0; i < it.total; ++i) {
-        const int s = ring.s;
-        if (!__all_sync(kFull, tma::bar_wait(tma::smem_addr(&bars[warp][s]), ring.parity))) {
-            if (lane == 0) {
-                atomicOr(&g_stream_err, 1u);
-                if (!drain(bars[warp], i, issued)) atomicOr(&g_stream_err, kDrainTimeoutBit);
-            }
-            return;                                      // no block barrier in this kernel
-        }
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_stream_err, 1u, issue,
+                                  [&](const Cursor& cc, int s) {
         const int64_t row = it.row(cc.k);
         if (row < out) {
             const unsigned char* st = wsm + (size_t)s * St::BYTES;
@@ -351,15 +334,8 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
             }
         }
-        __syncwarp();
-        if (lane == 0 && issued < it.total) {
-            issue(ic, s);
-            ic.next(it.n_w);
-            ++issued;
-        }
-        ring.next();
-        cc.next(it.n_w);
-    }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
 }
 
 // ---------------------------------------------------------------------------
