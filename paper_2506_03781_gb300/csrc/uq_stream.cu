@@ -32,6 +32,9 @@ __device__ unsigned int g_stream_err = 0;
 #ifndef UQ_FWD_STAGE_BYTES
 #define UQ_FWD_STAGE_BYTES 5632
 #endif
+#ifndef UQ_KEEP_STAGE_BYTES
+#define UQ_KEEP_STAGE_BYTES 9728
+#endif
 #ifndef UQ_STREAM_BWD_MIN_BLOCKS
 #define UQ_STREAM_BWD_MIN_BLOCKS 2
 #endif
@@ -225,9 +228,10 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                   const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
                   const float* __restrict__ ZB, uint8_t* __restrict__ CODES, float* __restrict__ WHAT,
                   int64_t out, int n_in, int R, int n_rb) {
+    static_assert(MODE != FWD_KEEP, "the keep step runs keep_stream_kernel");
     constexpr int mode = MODE;
-    constexpr bool need_x = MODE != FWD_KEEP, need_c = MODE != FWD_FULL;
-    using St = Stage<Q, WT, G_, need_x, false, need_c, UQ_FWD_STAGE_BYTES>;
+    constexpr bool need_c = MODE != FWD_FULL;
+    using St = Stage<Q, WT, G_, true, false, need_c, UQ_FWD_STAGE_BYTES>;
     constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
@@ -257,10 +261,8 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
         const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
         tma::fence_async_smem();
         tma::bar_arrive_tx(bar, TX);
-        if constexpr (need_x) {
-            tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
-            tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
-        }
+        tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
+        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
         if constexpr (need_c) tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
         tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
         tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
@@ -293,7 +295,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 unit_sort<Q, NG, false>(t, lane);
             }
             const float dl = pd[sub], zu = pz[sub];
-            const float sr = need_x ? __ldg(SR + row) : 0.f;
+            const float sr = __ldg(SR + row);
             const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * UE;
             float srt[L];
             if constexpr (mode == FWD_FULL) {
@@ -307,13 +309,7 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 uint32_t nc = 0;
                 uint32_t cv = 0u;
                 if constexpr (need_c) cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
-                if constexpr (mode == FWD_KEEP) {
-#pragma unroll
-                    for (int kq = 0; kq < 4; ++kq) {
-                        const int c = (cv >> (8 * kq)) & (L - 1);
-                        o[kq] = __fmul_rn(dl, __fsub_rn(t.lv[sub][c], zu));
-                    }
-                } else {
+                {
                     float w[4], s4[4];
                     WT::unpack(*reinterpret_cast<const typename WT::raw*>(st + St::OFF_W + el * St::WBYTES), w);
                     f4_to(*reinterpret_cast<const float4*>(st + St::OFF_S + el * 4), s4);
@@ -332,6 +328,114 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     *reinterpret_cast<uint32_t*>(CODES + ebase + el) = nc;
                 }
                 *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
+            }
+        }
+                                  });
+    if (!ok) return;                                 // no block barrier in this kernel
+}
+
+// ---------------------------------------------------------------------------
+// Forward of the steps that keep the codes (M*_B off its remap step)
+// ---------------------------------------------------------------------------
+//
+// W^ = Delta (l(code) - z_U) reads only the code bytes and the group
+// parameters, so a work unit holds little data for the pipeline's per-item
+// cost (the copies lane 0 issues, the bounded wait, the level table).  A work
+// item here is KU adjacent units of one row: its codes (KU UE bytes) and the
+// parameters of its KU NG groups arrive in five bulk copies, and the warp
+// maps them with the lane layout of one unit, KU times.  The arithmetic per
+// element is that of fwd_stream_kernel's keep mode.
+
+// Largest number of groups in one keep item (bounds the per-warp level table).
+constexpr int kKeepMaxGroups = 16;
+
+template <int Q, int G_, int KU>
+struct KeepStage {
+    using U1 = Stage<Q, WBF16, G_, false, false, true, UQ_KEEP_STAGE_BYTES>;    // lane mapping of one unit
+    static constexpr int LPG = U1::LPG, NG = U1::NG, NV = U1::NV, UE = U1::UE;
+    static constexpr int NGK = KU * NG;                 // groups per item
+    static constexpr int SZ_C = KU * UE, SZ_P = NGK * 4, SZ_A = NGK * Q * 4;
+    static constexpr int OFF_C = 0, OFF_D = SZ_C, OFF_Z = OFF_D + SZ_P, OFF_B = OFF_Z + SZ_P, OFF_A = OFF_B + SZ_P;
+    static constexpr int BYTES = align_up(OFF_A + SZ_A, 128);
+    static constexpr uint32_t TX = SZ_C + 3 * SZ_P + SZ_A;
+    static constexpr int FIT = UQ_KEEP_STAGE_BYTES / BYTES;
+    static constexpr int NST = FIT < 2 ? 2 : (FIT > kMaxStages ? kMaxStages : FIT);
+    static constexpr int WARP_BYTES = NST * BYTES;
+    static_assert(NGK <= kKeepMaxGroups, "level table");
+    static_assert(SZ_C % 16 == 0 && SZ_P % 16 == 0 && SZ_A % 16 == 0, "bulk copy sizes must be multiples of 16");
+};
+
+template <int Q, int G_, int KU>
+__global__ void __launch_bounds__(kThreads, UQ_STREAM_FWD_MIN_BLOCKS)
+keep_stream_kernel(const float* __restrict__ DELTA, const float* __restrict__ ZU, const float* __restrict__ ALPHA,
+                   const float* __restrict__ ZB, const uint8_t* __restrict__ CODES, float* __restrict__ WHAT,
+                   int64_t out, int n_in, int R, int n_rb) {
+    using St = KeepStage<Q, G_, KU>;
+    constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NGK = St::NGK, NV = St::NV, UE = St::UE, NST = St::NST;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ __align__(8) unsigned long long bars[kWarps][NST];
+    __shared__ float lvs[kWarps][NGK][L];               // levels of the item's groups
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int sub = lane / LPG, li = lane % LPG;
+    const int Gr = n_in / G_;
+    const Items it(n_in / (KU * UE), R, n_rb, warp);
+    unsigned char* wsm = smem + (size_t)warp * St::WARP_BYTES;
+    float (*lv)[L] = lvs[warp];
+
+    if (lane == 0) {
+        for (int s = 0; s < NST; ++s) tma::bar_init(tma::smem_addr(&bars[warp][s]), 1);
+        tma::bar_init_fence();
+    }
+    __syncwarp();
+
+    auto issue = [&](const Cursor& c, int s) {           // lane 0 only
+        const uint32_t bar = tma::smem_addr(&bars[warp][s]);
+        const int64_t row = it.row(c.k);
+        if (row >= out) { tma::bar_arrive(bar); return; }
+        const int64_t e0 = row * n_in + (int64_t)it.unit(c.j) * (KU * UE);
+        const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * NGK;
+        const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+        tma::fence_async_smem();
+        tma::bar_arrive_tx(bar, St::TX);
+        tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
+        tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
+        tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+    };
+
+    const bool ok = pipe_run<NST>(it, bars[warp], lane, &g_stream_err, 1u, issue,
+                                  [&](const Cursor& cc, int s) {
+        const int64_t row = it.row(cc.k);
+        if (row < out) {
+            const unsigned char* st = wsm + (size_t)s * St::BYTES;
+            const float* pd = reinterpret_cast<const float*>(st + St::OFF_D);
+            const float* pz = reinterpret_cast<const float*>(st + St::OFF_Z);
+            const float* pb = reinterpret_cast<const float*>(st + St::OFF_B);
+            const float* pa = reinterpret_cast<const float*>(st + St::OFF_A);
+#pragma unroll
+            for (int e = lane; e < NGK * L; e += 32) {
+                const int kk = e / L, c = e % L;
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
+                lv[kk][c] = level_of<Q>(c, a, pb[kk]);
+            }
+            __syncwarp();
+            const int64_t ebase = row * n_in + (int64_t)it.unit(cc.j) * (KU * UE);
+#pragma unroll
+            for (int ku = 0; ku < KU; ++ku) {
+                const int gi = ku * NG + sub;
+                const float dl = pd[gi], zu = pz[gi];
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int el = ku * UE + sub * G_ + 4 * li + 4 * LPG * v;
+                    const uint32_t cv = *reinterpret_cast<const uint32_t*>(st + St::OFF_C + el);
+                    float o[4];
+#pragma unroll
+                    for (int kq = 0; kq < 4; ++kq) o[kq] = __fmul_rn(dl, __fsub_rn(lv[gi][(cv >> (8 * kq)) & (L - 1)], zu));
+                    *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
+                }
             }
         }
                                   });
@@ -385,25 +489,51 @@ static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, c
 template <int Q, typename WT, int G_, int MODE>
 static cudaError_t run_fwd_stream_mode(const Shape& sh, const void* W, uq_params p, uint8_t* codes, float* what,
                                        cudaStream_t st) {
-    using St = Stage<Q, WT, G_, MODE != FWD_KEEP, false, MODE != FWD_FULL, UQ_FWD_STAGE_BYTES>;
+    using St = Stage<Q, WT, G_, true, false, MODE != FWD_FULL, UQ_FWD_STAGE_BYTES>;
     const int U = sh.n_in / St::UE;
     const int R = rows_per_block(U);
     const int n_rb = (int)((sh.out + R - 1) / R);
     const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
     auto kern = fwd_stream_kernel<Q, WT, G_, MODE>;
     int grid = 0;
-    cudaError_t e = grid_for<Stage<Q, WT, G_, MODE != FWD_KEEP, false, MODE != FWD_FULL, UQ_FWD_STAGE_BYTES>>(
-        kern, dyn, n_rb, grid);
+    cudaError_t e = grid_for<St>(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R,
                                       n_rb);
     return cudaGetLastError();
 }
 
+template <int Q, int G_, int KU>
+static cudaError_t run_keep_stream(const Shape& sh, uq_params p, const uint8_t* codes, float* what, cudaStream_t st) {
+    using St = KeepStage<Q, G_, KU>;
+    const int U = sh.n_in / (KU * St::UE);
+    const int R = rows_per_block(U);
+    const int n_rb = (int)((sh.out + R - 1) / R);
+    const size_t dyn = (size_t)kWarps * St::WARP_BYTES;
+    auto kern = keep_stream_kernel<Q, G_, KU>;
+    int grid = 0;
+    cudaError_t e = grid_for<St>(kern, dyn, n_rb, grid);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, dyn, st>>>(p.delta, p.zu, p.alpha, p.zb, codes, what, sh.out, sh.n_in, R, n_rb);
+    return cudaGetLastError();
+}
+
+// Units per keep item: as many adjacent units (up to 4 and kKeepMaxGroups
+// groups) as divide a row's units.
+template <int Q, int G_>
+static cudaError_t keep_stream(const Shape& sh, uq_params p, const uint8_t* codes, float* what, cudaStream_t st) {
+    constexpr int UE = KeepStage<Q, G_, 1>::UE, NG = KeepStage<Q, G_, 1>::NG;
+    constexpr int KMAX = kKeepMaxGroups / NG >= 4 ? 4 : 2;     // NG is 4 or 8
+    const int U = sh.n_in / UE;
+    if (U % KMAX == 0) return run_keep_stream<Q, G_, KMAX>(sh, p, codes, what, st);
+    if (KMAX == 4 && U % 2 == 0) return run_keep_stream<Q, G_, 2>(sh, p, codes, what, st);
+    return run_keep_stream<Q, G_, 1>(sh, p, codes, what, st);
+}
+
 template <int Q, typename WT, int G_>
 static cudaError_t run_fwd_stream(const Shape& sh, const void* W, uq_params p, uint8_t* codes, int mode,
                                   float* what, cudaStream_t st) {
-    if (mode == FWD_KEEP) return run_fwd_stream_mode<Q, WT, G_, FWD_KEEP>(sh, W, p, codes, what, st);
+    if (mode == FWD_KEEP) return keep_stream<Q, G_>(sh, p, codes, what, st);
     if (mode == FWD_REMAP) return run_fwd_stream_mode<Q, WT, G_, FWD_REMAP>(sh, W, p, codes, what, st);
     return run_fwd_stream_mode<Q, WT, G_, FWD_FULL>(sh, W, p, codes, what, st);
 }

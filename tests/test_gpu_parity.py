@@ -304,6 +304,24 @@ def test_pipelined_and_plain_paths_agree_across_shapes(n_in, g):
     C.assert_grads_close(gr, ref, mass, f"n_in={n_in} g={g}")
 
 
+@pytest.mark.parametrize("n_in,g,q", [(4096, 128, 3), (2048, 128, 1), (3072, 128, 4), (1536, 128, 2),
+                                      (1024, 32, 4), (768, 32, 3), (2048, 64, 2), (1536, 64, 3)])
+def test_keep_step_items_of_several_units(n_in, g, q):
+    """The keep step's work items are 4, 2 or 1 adjacent units of a row (by
+    what divides the row's units): W^ = Delta (l(code) - z_U) bit-exact with
+    the oracle for each item width, with rows packed several to a block and a
+    ragged last block; the codes are untouched."""
+    out = 37
+    raw, W, P, codes0, _ = C.make_inputs(out, n_in, q, g, seed=7 * n_in + g + q)
+    what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 1, 2)
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 1, 2)
+    C.assert_fwd_equal(what, codes, r_what, r_codes, f"keep n_in={n_in} g={g} q={q}")
+    assert np.array_equal(codes, codes0)
+    api.uq_check_device()
+    assert api.uq_last_error() == ""
+
+
 def test_host_buffer_apis_match_the_oracle():
     """HostStep and HostPipeline (pinned host buffers in, results back on the
     host) give the oracle's results; two independent problems are submitted
