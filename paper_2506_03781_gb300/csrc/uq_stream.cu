@@ -64,8 +64,6 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ float2 tabs[kWarps][NG][L];          // (l(c), l(c) - z_U) per group slot and code word
-    __shared__ float tau_s[kWarps][NG];
-    __shared__ float eg_s[kWarps][NG];              // element-independent part of the filter margin
     __shared__ float red[kRowRing][kWarps];       // per row block and warp: sum of Delta S3
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
@@ -143,17 +141,21 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                     for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
                     const float lvc = level_of<Q>(c, a, pb[kk]);
                     t[kk][c] = make_float2(lvc, lvc - pz[kk]);
-                    if (c == 0) {
-                        float m = fabsf(a[0]);
-#pragma unroll
-                        for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
-                        tau_s[warp][kk] = m;
-                        const float kg = __fmul_rn(__fmul_rn(pd[kk], pd[kk]), sr);
-                        eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, kg);
-                    }
                 }
                 __syncwarp();
-                const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+                const float dl = pd[sub], zu = pz[sub];
+                // tau and the filter margin of the lane's own group, on every lane
+                // (no divergent branch, no shared-memory round trip)
+                float tau, eg;
+                {
+                    float a[Q];
+#pragma unroll
+                    for (int jj = 0; jj < Q; ++jj) a[jj] = pa[sub * Q + jj];
+                    tau = fabsf(a[0]);
+#pragma unroll
+                    for (int jj = 1; jj < Q; ++jj) tau = fminf(tau, fabsf(a[jj]));
+                    eg = bwd_margin(zu, pb[sub], a, Q, __fmul_rn(__fmul_rn(dl, dl), sr));
+                }
                 const float kds = __fmul_rn(__fmul_rn(dl, dl), sr);     // Delta / s = r kds, r = 1 / den
                 const int unit = it.unit(j);
                 const int64_t ebase = row * n_in + (int64_t)unit * UE;
@@ -175,15 +177,20 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 const float S = seg_slot2<LPG>(acc, lane);
                 if (SR8::writer(lane)) {
                     const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
+                    // one select chain and one store per slot instead of a branch per
+                    // output array (the lanes of a warp hold different slots)
 #pragma unroll
                     for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
                         const int slot = slot0 + q8;
                         const float tot = acc[q8];
-                        if (slot == 0) DDELTA[grp] = tot;
-                        else if (slot == 1) DZU[grp] = -(dl * tot);
-                        else if (slot == 2) DZB[grp] = dl * tot;
-                        else if (slot == 3) prow += dl * tot;
-                        else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * __fmaf_rn(2.f, tot, -S);
+                        const float dt = dl * tot;
+                        const float val = slot == 0 ? tot : slot == 1 ? -dt : slot == 2 ? dt : dl * __fmaf_rn(2.f, tot, -S);
+                        float* dst = slot == 0 ? DDELTA + grp
+                                     : slot == 1 ? DZU + grp
+                                     : slot == 2 ? DZB + grp
+                                     : DALPHA + grp * Q + (slot >= 4 ? slot - 4 : 0);
+                        prow = slot == 3 ? prow + dt : prow;
+                        if (slot != 3 && slot < 4 + Q) *dst = val;
                     }
                 }
             }
