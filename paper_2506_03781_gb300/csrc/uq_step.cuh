@@ -90,8 +90,6 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][2];
     __shared__ StepTab<Q, NG> tabs[kWarps];
-    __shared__ float tau_s[kWarps][NG];
-    __shared__ float eg_s[kWarps][NG];            // element-independent part of the filter margin
     __shared__ float red[2][kWarps];              // ds_r partials (Delta S3 sums) of row blocks k, k + 1
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -172,17 +170,20 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
                 for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
                 const float lvc = level_of<Q>(c, a, pb[kk]);
                 t.a[kk][c] = make_float2(lvc, lvc - pz[kk]);
-                if (c == 0) {
-                    float m = fabsf(a[0]);
-#pragma unroll
-                    for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
-                    tau_s[warp][kk] = m;
-                    const float kg = __fmul_rn(__fmul_rn(pd[kk], pd[kk]), sr);
-                    eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, kg);
-                }
             }
             __syncwarp();
-            const float dl = pd[sub], zu = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+            const float dl = pd[sub], zu = pz[sub];
+            // tau and the filter margin of the lane's own group, on every lane
+            float tau, eg;
+            {
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[sub * Q + jj];
+                tau = fabsf(a[0]);
+#pragma unroll
+                for (int jj = 1; jj < Q; ++jj) tau = fminf(tau, fabsf(a[jj]));
+                eg = bwd_margin(zu, pb[sub], a, Q, __fmul_rn(__fmul_rn(dl, dl), sr));
+            }
             const float kds = __fmul_rn(__fmul_rn(dl, dl), sr);         // Delta / s = r kds, r = 1 / den
             const int64_t ebase = row * n_in + (int64_t)unit * UE;
             float acc[8];
@@ -212,28 +213,25 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
             if (SR8::writer(lane)) {
                 const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
 #pragma unroll
+                // one select chain and one update per slot (the lanes of a warp hold
+                // different slots): slot 0 dDelta = tot, 1 dz_U = -(Delta tot),
+                // 2 dz_B = Delta tot, 3 Delta S3 of the group (ds_r), 4 + j
+                // dalpha_j = Delta (2 P_j - S)
+#pragma unroll
                 for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
                     const int slot = slot0 + q8;
                     const float tot = acc[q8];
-                    if (slot == 0) {                               // dDelta = tot
-                        const float v = __fsub_rn(dl, __fmul_rn(lr_f, tot));
-                        pd[sub] = v;
-                        DELTA[grp] = v;
-                    } else if (slot == 1) {                        // dz_U = -(Delta tot)
-                        const float v = __fsub_rn(zu, __fmul_rn(lr_f, -(dl * tot)));
-                        pz[sub] = v;
-                        ZU[grp] = v;
-                    } else if (slot == 2) {                        // dz_B = Delta tot
-                        const float v = __fsub_rn(pb[sub], __fmul_rn(lr_b, dl * tot));
-                        pb[sub] = v;
-                        ZB[grp] = v;
-                    } else if (slot == 3) {
-                        prow += dl * tot;                          // Delta S3 of the group
-                    } else if (slot - 4 < Q) {                     // dalpha_j = Delta (2 P_j - S)
-                        const int j = slot - 4;
-                        const float v = __fsub_rn(pa[sub * Q + j], __fmul_rn(lr_b, dl * __fmaf_rn(2.f, tot, -S)));
-                        pa[sub * Q + j] = v;
-                        ALPHA[grp * Q + j] = v;
+                    const float dt = dl * tot;
+                    const int j = slot >= 4 ? slot - 4 : 0;
+                    const float gr = slot == 0 ? tot : slot == 1 ? -dt : slot == 2 ? dt : dl * __fmaf_rn(2.f, tot, -S);
+                    const float lr = slot <= 1 ? lr_f : lr_b;
+                    float* sp_ = slot == 0 ? pd + sub : slot == 1 ? pz + sub : slot == 2 ? pb + sub : pa + sub * Q + j;
+                    float* gp = slot == 0 ? DELTA + grp : slot == 1 ? ZU + grp : slot == 2 ? ZB + grp : ALPHA + grp * Q + j;
+                    prow = slot == 3 ? prow + dt : prow;
+                    if (slot != 3 && slot < 4 + Q) {
+                        const float v = __fsub_rn(*sp_, __fmul_rn(lr, gr));
+                        *sp_ = v;
+                        *gp = v;
                     }
                 }
             }
