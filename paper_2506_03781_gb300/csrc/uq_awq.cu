@@ -486,8 +486,6 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ float2 tabs[kWarps][NG][L];          // (l(c), l(c) - z_A) per group slot and code word
-    __shared__ float tau_s[kWarps][NG];
-    __shared__ float eg_s[kWarps][NG];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
     const int U = n_in / UE, Gr = n_in / G_;
@@ -536,16 +534,20 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
                 for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
                 const float lvc = level_of<Q>(c, a, pb[kk]);
                 tabs[warp][kk][c] = make_float2(lvc, lvc - pz[kk]);
-                if (c == 0) {
-                    float m = fabsf(a[0]);
-#pragma unroll
-                    for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
-                    tau_s[warp][kk] = m;
-                    eg_s[warp][kk] = bwd_margin(pz[kk], pb[kk], a, Q, pd[kk]);
-                }
             }
             __syncwarp();
-            const float dl = pd[sub], za = pz[sub], tau = tau_s[warp][sub], eg = eg_s[warp][sub];
+            const float dl = pd[sub], za = pz[sub];
+            // tau and the filter margin of the lane's own group, on every lane
+            float tau, eg;
+            {
+                float a[Q];
+#pragma unroll
+                for (int jj = 0; jj < Q; ++jj) a[jj] = pa[sub * Q + jj];
+                tau = fabsf(a[0]);
+#pragma unroll
+                for (int jj = 1; jj < Q; ++jj) tau = fminf(tau, fabsf(a[jj]));
+                eg = bwd_margin(za, pb[sub], a, Q, dl);
+            }
             const float rdl = rcp_approx(dl);
             float acc[8];
 #pragma unroll
@@ -586,14 +588,18 @@ awq_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ SA, 
             const float S = seg_slot2<LPG>(acc, lane);
             if (SR8::writer(lane)) {
                 const int64_t grp = row * Gr + (int64_t)it.unit(cc.j) * NG + sub;
+                // one select chain and one store per slot (slot 3 is unused here)
 #pragma unroll
                 for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
                     const int slot = slot0 + q8;
                     const float tot = acc[q8];
-                    if (slot == 0) DDELTA[grp] = tot;
-                    else if (slot == 1) DZA[grp] = -(dl * tot);
-                    else if (slot == 2) DZB[grp] = dl * tot;
-                    else if (slot >= 4 && slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * __fmaf_rn(2.f, tot, -S);
+                    const float dt = dl * tot;
+                    const float val = slot == 0 ? tot : slot == 1 ? -dt : slot == 2 ? dt : dl * __fmaf_rn(2.f, tot, -S);
+                    float* dst = slot == 0 ? DDELTA + grp
+                                 : slot == 1 ? DZA + grp
+                                 : slot == 2 ? DZB + grp
+                                 : DALPHA + grp * Q + (slot >= 4 ? slot - 4 : 0);
+                    if (slot != 3 && slot < 4 + Q) *dst = val;
                 }
             }
         }

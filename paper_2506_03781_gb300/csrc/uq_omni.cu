@@ -415,7 +415,6 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ __align__(8) unsigned long long bars[kWarps][NST];
     __shared__ float lvs[kWarps][NG][L];
-    __shared__ float tau_s[kWarps][NG];
     __shared__ float sums[kWarps][NG][8];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / LPG, li = lane % LPG;
@@ -463,15 +462,12 @@ omni_stream_bwd_kernel(const void* __restrict__ W, const float* __restrict__ BET
 #pragma unroll
                 for (int jj = 0; jj < Q; ++jj) a[jj] = pa[kk * Q + jj];
                 lvs[warp][kk][c] = level_of<Q>(c, a, pb[kk]);
-                if (c == 0) {
-                    float m = fabsf(a[0]);
-#pragma unroll
-                    for (int jj = 1; jj < Q; ++jj) m = fminf(m, fabsf(a[jj]));
-                    tau_s[warp][kk] = m;
-                }
             }
             __syncwarp();
-            const float tau = tau_s[warp][sub];
+            // tau of the lane's own group, on every lane
+            float tau = fabsf(pa[sub * Q]);
+#pragma unroll
+            for (int jj = 1; jj < Q; ++jj) tau = fminf(tau, fabsf(pa[sub * Q + jj]));
             // x = w / Delta_O + z_O: one reciprocal of Delta_O per group, the
             // filter proven equal to the IEEE one (shared_div_filter4)
             const float rdl = rcp_approx(dl);
