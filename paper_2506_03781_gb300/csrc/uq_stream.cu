@@ -78,31 +78,49 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
     }
     __syncthreads();
 
-    auto issue = [&](const Cursor& c, int s) {           // lane 0 only
+    // The eight copies of a unit, one per lane 0..7: source base, bytes per
+    // element (per group for the parameters), size and stage offset, from a
+    // per-block table, so the lanes start their copies side by side.
+    __shared__ struct CopySpec {
+        const unsigned char* base;
+        uint32_t per, size, off, grp;
+    } cps[8];
+    if (threadIdx.x < 8) {
+        const int i = threadIdx.x;
+        const unsigned char* b[8] = {static_cast<const unsigned char*>(W), reinterpret_cast<const unsigned char*>(S),
+                                     reinterpret_cast<const unsigned char*>(GUP), CODES,
+                                     reinterpret_cast<const unsigned char*>(DELTA), reinterpret_cast<const unsigned char*>(ZU),
+                                     reinterpret_cast<const unsigned char*>(ZB), reinterpret_cast<const unsigned char*>(ALPHA)};
+        const uint32_t per[8] = {(uint32_t)St::WBYTES, 4u, 4u, 1u, 4u, 4u, 4u, 4u * Q};
+        const uint32_t size[8] = {St::SZ_W, St::SZ_S, St::SZ_G, St::SZ_C, St::SZ_P, St::SZ_P, St::SZ_P, St::SZ_A};
+        const uint32_t off[8] = {St::OFF_W, St::OFF_S, St::OFF_G, St::OFF_C, St::OFF_D, St::OFF_Z, St::OFF_B, St::OFF_A};
+        cps[i] = CopySpec{b[i], per[i], size[i], off[i], i >= 4 ? 1u : 0u};
+    }
+    __syncthreads();
+    // issued by the whole warp: lane 0 arms the stage's mbarrier with the
+    // unit's bytes, then lanes 0..7 each start one copy
+    auto issue = [&](const Cursor& c, int s) {
         const uint32_t bar = tma::smem_addr(&bars[warp][s]);
         const int64_t row = it.row(c.k);
-        if (row >= out) { tma::bar_arrive(bar); return; }
-        const int64_t e0 = row * n_in + (int64_t)it.unit(c.j) * UE;
-        const int64_t g0 = row * Gr + (int64_t)it.unit(c.j) * NG;
-        const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
-        tma::fence_async_smem();
-        tma::bar_arrive_tx(bar, TX);
-        tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
-        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
-        tma::copy_g2s(d + St::OFF_G, GUP + e0, St::SZ_G, bar);
-        tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
-        tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
-    };
-    Cursor ic;                                            // next item to issue
-    long long issued = 0;
-    if (lane == 0) {
-        for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
-            issue(ic, s);
-            ic.next(it.n_w);
+        if (row >= out) {
+            if (lane == 0) tma::bar_arrive(bar);
+            return;
         }
+        if (lane == 0) tma::bar_arrive_tx(bar, TX);
+        __syncwarp();
+        if (lane < 8) {
+            const CopySpec cp = cps[lane];
+            const int64_t idx = cp.grp ? row * Gr + (int64_t)it.unit(c.j) * NG : row * n_in + (int64_t)it.unit(c.j) * UE;
+            const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
+            tma::fence_async_smem();
+            tma::copy_g2s(d + cp.off, cp.base + idx * cp.per, cp.size, bar);
+        }
+    };
+    Cursor ic;                                            // next item to issue (every lane)
+    long long issued = 0;
+    for (int s = 0; s < NST && issued < it.total; ++s, ++issued) {
+        issue(ic, s);
+        ic.next(it.n_w);
     }
 
     bool alive = true;
@@ -195,7 +213,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 }
             }
             __syncwarp();                                // stage s and the tables are free again
-            if (alive && lane == 0 && issued < it.total) {
+            if (alive && issued < it.total) {
                 issue(ic, s);
                 ic.next(it.n_w);
                 ++issued;
