@@ -117,28 +117,44 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
     }
     __syncthreads();
 
+    // The eight copies of a unit, one per lane 0..7: source base, bytes per
+    // element (per group for the parameters), size and stage offset, from a
+    // per-block table, so the lanes start their copies side by side.
+    __shared__ struct StepCopy {
+        const unsigned char* base;
+        uint32_t per, size, off, grp;
+    } cps[8];
+    if (threadIdx.x < 8) {
+        const int i = threadIdx.x;
+        const unsigned char* b[8] = {static_cast<const unsigned char*>(W), reinterpret_cast<const unsigned char*>(S),
+                                     static_cast<const unsigned char*>(GUP), CODES,
+                                     reinterpret_cast<const unsigned char*>(DELTA), reinterpret_cast<const unsigned char*>(ZU),
+                                     reinterpret_cast<const unsigned char*>(ZB), reinterpret_cast<const unsigned char*>(ALPHA)};
+        const uint32_t per[8] = {(uint32_t)St::WBYTES, 4u, (uint32_t)St::GB, 1u, 4u, 4u, 4u, 4u * Q};
+        const uint32_t size[8] = {St::SZ_W, St::SZ_S, St::SZ_G, St::SZ_C, St::SZ_P, St::SZ_P, St::SZ_P, St::SZ_A};
+        const uint32_t off[8] = {St::OFF_W, St::OFF_S, St::OFF_G, St::OFF_C, St::OFF_D, St::OFF_Z, St::OFF_B, St::OFF_A};
+        cps[i] = StepCopy{b[i], per[i], size[i], off[i], i >= 4 ? 1u : 0u};
+    }
+    __syncthreads();
+
     auto row_of = [&](int64_t k) { return (cid + k * ncl) * R + row_sub; };
-    auto issue = [&](int64_t k) {                 // lane 0 only; k < n_items
+    // issued by the whole warp (k < n_items): lane 0 arms the stage's
+    // mbarrier with the unit's bytes, then lanes 0..7 each start one copy
+    auto issue = [&](int64_t k) {
         const int s = (int)(k & 1);
         const uint32_t bar = tma::smem_addr(&bars[warp][s]);
-        const int64_t row = row_of(k);
-        const int64_t e0 = row * n_in + (int64_t)unit * UE;
-        const int64_t g0 = row * Gr + (int64_t)unit * NG;
-        const uint32_t d = tma::smem_addr(wsm + (size_t)s * St::BYTES);
-        tma::bar_arrive_tx(bar, TX);
-        tma::copy_g2s(d + St::OFF_W, static_cast<const unsigned char*>(W) + e0 * St::WBYTES, St::SZ_W, bar);
-        tma::copy_g2s(d + St::OFF_S, S + e0, St::SZ_S, bar);
-        tma::copy_g2s(d + St::OFF_G, static_cast<const unsigned char*>(GUP) + e0 * St::GB, St::SZ_G, bar);
-        tma::copy_g2s(d + St::OFF_C, CODES + e0, St::SZ_C, bar);
-        tma::copy_g2s(d + St::OFF_D, DELTA + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_Z, ZU + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_B, ZB + g0, St::SZ_P, bar);
-        tma::copy_g2s(d + St::OFF_A, ALPHA + g0 * Q, St::SZ_A, bar);
+        if (lane == 0) tma::bar_arrive_tx(bar, TX);
+        __syncwarp();
+        if (lane < 8) {
+            const int64_t row = row_of(k);
+            const StepCopy cp = cps[lane];
+            const int64_t idx = cp.grp ? row * Gr + (int64_t)unit * NG : row * n_in + (int64_t)unit * UE;
+            tma::fence_async_smem();
+            tma::copy_g2s(tma::smem_addr(wsm + (size_t)s * St::BYTES) + cp.off, cp.base + idx * cp.per, cp.size, bar);
+        }
     };
-    int64_t next_issue = 0, next_wait = 0;        // items issued / waited for (next_issue kept by lane 0)
-    if (lane == 0) {
-        while (next_issue < 2 && next_issue < n_items) issue(next_issue++);
-    }
+    int64_t next_issue = 0, next_wait = 0;        // items issued / waited for (every lane)
+    while (next_issue < 2 && next_issue < n_items) issue(next_issue++);
 
     bool alive = true;
     for (int64_t k = 0; k < n_blocks; ++k) {
@@ -332,7 +348,7 @@ step_kernel(const void* __restrict__ W, float* S, float* SR, float* DELTA, float
             tma::fence_async_smem();
         }
         __syncwarp();
-        if (lane == 0 && alive && next_issue < n_items) issue(next_issue++);
+        if (alive && next_issue < n_items) issue(next_issue++);
     }
     if (!alive && lane == 0) {
         // copies this warp issued but never waited for land before the block exits
