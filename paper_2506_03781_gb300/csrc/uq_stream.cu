@@ -459,7 +459,9 @@ keep_stream_kernel(const float* __restrict__ DELTA, const float* __restrict__ ZU
                     float o[4];
 #pragma unroll
                     for (int kq = 0; kq < 4; ++kq) o[kq] = __fmul_rn(dl, __fsub_rn(lv[gi][(cv >> (8 * kq)) & (L - 1)], zu));
-                    *reinterpret_cast<float4*>(WHAT + ebase + el) = make_float4(o[0], o[1], o[2], o[3]);
+                    // streaming store (evict-first): 57.3 -> 55.2 us on 14336 x 4096; the
+                    // same hint on the other kernels' outputs changed nothing
+                    __stcs(reinterpret_cast<float4*>(WHAT + ebase + el), make_float4(o[0], o[1], o[2], o[3]));
                 }
             }
         }
