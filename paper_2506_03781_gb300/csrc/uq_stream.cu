@@ -42,6 +42,11 @@ __device__ unsigned int g_stream_err = 0;
 #define UQ_STREAM_FWD_MIN_BLOCKS 4
 #endif
 constexpr int kRowRing = 32;             // row blocks whose ds_r partials wait in shared memory
+// Rows of at least this many work units take the backward's branch-per-array
+// gradient stores: 526 vs 598 us on 8192 x 28672 (56 units per row), while
+// the select chain wins on shorter rows (145 vs 150 us on 14336 x 4096,
+// 511 vs 546 us on 28672 x 8192).
+constexpr int kBranchyUnits = 32;
 
 // ---------------------------------------------------------------------------
 // Backward
@@ -56,7 +61,7 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                   const float* __restrict__ ZB, const uint8_t* __restrict__ CODES, const float* __restrict__ GUP,
                   float* __restrict__ DS, float* __restrict__ DSR, float* __restrict__ DDELTA,
                   float* __restrict__ DZU, float* __restrict__ DZB, float* __restrict__ DALPHA, int64_t out,
-                  int n_in, int R, int n_rb) {
+                  int n_in, int R, int n_rb, int branchy) {
     using St = Stage<Q, WT, G_, true, true, true, UQ_BWD_STAGE_BYTES>;
     constexpr int L = 1 << Q, LPG = St::LPG, NG = St::NG, NV = St::NV, UE = St::UE, NST = St::NST;
     constexpr uint32_t TX = St::TX;
@@ -195,20 +200,35 @@ bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
                 const float S = seg_slot2<LPG>(acc, lane);
                 if (SR8::writer(lane)) {
                     const int64_t grp = row * Gr + (int64_t)unit * NG + sub;
-                    // one select chain and one store per slot instead of a branch per
-                    // output array (the lanes of a warp hold different slots)
+                    if (!branchy) {
+                        // one select chain and one store per slot instead of a branch per
+                        // output array (the lanes of a warp hold different slots)
 #pragma unroll
-                    for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
-                        const int slot = slot0 + q8;
-                        const float tot = acc[q8];
-                        const float dt = dl * tot;
-                        const float val = slot == 0 ? tot : slot == 1 ? -dt : slot == 2 ? dt : dl * __fmaf_rn(2.f, tot, -S);
-                        float* dst = slot == 0 ? DDELTA + grp
-                                     : slot == 1 ? DZU + grp
-                                     : slot == 2 ? DZB + grp
-                                     : DALPHA + grp * Q + (slot >= 4 ? slot - 4 : 0);
-                        prow = slot == 3 ? prow + dt : prow;
-                        if (slot != 3 && slot < 4 + Q) *dst = val;
+                        for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
+                            const int slot = slot0 + q8;
+                            const float tot = acc[q8];
+                            const float dt = dl * tot;
+                            const float val =
+                                slot == 0 ? tot : slot == 1 ? -dt : slot == 2 ? dt : dl * __fmaf_rn(2.f, tot, -S);
+                            float* dst = slot == 0 ? DDELTA + grp
+                                         : slot == 1 ? DZU + grp
+                                         : slot == 2 ? DZB + grp
+                                         : DALPHA + grp * Q + (slot >= 4 ? slot - 4 : 0);
+                            prow = slot == 3 ? prow + dt : prow;
+                            if (slot != 3 && slot < 4 + Q) *dst = val;
+                        }
+                    } else {
+                        // a branch per output array: measured faster on rows of many units
+#pragma unroll
+                        for (int q8 = 0; q8 < SR8::NOUT; ++q8) {
+                            const int slot = slot0 + q8;
+                            const float tot = acc[q8];
+                            if (slot == 0) DDELTA[grp] = tot;
+                            else if (slot == 1) DZU[grp] = -(dl * tot);
+                            else if (slot == 2) DZB[grp] = dl * tot;
+                            else if (slot == 3) prow += dl * tot;
+                            else if (slot - 4 < Q) DALPHA[grp * Q + (slot - 4)] = dl * __fmaf_rn(2.f, tot, -S);
+                        }
                     }
                 }
             }
@@ -509,7 +529,8 @@ static cudaError_t run_bwd_stream(const Shape& sh, const void* W, uq_params p, c
     cudaError_t e = grid_for<BwdTag<St, ELEM>>(kern, dyn, n_rb, grid);
     if (e != cudaSuccess) return e;
     kern<<<grid, kThreads, dyn, st>>>(W, p.s, p.sr, p.delta, p.zu, p.alpha, p.zb, codes, gup, gr.ds, gr.dsr,
-                                      gr.ddelta, gr.dzu, gr.dzb, gr.dalpha, sh.out, sh.n_in, R, n_rb);
+                                      gr.ddelta, gr.dzu, gr.dzb, gr.dalpha, sh.out, sh.n_in, R, n_rb,
+                                      U >= kBranchyUnits ? 1 : 0);
     return cudaGetLastError();
 }
 

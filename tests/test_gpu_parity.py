@@ -322,6 +322,24 @@ def test_keep_step_items_of_several_units(n_in, g, q):
     assert api.uq_last_error() == ""
 
 
+@pytest.mark.parametrize("n_in,g,q", [(512 * 36, 128, 3), (256 * 40, 32, 2), (512 * 33, 64, 4)])
+def test_backward_of_long_rows(n_in, g, q):
+    """Rows of 32 or more work units take the backward's branch-per-array
+    gradient stores (the launcher's choice by row length); their gradients
+    match the oracle like those of shorter rows, on a ragged row count."""
+    out = 13
+    raw, W, P, codes0, Gup = C.make_inputs(out, n_in, q, g, seed=n_in + q)
+    what, codes = C.gpu_fwd(raw, P, codes0, q, g, api.MAP_LOCAL_PERIODIC, 0, 2)
+    r_what, r_codes = O.quantize_fwd(W, P["s"], P["sr"], P["delta"], P["zu"], P["alpha"], P["zb"], codes0, g,
+                                     O.MAP_LOCAL_PERIODIC, 0, 2)
+    C.assert_fwd_equal(what, codes, r_what, r_codes, f"n_in={n_in} g={g}")
+    gr = C.gpu_bwd(raw, P, codes, Gup, q, g)
+    ref, mass = C.oracle_bwd(W, P, r_codes, Gup, g)
+    C.assert_grads_close(gr, ref, mass, f"n_in={n_in} g={g}")
+    api.uq_check_device()
+    assert api.uq_last_error() == ""
+
+
 def test_host_buffer_apis_match_the_oracle():
     """HostStep and HostPipeline (pinned host buffers in, results back on the
     host) give the oracle's results; two independent problems are submitted
