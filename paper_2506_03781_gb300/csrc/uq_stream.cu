@@ -3,11 +3,12 @@
 //
 // Each warp runs its own pipeline over its work units (NG whole groups =
 // UE contiguous elements of one row, the lane mapping of uq_common.cuh):
-// lane 0 issues one bulk copy (cp.async.bulk, completion counted on an
-// mbarrier) per input stream of a unit -- weights, s, dL/dW^, code words and
-// the unit's group parameters -- into one of NST shared-memory stages, and
-// the warp computes from shared memory while the copies of the next units
-// are in flight.  Thread blocks are persistent: block b handles row blocks
+// one bulk copy (cp.async.bulk, completion counted on an mbarrier) per input
+// stream of a unit -- weights, s, dL/dW^, code words and the unit's group
+// parameters -- goes into one of NST shared-memory stages (issued by lane 0
+// in the forwards, by lanes 0..7 side by side in the backward), and the warp
+// computes from shared memory while the copies of the next units are in
+// flight.  Thread blocks are persistent: block b handles row blocks
 // b, b + gridDim.x, ...; within a row block the warps split the row's units
 // as in the non-pipelined kernels.  Every mbarrier wait is bounded (about one second of
 // GPU clock); a wait that runs out sets g_stream_err, which
@@ -44,8 +45,8 @@ __device__ unsigned int g_stream_err = 0;
 constexpr int kRowRing = 32;             // row blocks whose ds_r partials wait in shared memory
 // Rows of at least this many work units take the backward's branch-per-array
 // gradient stores: 526 vs 598 us on 8192 x 28672 (56 units per row), while
-// the select chain wins on shorter rows (145 vs 150 us on 14336 x 4096,
-// 511 vs 546 us on 28672 x 8192).
+// the select chain wins on shorter rows (153 vs 160 us on 14336 x 4096,
+// 516 vs 546 us on 28672 x 8192).
 constexpr int kBranchyUnits = 32;
 
 // ---------------------------------------------------------------------------
@@ -54,6 +55,8 @@ constexpr int kBranchyUnits = 32;
 
 // ELEM: the whole-element filter (a filtered element drops out of every
 // gradient); otherwise the filter cuts the straight-through path only.
+// branchy (warp-uniform): write the group gradients with a branch per output
+// array instead of the select chain (the launcher's choice for long rows).
 template <int Q, typename WT, int G_, bool ELEM>
 __global__ void __launch_bounds__(kThreads, UQ_STREAM_BWD_MIN_BLOCKS)
 bwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const float* __restrict__ SR,
@@ -388,8 +391,8 @@ fwd_stream_kernel(const void* __restrict__ W, const float* __restrict__ S, const
 // cost (the copies lane 0 issues, the bounded wait, the level table).  A work
 // item here is KU adjacent units of one row: its codes (KU UE bytes) and the
 // parameters of its KU NG groups arrive in five bulk copies, and the warp
-// maps them with the lane layout of one unit, KU times.  The arithmetic per
-// element is that of fwd_stream_kernel's keep mode.
+// maps them with the lane layout of one unit, KU times.  Per element:
+// W^ = fl(Delta fl(l(c) - z_U)), l(c) = level_of(c) of the element's group.
 
 // Largest number of groups in one keep item (bounds the per-warp level table).
 constexpr int kKeepMaxGroups = 16;
