@@ -20,6 +20,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -141,10 +142,22 @@ def measured_peaks():
         return None
 
 
+def strip_comments(src):
+    """C/C++ source without its comments and with runs of whitespace
+    collapsed, so that edits to comments or layout keep the hash (string
+    literals hold no comment markers in these files)."""
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    return " ".join(src.split())
+
+
 def kernel_hash():
+    """Hash of the code (comments and layout ignored) of the backward's source
+    files: a recorded DRAM-traffic capture is used only for the code it was
+    taken on."""
     h = hashlib.sha256()
     for f in ("uq_stream.cu", "uq_common.cuh", "uq_pipe.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2506_03781_gb300", "csrc", f), "rb").read())
+        h.update(strip_comments(open(os.path.join(ROOT, "paper_2506_03781_gb300", "csrc", f)).read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -80,3 +80,16 @@ def test_clock_record_from_nvidia_smi_lines():
     assert bench.parse_clock_samples([]) == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
     # the query the sampler issues has exactly the fields the parser reads
     assert bench.ClockSampler.FIELDS.count(",") == 7
+
+
+def test_kernel_hash_ignores_comments_and_layout():
+    """The backward's traffic record is keyed by a hash of its code with the
+    comments and the layout removed: a comment or a re-indentation keeps the
+    key, a change of code does not."""
+    import bench
+    src = "int a = 1; // one\n/* block\n comment */ int  b =\n 2;"
+    assert bench.strip_comments(src) == "int a = 1; int b = 2;"
+    assert bench.strip_comments("x /* y */ z // w") == "x z"
+    assert bench.strip_comments("int a = 1;") != bench.strip_comments("int a = 2;")
+    h = bench.kernel_hash()
+    assert len(h) == 16 and h == bench.kernel_hash()
