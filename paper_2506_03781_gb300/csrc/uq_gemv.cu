@@ -583,6 +583,12 @@ bcq_gemv_wide_kernel(const __grid_constant__ CUtensorMap tm_planes, const __grid
         tma::bar_init_fence();
     }
     __syncwarp();
+    // Launched as a programmatic dependent of the previous kernel on the stream
+    // (the previous call's tile sum, which reads the partials this grid
+    // overwrites, or whatever produced the inputs): nothing global is read or
+    // written before that grid has completed.  Only the launch and the set-up
+    // above overlap it.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     const int total = batch * my_nb;                           // items: token-major, this warp's batches
     int issued = 0, waited = 0, ik = 0;
@@ -689,7 +695,9 @@ __global__ void __launch_bounds__(256)
 bcq_gemv_reduce_kernel(const float* __restrict__ PART, float* __restrict__ Y, int64_t n, int n_tiles) {
     // Launched as a programmatic dependent of the product kernel: it may start
     // while that kernel still runs, and waits here until the product grid has
-    // completed and its partials are visible.
+    // completed and its partials are visible.  The next product kernel on the
+    // stream may be scheduled once every block of this grid has started.
+    asm volatile("griddepcontrol.launch_dependents;");
     asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         float acc = 0.f;
@@ -981,8 +989,17 @@ static cudaError_t run_gemv_wide(const uint32_t* planes, const float* astar, con
         const int n_tiles = n_in / kWideCols;
         int64_t n_rb = 0, rpb = 0;
         gemv_row_blocks(out, n_tiles, per_sm, n_rb, rpb, (double)kWideLutRows);
-        kern<<<(unsigned)(n_rb * n_tiles), NW * 32, DYN, st>>>(mp, ma, mz, x, work, out, n_in, batch, n_tiles, rpb);
-        e = cudaGetLastError();
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.gridDim = dim3((unsigned)(n_rb * n_tiles));
+        cfg.blockDim = dim3(NW * 32);
+        cfg.dynamicSmemBytes = DYN;
+        cfg.stream = st;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, kern, mp, ma, mz, x, work, out, n_in, batch, n_tiles, rpb);
         if (e != cudaSuccess) return e;
         return gemv_reduce(work, y, (int64_t)batch * out, n_tiles, st);
     } else {
