@@ -396,22 +396,27 @@ uq_status uq_export_bcq_half(const void* W, uq_wdtype wdtype, int64_t out, int64
  * bitplanes [q, out, in/32] uint32, alpha_star [out, in/g, q] and
  * zb_star [out, in/g] fp32 as uq_export_bcq writes them; x [batch, in]
  * (xdtype fp32 or bf16), y [batch, out] fp32, both row-major.  The columns
- * are split into tiles of 512; each tile's contribution is formed from
+ * are split into tiles: 1024 columns (32 per lane) when in is a multiple of
+ * 1024 and g <= 256, else 512.  Each tile's contribution is formed from
  * per-8-column partial sums of x (one table lookup per plane byte) and
  * written to `workspace` (caller-owned device memory of at least
  * uq_bcq_gemv_workspace_bytes(out, in, batch) bytes, overwritten), then the
- * tiles are summed in order into y.  fp32 throughout, fixed order:
- * deterministic, and within a small multiple of the fp32 unit roundoff of
- * sum_i (sum_j |alpha*_j| + |z*|) |x_i| of the exact product.  Shapes as
- * uq_quantize_fwd, except that g must divide 512 or be a multiple of 512
- * (32, 64, 128, 256, 512, 1024, ...; any other g, e.g. 384 or 640, is
+ * tiles are summed in order into y.  fp32 throughout, fixed order for a
+ * given shape: deterministic, and within a small multiple of the fp32 unit
+ * roundoff of sum_i (sum_j |alpha*_j| + |z*|) |x_i| of the exact product
+ * (the two tilings add in different orders, both within that bound).
+ * Shapes as uq_quantize_fwd, except that g must divide 512 or be a multiple
+ * of 512 (32, 64, 128, 256, 512, 1024, ...; any other g, e.g. 384 or 640, is
  * UQ_ERR_UNSUPPORTED); 1 <= batch <= 64 (each token re-reads the planes).
- * When in is a multiple of 512 and g <= 128 the call also encodes three TMA
- * tensor maps on the host (through the runtime's driver entry point; stack
- * memory only, nothing is allocated) and the kernel stages its rows with
- * them; any other shape, or a driver without the encoder, takes per-thread
- * asynchronous copies.  Only the staging differs: both run the same
- * arithmetic in the same order.
+ * The 1024-column tiles, and the 512-column ones when in is a multiple of
+ * 512 and g <= 128, are staged with TMA tensor maps that the call encodes on
+ * the host (through the runtime's driver entry point; stack memory only,
+ * nothing is allocated); any other shape, or a driver without the encoder,
+ * takes per-thread asynchronous copies (same arithmetic as the 512-column
+ * tensor-map path).  The 1024-column product is launched as a programmatic
+ * dependent of the preceding work on the stream: it is scheduled early but
+ * reads and writes nothing before that work has completed, so stream order
+ * is kept.
  * Reads every input, writes y and the workspace.  A too small workspace is
  * UQ_ERR_ARG.
  */
